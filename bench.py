@@ -1,0 +1,300 @@
+"""Throughput benchmark of the AECCT batched decoder on GB300.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl {cuda,reference}] [--workload KEY]
+
+A step decodes one batch of the workload (default: Polar(64,32), d = 64, N = 6, 8 heads,
+B = 65,536 received words, BPSK/AWGN at Eb/N0 cycling over 4, 5, 6 dB) through the C ABI
+(aecct_decode).  Inputs are resident in HBM before the timed region; L2 is flushed between
+steps by writing a 256 MB buffer outside the timed events.  One JSON line is printed by
+rank 0.  Under torchrun each rank decodes its own batch (weak scaling, no collective on the
+data path); the time is the maximum over ranks.
+
+--impl reference times the CPU oracle (the plain C forward pass) on a bounded sample of
+the same workload on the host cores, and reports the same metric.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2410_05911_gb300 import inputs as I  # noqa: E402
+
+METRIC = "decoded codewords/s"
+UNIT = "codewords/s"
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return dict(hbm_gbs=p["hbm_gbs"], bf16_tflops=p["bf16_tflops"],
+                    bf16_tflops_sustained=p.get("bf16_tflops_sustained", p["bf16_tflops"]), source="measured")
+    return dict(hbm_gbs=6800.0, bf16_tflops=1900.0, bf16_tflops_sustained=1700.0, source="fallback")
+
+
+def work_per_word(w: I.Workload):
+    """Algorithmic work per decoded word: the paper's integer additions of the linear layers
+    ((2n-k) d^2 per d x d layer, App. A) counted as 2 ops per multiply-accumulate, 12 d^2 per
+    token per block; plus HBM bytes y in (4n), bits + syndrome out (n + n-k)."""
+    T, d, N = w.code.T, w.d, w.n_layers
+    return dict(int_ops=2 * 12 * T * d * d * N, io_bytes=4 * w.code.n + w.code.n + (w.code.n - w.code.k))
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons during the timed region."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                          "-i", str(self.gpu), "-lms", "100"], stdout=subprocess.PIPE,
+                                         stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if not self.lines:
+            return None
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx = max(mx, float(parts[1]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[4:8]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return dict(sm_mhz=float(np.median(sm)), sm_max_mhz=mx, reasons=sorted(reasons), samples=len(sm))
+
+
+def cpu_oracle_rate(model, y, budget_s: float = 12.0, chunk: int = 64, max_words: int = 8192):
+    """Oracle decode rate (words/s) on the host cores over a bounded prefix of y."""
+    from oracle import oracle as O
+
+    cores = os.cpu_count() or 1
+    done, t0 = 0, time.perf_counter()
+    while done < min(max_words, y.shape[0]):
+        O.decode(model, y[done:done + chunk], nthreads=cores)
+        done += chunk
+        if time.perf_counter() - t0 > budget_s:
+            break
+    dt = time.perf_counter() - t0
+    return done / dt, done, dt, cores
+
+
+def run_reference(args, rank, world):
+    w = I.workload(args.workload)
+    model = I.workload_model(args.workload)
+    if rank != 0:
+        return
+    chunk = max(16, w.code.T and 64)
+    ys = [I.channel_batch(w.code, 1024, e, seed=7 + i).y for i, e in enumerate(w.ebn0_db)]
+    per_step_budget = max(1.0, 60.0 / max(1, args.steps + args.warmup))
+    from oracle import oracle as O
+
+    cores = os.cpu_count() or 1
+    for s in range(args.warmup):
+        O.decode(model, ys[s % len(ys)][:16], nthreads=cores)
+    words, secs = 0, 0.0
+    for s in range(args.steps):
+        y = ys[s % len(ys)]
+        t0 = time.perf_counter()
+        done = 0
+        while done < y.shape[0]:
+            O.decode(model, y[done:done + chunk], nthreads=cores)
+            done += chunk
+            if time.perf_counter() - t0 > per_step_budget:
+                break
+        secs += time.perf_counter() - t0
+        words += done
+    value = words / secs
+    line = dict(metric=METRIC, value=value, unit=UNIT, n_gpus=world, steps=args.steps, warmup=args.warmup,
+                ms_per_step=1e3 * secs / args.steps, higher_is_better=True, scaling="weak", vs_baseline=None,
+                dtype="i8/f32", data="synthetic", impl="reference",
+                config=dict(workload=workload_label(w), batch=w.batch),
+                cpu_baseline=dict(value=value, unit=UNIT, cores=cores, kind="oracle",
+                                  sample=f"{words} words over {args.steps} steps, each a time-bounded prefix of a "
+                                         f"1024-word batch of the workload"),
+                e2e=dict(value=value, unit=UNIT, h2d_bytes_per_step=0, d2h_bytes_per_step=0))
+    print(json.dumps(line), flush=True)
+
+
+def workload_label(w: I.Workload) -> str:
+    return (f"{w.code.name} d={w.d} N={w.n_layers} heads=8 (4 first-ring/4 second-ring) T={w.code.T} "
+            f"B={w.batch} Eb/N0={'/'.join(str(e) for e in w.ebn0_db)} dB")
+
+
+def run_cuda(args, rank, world, local_rank):
+    import torch
+
+    from paper_2410_05911_gb300 import aecct
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    w = I.workload(args.workload)
+    model = I.workload_model(args.workload)
+    B = args.batch or w.batch
+    dec = aecct.Decoder(model)
+    q = dec.query()
+    # inputs: one batch per Eb/N0 point, resident on the device
+    ys_host = [I.channel_batch(w.code, B, e, seed=1000 * rank + 11 + i).y for i, e in enumerate(w.ebn0_db)]
+    ys = [torch.from_numpy(y).to(dev) for y in ys_host]
+    bits = torch.empty((B, w.code.n), dtype=torch.uint8, device=dev)
+    syn = torch.empty((B, w.code.n - w.code.k), dtype=torch.uint8, device=dev)
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(i):
+        dec.decode(ys[i % len(ys)], out=(bits, syn, None), stream=stream)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    if dec.synchronize() != aecct.AECCT_OK:
+        raise RuntimeError("warm-up decode failed")
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    torch.cuda.synchronize()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    with ClockSampler(local_rank) as clk:
+        time.sleep(0.3)
+        for i in range(args.steps):
+            flush.fill_(float(i))
+            evs[i][0].record(stream)
+            step(i)
+            evs[i][1].record(stream)
+        torch.cuda.synchronize()
+        time.sleep(0.2)
+    if world > 1:
+        dist.barrier()
+    if dec.synchronize() != aecct.AECCT_OK:
+        raise RuntimeError("timed decode reported an error")
+    ms = [a.elapsed_time(b) for a, b in evs]
+    total_s = sum(ms) / 1e3
+    if world > 1:
+        t = torch.tensor([total_s], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_s = float(t.item())
+    value = world * B * args.steps / total_s
+    kernel_s = total_s / args.steps
+
+    # end to end through the public host-buffer entry point: pinned y in, bits + syndrome out
+    y_pin = torch.from_numpy(ys_host[0]).pin_memory()
+    e2e_steps = max(3, min(args.steps, 20))
+    dec.decode_host(y_pin.numpy(), want_logits=False)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for i in range(e2e_steps):
+        dec.decode_host(y_pin.numpy(), want_logits=False)
+    e2e_s = (time.perf_counter() - t0) / e2e_steps
+    if world > 1:
+        t = torch.tensor([e2e_s], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+    e2e = dict(value=world * B / e2e_s, unit=UNIT, h2d_bytes_per_step=4 * B * w.code.n,
+               d2h_bytes_per_step=B * w.code.n + B * (w.code.n - w.code.k))
+
+    if rank != 0:
+        return
+    pk = peaks()
+    wk = work_per_word(w)
+    achieved_tops = wk["int_ops"] * B / kernel_s / 1e12
+    roof = dict(bound="tensor", achieved=achieved_tops, peak=pk["bf16_tflops"], unit="TFLOP/s",
+                frac=achieved_tops / pk["bf16_tflops"], traffic=args.traffic,
+                kernel=f"aecct_decoder_kernel<{w.d}>", work="2*12*T*d^2*N int ops per word (bf16 tensor cores, "
+                "exact integers); peak = measured bf16 dense burst")
+    cpu = None
+    if not args.no_cpu_baseline:
+        rate, words, secs, cores = cpu_oracle_rate(model, ys_host[0], budget_s=args.cpu_budget)
+        cpu = dict(value=rate, unit=UNIT, cores=cores, kind="oracle",
+                   sample=f"first {words} words of the {w.ebn0_db[0]} dB batch ({secs:.1f} s)")
+    line = dict(
+        metric=METRIC, value=value, unit=UNIT, n_gpus=world, steps=args.steps, warmup=args.warmup,
+        ms_per_step=1e3 * kernel_s, higher_is_better=True, scaling="weak", vs_baseline=None, dtype="i8/f32",
+        data="synthetic",
+        config=dict(workload=workload_label(w), batch=B, tokens=w.code.T, cluster_ctas=q["cluster_ctas"],
+                    words_per_group=q["words_per_group"], l2="flushed between steps (256 MB write)",
+                    info_gbit_s=value * w.code.k / 1e9, hbm_io_gbs=value * wk["io_bytes"] / 1e9),
+        e2e=e2e, roofline=roof, cpu_baseline=cpu, gpu_launches=args.steps, clocks=clk.summary())
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="cuda", choices=["cuda", "reference"])
+    ap.add_argument("--workload", default="polar64_32", choices=sorted(I.WORKLOADS))
+    ap.add_argument("--batch", type=int, default=0, help="override the batch size (0 = the workload's)")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--traffic", type=float, default=None, help="ncu DRAM bytes per launch, if measured")
+    args = ap.parse_args()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+
+        backend = "nccl" if args.impl == "cuda" else "gloo"
+        if backend == "nccl":
+            import torch
+            torch.cuda.set_device(local_rank)
+        dist.init_process_group(backend=backend)
+    try:
+        if args.impl == "reference":
+            run_reference(args, rank, world)
+        else:
+            run_cuda(args, rank, world, local_rank)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,179 @@
+/*
+ * aecct.h -- C ABI of the GB300 (sm_103a) AECCT decoder library (libaecct.so).
+ *
+ * The library runs the batched inference forward pass of the Accelerated Error
+ * Correction Code Transformer ("Accelerating Error Correction Code Transformers",
+ * Levy, Choukroun, Wolf): received words y (Sec. 3, "Problem Settings") go through
+ * the preprocessing h(y) = [|y|, 1 - 2 s(y)], a per-position embedding with the
+ * spectral positional encoding concatenated (Sec. 4.3), N Post-LN encoder blocks
+ * (Sec. 5) whose linear layers are AAP ternary-weight / int8-activation layers
+ * (Sec. 4.1, eqs. Quant and AAPLinear) and whose attention is head-partitioned
+ * (Sec. 4.2, HPSA), and the output head eps = W_o^T (W_{d->1} Phi) (Sec. 3, ECCT),
+ * followed by hard decisions x_hat = y * eps (Sec. 3).
+ *
+ * Conventions
+ *   - Every function returns an aecct_status (0 = success, negative = error).
+ *   - Pointers documented as HOST are read during the call only; the caller keeps
+ *     ownership.  Pointers documented as DEVICE must point to CUDA device memory of
+ *     the current device; the caller keeps ownership.
+ *   - The arithmetic is IEEE fp32 with one fixed order of operations (pairwise
+ *     feature-row sums, separately rounded multiply/add in the quantiser and
+ *     dequantiser, base-2 softmax with a degree-7 Taylor-series exp2, ascending key
+ *     order), so results are deterministic and do not depend on the batch size or
+ *     on how codewords are spread over the GPU.
+ *   - A handle serves one decode at a time; concurrent decodes need separate handles.
+ */
+#ifndef AECCT_H
+#define AECCT_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  AECCT_OK = 0,
+  AECCT_ERR_INVALID_ARG = -1,  /* a dimension, value or pointer argument is invalid */
+  AECCT_ERR_UNSUPPORTED = -2,  /* valid model outside the compiled kernel set (d, heads, T) */
+  AECCT_ERR_OUT_OF_MEMORY = -3,
+  AECCT_ERR_CUDA = -4,         /* a CUDA runtime call or kernel launch failed (see aecct_last_error) */
+  AECCT_ERR_TIMEOUT = -5,      /* a device-side wait exceeded its limit; the kernel stopped early */
+  AECCT_ERR_NO_DEVICE = -6     /* no sm_103 device is current */
+} aecct_status;
+
+typedef struct aecct_handle aecct_handle; /* opaque */
+
+/*
+ * Model description (inference form).  All pointers are HOST and are deep-copied by
+ * aecct_create.  T = 2n - k tokens (n variable nodes, then n-k check nodes), F = 4d.
+ *
+ *   n, k          code length and dimension (0 < k < n); H has n-k rows.
+ *   d             embedding width; this build supports d in {32, 64, 128}.
+ *   n_layers      N >= 1 encoder blocks.
+ *   heads         attention heads; this build supports heads == 8 (d_h = d/8).
+ *   h_first       number of first-ring heads (Sec. 4.2); heads [0, h_first) attend over
+ *                 the first-ring mask, heads [h_first, heads) over the second-ring mask.
+ *   d_spe         width of the SPE table (0 <= d_spe < d); the per-position embedding
+ *                 fills the first d - d_spe features (Sec. 4.3; Sec. 5 ablation text).
+ *   ffn_mult      feed-forward width multiplier; must be 4.
+ *   activation    0 = ReLU (Sec. 4 item 4).  Other values are rejected.
+ *   cluster_ctas  0 = choose automatically; otherwise the number of CTAs (1..8) that
+ *                 share one group of codewords (tuning knob).
+ *   H             [(n-k)][n] uint8 row-major, entries 0/1, no all-zero row or column.
+ *   emb           [T][d-d_spe] fp32: token t's embedding row, scaled by h_t (Sec. 3, ECCT).
+ *   spe           [T][d_spe] fp32: spectral positional encoding table (Sec. 4.3);
+ *                 may be NULL when d_spe == 0.
+ *   w_packed      ternary weights of all blocks, 2 bits each.  Per block, in this order:
+ *                 W_q [d][d], W_k [d][d], W_v [d][d], W_o [d][d], W_1 [F][d], W_2 [d][F]
+ *                 (row = output unit, d_out rows of d_in weights).  A row of d_in weights
+ *                 takes d_in/4 bytes; weight i sits in bits 2*(i%4)..2*(i%4)+1 of byte i/4,
+ *                 coded 00 = 0, 01 = +1, 11 = -1 (10 is invalid).  Total bytes:
+ *                 n_layers * 12 * d * d / 4.
+ *   w_scale       [n_layers][6] per-tensor scales gamma*delta (eq. Ternary), same order.
+ *   bias          per block d_q, d_k, d_v, d_o, F, d fp32 values (b_q b_k b_v b_o b_1 b_2).
+ *   ln_gamma      [n_layers][2][d] LayerNorm weights (after attention, after FFN).
+ *   ln_beta       [n_layers][2][d] LayerNorm biases.
+ *   w_d1, b_d1    [d] and scalar: the W_{d->1} projection and its bias.
+ *   w_out, b_out  [T][n] row-major and [n]: the W_o projection (T -> n) and its bias.
+ *   ln_eps        LayerNorm epsilon (added to the biased variance).
+ *   alpha_floor   lower bound on the absmax alpha of eq. Quant (an all-zero row maps to
+ *                 zero codes instead of dividing by zero).
+ *   wait_limit_cycles  0 = default (about 2^32 SM cycles); bound on every device-side
+ *                 wait, after which the kernel stops and decode reports AECCT_ERR_TIMEOUT.
+ */
+typedef struct {
+  int32_t n, k, d, n_layers, heads, h_first, d_spe, ffn_mult, activation, cluster_ctas;
+  const uint8_t *H;
+  const float *emb;
+  const float *spe;
+  const uint8_t *w_packed;
+  const float *w_scale;
+  const float *bias;
+  const float *ln_gamma;
+  const float *ln_beta;
+  const float *w_d1;
+  float b_d1;
+  const float *w_out;
+  const float *b_out;
+  float ln_eps;
+  float alpha_floor;
+  int64_t wait_limit_cycles;
+} aecct_model_desc;
+
+/* Validate the description, build the HPSA masks from H (Sec. 4.2: first ring = Tanner
+ * graph neighbours, second ring = nodes at distance two, plus the node itself), lay the
+ * weights out for the tensor cores and copy everything to the current device.  On
+ * success *out receives a new handle.  Errors: INVALID_ARG (bad dimension, H not 0/1,
+ * zero row/column in H, h_first > heads, d_spe >= d, packed code 10, NULL pointer),
+ * UNSUPPORTED (d, heads, ffn_mult or T outside this build), NO_DEVICE, OUT_OF_MEMORY, CUDA. */
+int aecct_create(const aecct_model_desc *desc, aecct_handle **out);
+
+/* Decode B received words.  y_dev: DEVICE fp32 [B][n] channel outputs y = x_s + noise
+ * (Sec. 3).  Outputs (DEVICE, written for every word):
+ *   bits_dev      uint8 [B][n]: decoded bits, 1 where y_j * eps_j < 0 (x_hat = y * eps);
+ *   syndrome_dev  uint8 [B][n-k] or NULL: H times the decoded bits over GF(2)
+ *                 (all zero iff the decoded word is a codeword);
+ *   logits_dev    fp32 [B][n] or NULL: the network output eps (multiplicative-noise
+ *                 prediction, Sec. 3).
+ * Runs asynchronously on cuda_stream (a cudaStream_t; NULL = legacy default stream).
+ * B == 0 is a no-op.  Errors: INVALID_ARG (B < 0, NULL y/bits with B > 0), CUDA,
+ * and TIMEOUT reported for an earlier decode on this handle whose kernel stopped. */
+int aecct_decode(aecct_handle *h, const float *y_dev, int64_t B, uint8_t *bits_dev, uint8_t *syndrome_dev,
+                 float *logits_dev, void *cuda_stream);
+
+/* Same as aecct_decode but with HOST buffers (pageable or pinned): copies y to the device,
+ * decodes, copies the outputs back and waits for completion.  Staging memory is owned by
+ * the handle and grows on demand. */
+int aecct_decode_host(aecct_handle *h, const float *y_host, int64_t B, uint8_t *bits_host, uint8_t *syndrome_host,
+                      float *logits_host, void *cuda_stream);
+
+/* Wait for the handle's last decode and report whether its kernel stopped on a
+ * device-side timeout (AECCT_ERR_TIMEOUT) or a CUDA error occurred. */
+int aecct_synchronize(aecct_handle *h);
+
+/* Record the integer core of the next decodes for words 0..cap_B-1 (cap_B = 0 stops).
+ * DEVICE buffers, caller-owned, T = 2n-k, W = 4d, gemm g: 0 = QKV (K = d, N = 3d,
+ * columns q|k|v), 1 = O (K = d, N = d), 2 = FFN1 (K = d, N = 4d), 3 = FFN2 (K = 4d, N = d):
+ *   q_dev      int8  [cap_B][n_layers][4][T][W]  Quant(x) codes of the GEMM input row (first K used)
+ *   acc_dev    int32 [cap_B][n_layers][4][T][W]  integer accumulators sum_i q_i t_oi (first N used)
+ *   alpha_dev  fp32  [cap_B][n_layers][4][T]     max(absmax, alpha_floor) of the input row
+ *   syn_dev    uint8 [cap_B][n-k]                syndrome s(y) of the channel output (Sec. 3)
+ * Any of the four may be NULL.  Unused entries are left untouched. */
+int aecct_set_capture(aecct_handle *h, int64_t cap_B, int8_t *q_dev, int32_t *acc_dev, float *alpha_dev,
+                      uint8_t *syn_dev);
+
+/* Launch facts of the handle (for benchmarks): CTAs per codeword group, codewords per
+ * group, the number of clusters a decode launches at most, threads per CTA, dynamic
+ * shared memory bytes per CTA, and TMEM columns per CTA.  Any pointer may be NULL. */
+int aecct_query(const aecct_handle *h, int32_t *cluster_ctas, int32_t *words_per_group, int32_t *max_clusters,
+                int32_t *threads_per_cta, int32_t *smem_bytes, int32_t *tmem_cols);
+
+int aecct_destroy(aecct_handle *h);
+
+/* Static description of a status code. */
+const char *aecct_status_string(int status);
+
+/* Text of the last CUDA error seen by this thread inside the library ("" if none). */
+const char *aecct_last_error(void);
+
+/*
+ * Diagnostics (no counterpart in the paper).
+ *
+ * aecct_selftest_mma: one CTA stages A [128][K] and B [N][K] (HOST int8 values, row-major,
+ * converted to bf16) in shared memory, multiplies them on the tensor cores
+ * (tcgen05.mma kind::f16, fp32 accumulators in tensor memory) and returns
+ * out_host [128][N] fp32 = A * B^T.  K in {16, 32, ..., 128}, N in {16, 32, ..., 256}.
+ *
+ * aecct_selftest_timeout: one warp waits on a shared-memory barrier that nothing
+ * completes, with a limit of limit_cycles; *status_host receives AECCT_ERR_TIMEOUT
+ * when the bounded wait gave up as designed (AECCT_OK would mean the barrier completed).
+ */
+int aecct_selftest_mma(const int8_t *a_host, const int8_t *b_host, int32_t K, int32_t N, float *out_host);
+int aecct_selftest_timeout(int64_t limit_cycles, int32_t *status_host);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* AECCT_H */

@@ -1,0 +1,267 @@
+"""Python binding of libaecct (the C ABI in include/aecct.h).
+
+Argument marshalling only: every step of the decoder runs in the CUDA library.  PyTorch
+provides device memory and streams.  There is no CPU fallback: if the library cannot be
+loaded, or no sm_103 GPU is present, the calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Tuple
+
+import numpy as np
+
+from . import build_lib
+
+AECCT_OK = 0
+AECCT_ERR_INVALID_ARG = -1
+AECCT_ERR_UNSUPPORTED = -2
+AECCT_ERR_OUT_OF_MEMORY = -3
+AECCT_ERR_CUDA = -4
+AECCT_ERR_TIMEOUT = -5
+AECCT_ERR_NO_DEVICE = -6
+
+EXPORTED_SYMBOLS = (
+    "aecct_create", "aecct_decode", "aecct_decode_host", "aecct_synchronize", "aecct_set_capture",
+    "aecct_query", "aecct_destroy", "aecct_status_string", "aecct_last_error", "aecct_selftest_mma",
+    "aecct_selftest_timeout",
+)
+
+
+class AecctError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        self.status = status
+        super().__init__(f"{what}: {status_string(status)} ({status}) {last_error()}".strip())
+
+
+class ModelDesc(ctypes.Structure):
+    _fields_ = [
+        ("n", ctypes.c_int32), ("k", ctypes.c_int32), ("d", ctypes.c_int32), ("n_layers", ctypes.c_int32),
+        ("heads", ctypes.c_int32), ("h_first", ctypes.c_int32), ("d_spe", ctypes.c_int32),
+        ("ffn_mult", ctypes.c_int32), ("activation", ctypes.c_int32), ("cluster_ctas", ctypes.c_int32),
+        ("H", ctypes.c_void_p), ("emb", ctypes.c_void_p), ("spe", ctypes.c_void_p), ("w_packed", ctypes.c_void_p),
+        ("w_scale", ctypes.c_void_p), ("bias", ctypes.c_void_p), ("ln_gamma", ctypes.c_void_p),
+        ("ln_beta", ctypes.c_void_p), ("w_d1", ctypes.c_void_p), ("b_d1", ctypes.c_float),
+        ("w_out", ctypes.c_void_p), ("b_out", ctypes.c_void_p), ("ln_eps", ctypes.c_float),
+        ("alpha_floor", ctypes.c_float), ("wait_limit_cycles", ctypes.c_int64),
+    ]
+
+
+_lib = None
+
+
+def library_path() -> str:
+    return build_lib.LIB_PATH
+
+
+def load(build_if_missing: bool = True):
+    """Load libaecct.so from the package's _build directory (building it if asked)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = build_lib.LIB_PATH
+    if not os.path.exists(path):
+        if not build_if_missing:
+            raise OSError(f"libaecct.so not built at {path}")
+        build_lib.build()
+    L = ctypes.CDLL(path)
+    P, I32, I64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
+    L.aecct_create.argtypes = [ctypes.POINTER(ModelDesc), ctypes.POINTER(P)]
+    L.aecct_decode.argtypes = [P, P, I64, P, P, P, P]
+    L.aecct_decode_host.argtypes = [P, P, I64, P, P, P, P]
+    L.aecct_synchronize.argtypes = [P]
+    L.aecct_set_capture.argtypes = [P, I64, P, P, P, P]
+    L.aecct_query.argtypes = [P] + [ctypes.POINTER(I32)] * 6
+    L.aecct_destroy.argtypes = [P]
+    L.aecct_status_string.argtypes = [ctypes.c_int]
+    L.aecct_status_string.restype = ctypes.c_char_p
+    L.aecct_last_error.argtypes = []
+    L.aecct_last_error.restype = ctypes.c_char_p
+    L.aecct_selftest_mma.argtypes = [P, P, I32, I32, P]
+    L.aecct_selftest_timeout.argtypes = [I64, ctypes.POINTER(I32)]
+    for name in EXPORTED_SYMBOLS:
+        fn = getattr(L, name)
+        if fn.restype is None or fn.restype is ctypes.c_int:
+            if name not in ("aecct_status_string", "aecct_last_error"):
+                fn.restype = ctypes.c_int
+    _lib = L
+    return L
+
+
+def status_string(status: int) -> str:
+    return load().aecct_status_string(int(status)).decode()
+
+
+def last_error() -> str:
+    return load().aecct_last_error().decode()
+
+
+def _check(status: int, what: str) -> None:
+    if status != AECCT_OK:
+        raise AecctError(status, what)
+
+
+def pack_ternary(t: np.ndarray) -> np.ndarray:
+    """Pack int8 ternary values [rows][cols] (cols % 4 == 0) into the 2-bit ABI format:
+    value i of a row goes to bits 2*(i%4) of byte i/4, coded 0 -> 00, +1 -> 01, -1 -> 11."""
+    t = np.asarray(t, dtype=np.int8)
+    rows, cols = t.shape
+    assert cols % 4 == 0
+    code = np.where(t == 1, 1, np.where(t == -1, 3, 0)).astype(np.uint8)
+    if not np.isin(t, (-1, 0, 1)).all():
+        raise ValueError("ternary weights must be in {-1, 0, 1}")
+    c = code.reshape(rows, cols // 4, 4)
+    return (c[..., 0] | (c[..., 1] << 2) | (c[..., 2] << 4) | (c[..., 3] << 6)).astype(np.uint8)
+
+
+class _HostModel:
+    """Contiguous host copies of a model's tensors, in the ABI layout (kept alive with the desc)."""
+
+    def __init__(self, model, cluster_ctas: int = 0, wait_limit_cycles: int = 0):
+        d, F = model.d, model.ffn_mult * model.d
+        self.H = np.ascontiguousarray(model.H, dtype=np.uint8)
+        self.emb = np.ascontiguousarray(model.emb, dtype=np.float32)
+        self.spe = np.ascontiguousarray(model.spe, dtype=np.float32)
+        packed = []
+        for layer in model.w_tern:
+            for t in layer:
+                packed.append(pack_ternary(t).ravel())
+        self.w_packed = np.ascontiguousarray(np.concatenate(packed) if packed else np.zeros(1, np.uint8))
+        self.w_scale = np.ascontiguousarray(model.w_scale, dtype=np.float32).reshape(-1)
+        self.bias = np.ascontiguousarray(
+            np.concatenate([np.asarray(b, np.float32).ravel() for layer in model.bias for b in layer]))
+        self.ln_gamma = np.ascontiguousarray(model.ln_gamma, dtype=np.float32).reshape(-1)
+        self.ln_beta = np.ascontiguousarray(model.ln_beta, dtype=np.float32).reshape(-1)
+        self.w_d1 = np.ascontiguousarray(model.w_d1, dtype=np.float32)
+        self.w_out = np.ascontiguousarray(model.w_out, dtype=np.float32)
+        self.b_out = np.ascontiguousarray(model.b_out, dtype=np.float32)
+        ptr = lambda a: a.ctypes.data if a.size else None  # noqa: E731
+        self.desc = ModelDesc(
+            model.n, model.k, model.d, model.n_layers, model.heads, model.h_first, model.d_spe, model.ffn_mult,
+            model.activation, int(cluster_ctas), ptr(self.H), ptr(self.emb), ptr(self.spe), ptr(self.w_packed),
+            ptr(self.w_scale), ptr(self.bias), ptr(self.ln_gamma), ptr(self.ln_beta), ptr(self.w_d1),
+            float(model.b_d1), ptr(self.w_out), ptr(self.b_out), float(model.ln_eps), float(model.alpha_floor),
+            int(wait_limit_cycles))
+
+
+def create_handle(model, cluster_ctas: int = 0, wait_limit_cycles: int = 0):
+    """aecct_create on a model (see inputs.ModelTensors); returns (status, handle or None)."""
+    L = load()
+    hm = _HostModel(model, cluster_ctas, wait_limit_cycles)
+    h = ctypes.c_void_p()
+    st = L.aecct_create(ctypes.byref(hm.desc), ctypes.byref(h))
+    return st, (h if st == AECCT_OK else None)
+
+
+class Decoder:
+    """A decoder handle on the current CUDA device.
+
+    decode(y) takes a float32 CUDA tensor [B, n] and returns (bits uint8 [B, n],
+    syndrome uint8 [B, n-k] or None, logits float32 [B, n] or None), computed on
+    torch.cuda.current_stream().
+    """
+
+    def __init__(self, model, cluster_ctas: int = 0, wait_limit_cycles: int = 0):
+        import torch
+
+        if not torch.cuda.is_available():
+            raise AecctError(AECCT_ERR_NO_DEVICE, "Decoder")
+        self._torch = torch
+        self.n, self.k = model.n, model.k
+        self.m = model.n - model.k
+        self.T = 2 * model.n - model.k
+        self.d, self.n_layers = model.d, model.n_layers
+        self._L = load()
+        st, h = create_handle(model, cluster_ctas, wait_limit_cycles)
+        _check(st, "aecct_create")
+        self._h = h
+        self._cap = None
+
+    def close(self) -> None:
+        if getattr(self, "_h", None) is not None:
+            self._L.aecct_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def query(self) -> dict:
+        vals = [ctypes.c_int32() for _ in range(6)]
+        _check(self._L.aecct_query(self._h, *[ctypes.byref(v) for v in vals]), "aecct_query")
+        keys = ("cluster_ctas", "words_per_group", "max_clusters", "threads_per_cta", "smem_bytes", "tmem_cols")
+        return {k: v.value for k, v in zip(keys, vals)}
+
+    def decode(self, y, want_syndrome: bool = True, want_logits: bool = True, out=None, stream=None):
+        torch = self._torch
+        if not (y.is_cuda and y.dtype == torch.float32 and y.dim() == 2 and y.shape[1] == self.n):
+            raise ValueError("y must be a float32 CUDA tensor of shape [B, n]")
+        y = y.contiguous()
+        B = y.shape[0]
+        if out is None:
+            bits = torch.empty((B, self.n), dtype=torch.uint8, device=y.device)
+            syn = torch.empty((B, self.m), dtype=torch.uint8, device=y.device) if want_syndrome else None
+            logits = torch.empty((B, self.n), dtype=torch.float32, device=y.device) if want_logits else None
+        else:
+            bits, syn, logits = out
+        s = stream if stream is not None else torch.cuda.current_stream(y.device)
+        st = self._L.aecct_decode(self._h, y.data_ptr(), B, bits.data_ptr(), syn.data_ptr() if syn is not None else None,
+                                  logits.data_ptr() if logits is not None else None, s.cuda_stream)
+        _check(st, "aecct_decode")
+        return bits, syn, logits
+
+    def decode_host(self, y: np.ndarray, want_syndrome: bool = True, want_logits: bool = True):
+        """End-to-end call with host arrays: copies in, decodes, copies out, waits."""
+        y = np.ascontiguousarray(y, dtype=np.float32)
+        B = y.shape[0]
+        bits = np.empty((B, self.n), np.uint8)
+        syn = np.empty((B, self.m), np.uint8) if want_syndrome else None
+        logits = np.empty((B, self.n), np.float32) if want_logits else None
+        st = self._L.aecct_decode_host(self._h, y.ctypes.data, B, bits.ctypes.data,
+                                       syn.ctypes.data if syn is not None else None,
+                                       logits.ctypes.data if logits is not None else None, None)
+        _check(st, "aecct_decode_host")
+        return bits, syn, logits
+
+    def synchronize(self) -> int:
+        return self._L.aecct_synchronize(self._h)
+
+    def set_capture(self, cap_B: int):
+        """Allocate capture buffers for the first cap_B words (0 disables); returns the tensors."""
+        torch = self._torch
+        if cap_B <= 0:
+            _check(self._L.aecct_set_capture(self._h, 0, None, None, None, None), "aecct_set_capture")
+            self._cap = None
+            return None
+        W = 4 * self.d
+        dev = torch.device("cuda", torch.cuda.current_device())
+        cap = dict(
+            q=torch.zeros((cap_B, self.n_layers, 4, self.T, W), dtype=torch.int8, device=dev),
+            acc=torch.zeros((cap_B, self.n_layers, 4, self.T, W), dtype=torch.int32, device=dev),
+            alpha=torch.zeros((cap_B, self.n_layers, 4, self.T), dtype=torch.float32, device=dev),
+            syn_in=torch.zeros((cap_B, self.m), dtype=torch.uint8, device=dev),
+        )
+        _check(self._L.aecct_set_capture(self._h, cap_B, cap["q"].data_ptr(), cap["acc"].data_ptr(),
+                                         cap["alpha"].data_ptr(), cap["syn_in"].data_ptr()), "aecct_set_capture")
+        self._cap = cap
+        return cap
+
+
+def selftest_mma(a: np.ndarray, b: np.ndarray) -> np.ndarray:
+    """tcgen05 MMA self-test: returns A [128, K] @ B[N, K]^T computed on the tensor cores."""
+    a = np.ascontiguousarray(a, dtype=np.int8)
+    b = np.ascontiguousarray(b, dtype=np.int8)
+    assert a.shape[0] == 128 and a.shape[1] == b.shape[1]
+    out = np.zeros((128, b.shape[0]), np.float32)
+    _check(load().aecct_selftest_mma(a.ctypes.data, b.ctypes.data, a.shape[1], b.shape[0], out.ctypes.data),
+           "aecct_selftest_mma")
+    return out
+
+
+def selftest_timeout(limit_cycles: int) -> int:
+    st = ctypes.c_int32(99)
+    _check(load().aecct_selftest_timeout(int(limit_cycles), ctypes.byref(st)), "aecct_selftest_timeout")
+    return st.value

@@ -1,0 +1,123 @@
+// aecct_internal.h -- parameters shared by the host side (api.cu) and the decoder kernel
+// (decoder_kernel.cu) of libaecct.  Not part of the public ABI.
+#pragma once
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <cstdint>
+
+namespace aecct {
+
+constexpr int kRows = 128;          // token rows per CTA: one M = 128 tensor-core tile
+constexpr int kHeads = 8;           // this build: 8 attention heads
+constexpr int kEpiWarps = 16;       // CUDA-core warps: 4 TMEM lane quadrants x 4 column slices
+constexpr int kEpiThreads = kEpiWarps * 32;
+constexpr int kProducerWarp = 16;   // issues the bulk copies of weight chunks
+constexpr int kMmaWarp = 17;        // allocates TMEM and issues tcgen05.mma
+constexpr int kThreads = 18 * 32;
+constexpr int kMaxCluster = 8;
+constexpr uint32_t kStageBytes = 16384;  // one weight chunk: <= 128 rows x 64 K bf16
+constexpr int kMaxChunks = 32;           // weight chunks per block (QKV, O, FFN1, FFN2)
+constexpr int kOutBitsBytes = 4096;      // decoded bits of the codewords one CTA finishes
+
+// One weight chunk of a block: rows [n0, n0 + nrows) and K columns [k0, k0 + kcols) of the
+// block's GEMM `gemm` (0 = QKV, 1 = O, 2 = FFN1, 3 = FFN2), stored as a K-major bf16 tile
+// of 8 x 16-byte core matrices at byte offset `off` of the block's weight stream.
+struct ChunkDesc {
+  uint32_t off;
+  uint32_t bytes;
+  uint16_t gemm, n0, nrows, k0, kcols, pad;
+};
+
+// Per-block parameter vector layout (floats), D = model width.
+struct LayerParamLayout {
+  __host__ __device__ static constexpr int bqkv(int) { return 0; }        // b_q | b_k | b_v  (3D)
+  __host__ __device__ static constexpr int bo(int D) { return 3 * D; }     // b_o (D)
+  __host__ __device__ static constexpr int b1(int D) { return 4 * D; }     // b_1 (4D)
+  __host__ __device__ static constexpr int b2(int D) { return 8 * D; }     // b_2 (D)
+  __host__ __device__ static constexpr int ln1g(int D) { return 9 * D; }
+  __host__ __device__ static constexpr int ln1b(int D) { return 10 * D; }
+  __host__ __device__ static constexpr int ln2g(int D) { return 11 * D; }
+  __host__ __device__ static constexpr int ln2b(int D) { return 12 * D; }
+  __host__ __device__ static constexpr int sw(int D) { return 13 * D; }    // 6 scales gamma*delta (+2 pad)
+  __host__ __device__ static constexpr int stride(int D) { return 13 * D + 8; }
+};
+
+struct DecodeParams {
+  // problem shape
+  int n, k, T, m, n_layers, h_first, d_spe;
+  int C;           // CTAs per cluster (they share one group of codewords)
+  int G;           // codewords per group
+  int n_clusters;  // clusters launched
+  int64_t B, n_groups;
+  // inputs / outputs (device)
+  const float *y;
+  uint8_t *bits;
+  uint8_t *syn;
+  float *logits;
+  // model (device)
+  const uint8_t *wstream;  // bf16 weight chunks, block after block
+  uint32_t layer_bytes;
+  int n_chunks;
+  ChunkDesc chunks[kMaxChunks];
+  const float *lparams;  // [n_layers][LayerParamLayout::stride(D)]
+  const float *emb;      // [T][D - d_spe]
+  const float *spe;      // [T][d_spe]
+  const float *w_d1;     // [D]
+  float b_d1;
+  const float *w_out;    // [T][n]
+  const float *b_out;    // [n]
+  const uint32_t *hrow_off;  // [m + 1] check i -> variables
+  const uint16_t *hrow_idx;
+  const uint32_t *mask_off[2];  // [T + 1] token -> neighbour tokens, ascending; 0 = first ring, 1 = second
+  const uint16_t *mask_idx[2];
+  float ln_eps, alpha_floor, att_scale;
+  // integer-core capture (device, optional)
+  int64_t cap_B;
+  int8_t *cap_q;
+  int32_t *cap_acc;
+  float *cap_alpha;
+  uint8_t *cap_syn;
+  // control
+  int *err;  // device word, bit 0 = a bounded wait timed out
+  long long wait_limit;
+};
+
+// Byte offset of element (r, c) in a K-major no-swizzle operand tile whose rows hold kdim
+// elements of 2 bytes: core matrix (r/8, c/8) is 128 contiguous bytes, core matrices along
+// K are adjacent (lbo = 128), 8-row groups are kdim/8 * 128 bytes apart (sbo).
+__host__ __device__ constexpr inline uint32_t core_off(uint32_t r, uint32_t c, uint32_t kdim) {
+  return (r >> 3) * (kdim >> 3) * 128u + (c >> 3) * 128u + (r & 7u) * 16u + (c & 7u) * 2u;
+}
+
+template <int D>
+struct SmemLayout {
+  static constexpr uint32_t kKvStride = 8u * D + 16u;  // token row: 8 heads x (K | V) x d_h fp32, + 16 B pad
+  static constexpr uint32_t kKvBytes = kRows * kKvStride;
+  static constexpr uint32_t kUqBytes = kRows * 4u * D * 2u;  // FFN2 operand: 128 x 4D bf16
+  __host__ __device__ static constexpr uint32_t align1k(uint32_t v) { return (v + 1023u) & ~1023u; }
+  static constexpr uint32_t kRegionU = align1k(kKvBytes > kUqBytes ? kKvBytes : kUqBytes);
+  static constexpr uint32_t kAopBytes = kRows * D * 2u;  // QKV / O / FFN1 operand: 128 x D bf16
+  static constexpr int kStages = (D == 128) ? 3 : 4;
+  static constexpr uint32_t kOffU = 0;
+  static constexpr uint32_t kOffAop = kRegionU;
+  static constexpr uint32_t kOffW = align1k(kOffAop + kAopBytes);
+  static constexpr uint32_t kOffRed = kOffW + kStages * kStageBytes;  // 2 x 4 x 128 floats
+  static constexpr uint32_t kOffZ = kOffRed + 4096;                   // 128 floats
+  static constexpr uint32_t kOffObits = kOffZ + 512;                  // decoded bits
+  static constexpr uint32_t kOffBar = kOffObits + kOutBitsBytes;      // mbarriers
+  static constexpr uint32_t kOffMisc = kOffBar + 256;                 // tmem base, abort flag, peer bases
+  static constexpr uint32_t kTotal = kOffMisc + 128;
+  static constexpr uint32_t kTmemCols = 4u * D;
+};
+
+// decoder_kernel.cu
+template <int D>
+cudaError_t launch_decode(const DecodeParams &p, cudaStream_t stream);
+template <int D>
+cudaError_t prepare_decode_kernel(int cluster_ctas, int *max_active_clusters);
+
+// api.cu diagnostics kernels live in selftest.cu
+cudaError_t run_selftest_mma(const int8_t *a_host, const int8_t *b_host, int K, int N, float *out_host);
+cudaError_t run_selftest_timeout(long long limit_cycles, int *status_host);
+
+}  // namespace aecct

@@ -1,0 +1,508 @@
+// api.cu -- host side of libaecct's C ABI (include/aecct.h).
+//
+// aecct_create validates the model description, builds the HPSA neighbour lists from H
+// (Sec. 4.2), unpacks the 2-bit ternary weights into bf16 tensor-core tiles, picks how many
+// CTAs share a group of codewords, and copies everything to the device once.  aecct_decode
+// launches the fused decoder kernel (decoder_kernel.cu) on the caller's stream.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdlib>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "../../include/aecct.h"
+#include "aecct_internal.h"
+
+using namespace aecct;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+int cuda_fail(cudaError_t e, const char *what) {
+  g_last_error = std::string(what) + ": " + cudaGetErrorString(e);
+  return AECCT_ERR_CUDA;
+}
+
+}  // namespace
+
+struct aecct_handle {
+  int n = 0, k = 0, T = 0, m = 0, d = 0, n_layers = 0, h_first = 0, d_spe = 0;
+  int C = 1, G = 1, max_clusters = 0;
+  float ln_eps = 0, alpha_floor = 0, att_scale = 0, b_d1 = 0;
+  long long wait_limit = 0;
+  int device = 0;
+  std::vector<void *> allocs;
+  uint8_t *wstream = nullptr;
+  uint32_t layer_bytes = 0;
+  int n_chunks = 0;
+  ChunkDesc chunks[kMaxChunks] = {};
+  float *lparams = nullptr, *emb = nullptr, *spe = nullptr, *w_d1 = nullptr, *w_out = nullptr, *b_out = nullptr;
+  uint32_t *hrow_off = nullptr, *mask_off[2] = {nullptr, nullptr};
+  uint16_t *hrow_idx = nullptr, *mask_idx[2] = {nullptr, nullptr};
+  int *d_err = nullptr;
+  int *h_err = nullptr;  // pinned
+  cudaEvent_t ev = nullptr;
+  bool ev_pending = false;
+  int pending_status = AECCT_OK;
+  // capture
+  int64_t cap_B = 0;
+  int8_t *cap_q = nullptr;
+  int32_t *cap_acc = nullptr;
+  float *cap_alpha = nullptr;
+  uint8_t *cap_syn = nullptr;
+  // host-buffer staging
+  int64_t stage_B = 0;
+  float *st_y = nullptr, *st_logits = nullptr;
+  uint8_t *st_bits = nullptr, *st_syn = nullptr;
+};
+
+namespace {
+
+template <typename T>
+int dev_upload(aecct_handle *h, T **dst, const T *src, size_t count) {
+  void *p = nullptr;
+  const size_t bytes = sizeof(T) * (count ? count : 1);
+  cudaError_t e = cudaMalloc(&p, bytes);
+  if (e != cudaSuccess) return e == cudaErrorMemoryAllocation ? AECCT_ERR_OUT_OF_MEMORY : cuda_fail(e, "cudaMalloc");
+  h->allocs.push_back(p);
+  if (count && src) {
+    e = cudaMemcpy(p, src, sizeof(T) * count, cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpy");
+  }
+  *dst = static_cast<T *>(p);
+  return AECCT_OK;
+}
+
+void free_handle(aecct_handle *h) {
+  if (!h) return;
+  for (void *p : h->allocs) cudaFree(p);
+  cudaFree(h->st_y);
+  cudaFree(h->st_logits);
+  cudaFree(h->st_bits);
+  cudaFree(h->st_syn);
+  if (h->h_err) cudaFreeHost(h->h_err);
+  if (h->ev) cudaEventDestroy(h->ev);
+  delete h;
+}
+
+uint16_t f2bf_bits(float f) {
+  // exact for the integers -1, 0, 1
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  return static_cast<uint16_t>(u >> 16);
+}
+
+int validate(const aecct_model_desc *d) {
+  if (!d) return AECCT_ERR_INVALID_ARG;
+  if (d->n <= 0 || d->k <= 0 || d->k >= d->n) return AECCT_ERR_INVALID_ARG;
+  if (d->d <= 0 || d->heads <= 0 || d->d % d->heads != 0) return AECCT_ERR_INVALID_ARG;
+  if (d->n_layers < 1 || d->n_layers > 4096) return AECCT_ERR_INVALID_ARG;
+  if (d->h_first < 0 || d->h_first > d->heads) return AECCT_ERR_INVALID_ARG;
+  if (d->d_spe < 0 || d->d_spe >= d->d) return AECCT_ERR_INVALID_ARG;
+  if (d->ffn_mult <= 0) return AECCT_ERR_INVALID_ARG;
+  if (d->activation < 0 || d->activation > 1) return AECCT_ERR_INVALID_ARG;
+  if (d->cluster_ctas < 0 || d->cluster_ctas > 64) return AECCT_ERR_INVALID_ARG;
+  if (!d->H || !d->emb || !d->w_packed || !d->w_scale || !d->bias || !d->ln_gamma || !d->ln_beta || !d->w_d1 ||
+      !d->w_out || !d->b_out)
+    return AECCT_ERR_INVALID_ARG;
+  if (d->d_spe > 0 && !d->spe) return AECCT_ERR_INVALID_ARG;
+  if (!(d->ln_eps >= 0.0f) || !std::isfinite(d->ln_eps)) return AECCT_ERR_INVALID_ARG;
+  if (!(d->alpha_floor > 0.0f) || !std::isfinite(d->alpha_floor)) return AECCT_ERR_INVALID_ARG;
+  if (d->wait_limit_cycles < 0) return AECCT_ERR_INVALID_ARG;
+  const int n = d->n, m = d->n - d->k;
+  for (int i = 0; i < m; ++i) {
+    int row = 0;
+    for (int j = 0; j < n; ++j) {
+      const uint8_t v = d->H[(size_t)i * n + j];
+      if (v > 1) return AECCT_ERR_INVALID_ARG;
+      row += v;
+    }
+    if (row == 0) return AECCT_ERR_INVALID_ARG;
+  }
+  for (int j = 0; j < n; ++j) {
+    int col = 0;
+    for (int i = 0; i < m; ++i) col += d->H[(size_t)i * n + j];
+    if (col == 0) return AECCT_ERR_INVALID_ARG;
+  }
+  // shape limits of this build
+  if (d->heads != kHeads) return AECCT_ERR_UNSUPPORTED;
+  if (d->d != 32 && d->d != 64 && d->d != 128) return AECCT_ERR_UNSUPPORTED;
+  if (d->ffn_mult != 4 || d->activation != 0) return AECCT_ERR_UNSUPPORTED;
+  const int T = 2 * n - d->k;
+  if (T > kMaxCluster * kRows || T > 65535) return AECCT_ERR_UNSUPPORTED;
+  // packed weights: no code 10
+  const size_t nbytes = (size_t)d->n_layers * 12u * d->d * d->d / 4u;
+  for (size_t i = 0; i < nbytes; ++i) {
+    const uint8_t b = d->w_packed[i];
+    for (int s = 0; s < 4; ++s)
+      if (((b >> (2 * s)) & 3u) == 2u) return AECCT_ERR_INVALID_ARG;
+  }
+  return AECCT_OK;
+}
+
+// 2-bit code -> ternary value
+inline int8_t tern(uint8_t code) { return code == 1 ? 1 : (code == 3 ? -1 : 0); }
+
+struct Gemm {
+  int N, K;
+};
+
+}  // namespace
+
+extern "C" {
+
+const char *aecct_status_string(int status) {
+  switch (status) {
+    case AECCT_OK: return "ok";
+    case AECCT_ERR_INVALID_ARG: return "invalid argument";
+    case AECCT_ERR_UNSUPPORTED: return "unsupported model shape for this build";
+    case AECCT_ERR_OUT_OF_MEMORY: return "out of device memory";
+    case AECCT_ERR_CUDA: return "CUDA error";
+    case AECCT_ERR_TIMEOUT: return "device-side wait timed out";
+    case AECCT_ERR_NO_DEVICE: return "no sm_103 device";
+    default: return "unknown status";
+  }
+}
+
+const char *aecct_last_error(void) { return g_last_error.c_str(); }
+
+int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
+  if (!out) return AECCT_ERR_INVALID_ARG;
+  *out = nullptr;
+  int rc = validate(desc);
+  if (rc) return rc;
+  const aecct_model_desc &d = *desc;
+  const int n = d.n, k = d.k, m = n - k, T = 2 * n - k, D = d.d, F = 4 * D;
+
+  // choose the number of CTAs that share a group: densest packing of T-token words over C x 128 rows
+  int best_C = 0, best_G = 0;
+  double best_eff = -1.0;
+  const int cmin = (T + kRows - 1) / kRows;
+  for (int C = cmin; C <= kMaxCluster; ++C) {
+    if (d.cluster_ctas && C != d.cluster_ctas) continue;
+    const int G = (C * kRows) / T;
+    if (G < 1) continue;
+    if (((G + C - 1) / C) * n > kOutBitsBytes) continue;
+    const double eff = static_cast<double>(G * T) / (C * kRows);
+    if (eff > best_eff + 1e-9) best_eff = eff, best_C = C, best_G = G;
+  }
+  if (!best_C) return d.cluster_ctas ? AECCT_ERR_INVALID_ARG : AECCT_ERR_UNSUPPORTED;
+
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return AECCT_ERR_NO_DEVICE;
+  cudaDeviceProp prop;
+  e = cudaGetDeviceProperties(&prop, dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDeviceProperties");
+  if (prop.major != 10) {
+    g_last_error = "device is not compute capability 10.x";
+    return AECCT_ERR_NO_DEVICE;
+  }
+  int max_clusters = 0;
+  if (D == 32) e = prepare_decode_kernel<32>(best_C, &max_clusters);
+  else if (D == 64) e = prepare_decode_kernel<64>(best_C, &max_clusters);
+  else e = prepare_decode_kernel<128>(best_C, &max_clusters);
+  if (e != cudaSuccess) return cuda_fail(e, "kernel occupancy");
+  if (max_clusters < 1) {
+    g_last_error = "no cluster of this size fits on the device";
+    return AECCT_ERR_UNSUPPORTED;
+  }
+
+  aecct_handle *h = new aecct_handle();
+  h->n = n, h->k = k, h->T = T, h->m = m, h->d = D, h->n_layers = d.n_layers, h->h_first = d.h_first;
+  h->d_spe = d.d_spe, h->C = best_C, h->G = best_G, h->max_clusters = max_clusters;
+  h->ln_eps = d.ln_eps, h->alpha_floor = d.alpha_floor, h->b_d1 = d.b_d1, h->device = dev;
+  h->att_scale = static_cast<float>(1.4426950408889634074 / std::sqrt(static_cast<double>(D / kHeads)));
+  h->wait_limit = d.wait_limit_cycles ? d.wait_limit_cycles : (1LL << 32);
+
+  // ---- H rows (check -> variables) for the syndromes
+  std::vector<uint32_t> hoff(m + 1, 0);
+  std::vector<uint16_t> hidx;
+  for (int i = 0; i < m; ++i) {
+    for (int j = 0; j < n; ++j)
+      if (d.H[(size_t)i * n + j]) hidx.push_back(static_cast<uint16_t>(j));
+    hoff[i + 1] = static_cast<uint32_t>(hidx.size());
+  }
+  // ---- HPSA neighbour lists (Sec. 4.2): token t < n is variable t, token n + i is check i
+  std::vector<uint32_t> moff[2];
+  std::vector<uint16_t> midx[2];
+  for (int mk = 0; mk < 2; ++mk) moff[mk].assign(T + 1, 0);
+  std::vector<uint8_t> row(T);
+  for (int t = 0; t < T; ++t) {
+    // first ring: Tanner-graph neighbours
+    std::fill(row.begin(), row.end(), 0);
+    if (t < n) {
+      for (int i = 0; i < m; ++i)
+        if (d.H[(size_t)i * n + t]) row[n + i] = 1;
+    } else {
+      for (int j = 0; j < n; ++j)
+        if (d.H[(size_t)(t - n) * n + j]) row[j] = 1;
+    }
+    for (int u = 0; u < T; ++u)
+      if (row[u]) midx[0].push_back(static_cast<uint16_t>(u));
+    moff[0][t + 1] = static_cast<uint32_t>(midx[0].size());
+    // second ring: same-type nodes at distance two, and the node itself
+    std::fill(row.begin(), row.end(), 0);
+    if (t < n) {
+      for (int i = 0; i < m; ++i)
+        if (d.H[(size_t)i * n + t])
+          for (int j = 0; j < n; ++j)
+            if (d.H[(size_t)i * n + j]) row[j] = 1;
+    } else {
+      const int i0 = t - n;
+      for (int j = 0; j < n; ++j)
+        if (d.H[(size_t)i0 * n + j])
+          for (int i = 0; i < m; ++i)
+            if (d.H[(size_t)i * n + j]) row[n + i] = 1;
+    }
+    for (int u = 0; u < T; ++u)
+      if (row[u]) midx[1].push_back(static_cast<uint16_t>(u));
+    moff[1][t + 1] = static_cast<uint32_t>(midx[1].size());
+  }
+
+  // ---- weights: 2-bit codes -> bf16 K-major core-matrix chunks, in the order the MMA consumes them
+  const Gemm gemms[4] = {{3 * D, D}, {D, D}, {F, D}, {D, F}};
+  int nch = 0;
+  uint32_t off = 0;
+  for (int g = 0; g < 4; ++g) {
+    const int KB = gemms[g].K < 64 ? gemms[g].K : 64;
+    for (int n0 = 0; n0 < gemms[g].N; n0 += 128) {
+      const int NB = (gemms[g].N - n0) < 128 ? (gemms[g].N - n0) : 128;
+      for (int k0 = 0; k0 < gemms[g].K; k0 += KB) {
+        ChunkDesc &c = h->chunks[nch++];
+        c.off = off;
+        c.bytes = static_cast<uint32_t>(NB * KB * 2);
+        c.gemm = static_cast<uint16_t>(g);
+        c.n0 = static_cast<uint16_t>(n0);
+        c.nrows = static_cast<uint16_t>(NB);
+        c.k0 = static_cast<uint16_t>(k0);
+        c.kcols = static_cast<uint16_t>(KB);
+        off += c.bytes;
+      }
+    }
+  }
+  h->n_chunks = nch;
+  h->layer_bytes = off;
+  std::vector<uint16_t> ws((size_t)d.n_layers * off / 2, 0);
+  {
+    const size_t per_layer_packed = 12u * (size_t)D * D / 4u;
+    std::vector<int8_t> W[4];
+    for (int l = 0; l < d.n_layers; ++l) {
+      const uint8_t *pk = d.w_packed + per_layer_packed * l;
+      // the six matrices in ABI order, unpacked
+      auto unpack = [&](const uint8_t *src, int rows, int cols, int8_t *dst) {
+        for (int r = 0; r < rows; ++r)
+          for (int c = 0; c < cols; ++c) {
+            const uint8_t byte = src[(size_t)r * (cols / 4) + c / 4];
+            dst[(size_t)r * cols + c] = tern((byte >> (2 * (c % 4))) & 3u);
+          }
+      };
+      for (int g = 0; g < 4; ++g) W[g].assign((size_t)gemms[g].N * gemms[g].K, 0);
+      const size_t dd4 = (size_t)D * D / 4;
+      unpack(pk, D, D, W[0].data());                                 // W_q -> QKV rows [0, D)
+      unpack(pk + dd4, D, D, W[0].data() + (size_t)D * D);           // W_k -> rows [D, 2D)
+      unpack(pk + 2 * dd4, D, D, W[0].data() + (size_t)2 * D * D);   // W_v -> rows [2D, 3D)
+      unpack(pk + 3 * dd4, D, D, W[1].data());                       // W_o
+      unpack(pk + 4 * dd4, F, D, W[2].data());                       // W_1
+      unpack(pk + 4 * dd4 + (size_t)F * D / 4, D, F, W[3].data());   // W_2
+      uint16_t *lw = ws.data() + (size_t)l * off / 2;
+      for (int c = 0; c < nch; ++c) {
+        const ChunkDesc &ch = h->chunks[c];
+        const Gemm gm = gemms[ch.gemm];
+        uint8_t *base = reinterpret_cast<uint8_t *>(lw) + ch.off;
+        for (int rr = 0; rr < ch.nrows; ++rr)
+          for (int cc = 0; cc < ch.kcols; ++cc) {
+            const int8_t v = W[ch.gemm][(size_t)(ch.n0 + rr) * gm.K + ch.k0 + cc];
+            const uint16_t bits = f2bf_bits(static_cast<float>(v));
+            std::memcpy(base + core_off(rr, cc, ch.kcols), &bits, 2);
+          }
+      }
+    }
+  }
+  // ---- per-block parameter vectors
+  const int LPS = LayerParamLayout::stride(D);
+  std::vector<float> lpv((size_t)d.n_layers * LPS, 0.0f);
+  for (int l = 0; l < d.n_layers; ++l) {
+    float *v = lpv.data() + (size_t)l * LPS;
+    std::memcpy(v, d.bias + (size_t)l * 9 * D, sizeof(float) * 9 * D);  // b_q b_k b_v b_o b_1 b_2
+    std::memcpy(v + LayerParamLayout::ln1g(D), d.ln_gamma + (size_t)l * 2 * D, sizeof(float) * D);
+    std::memcpy(v + LayerParamLayout::ln1b(D), d.ln_beta + (size_t)l * 2 * D, sizeof(float) * D);
+    std::memcpy(v + LayerParamLayout::ln2g(D), d.ln_gamma + (size_t)l * 2 * D + D, sizeof(float) * D);
+    std::memcpy(v + LayerParamLayout::ln2b(D), d.ln_beta + (size_t)l * 2 * D + D, sizeof(float) * D);
+    std::memcpy(v + LayerParamLayout::sw(D), d.w_scale + (size_t)l * 6, sizeof(float) * 6);
+  }
+  const int de = D - d.d_spe;
+  if ((rc = dev_upload(h, &h->wstream, reinterpret_cast<const uint8_t *>(ws.data()), ws.size() * 2)) ||
+      (rc = dev_upload(h, &h->lparams, lpv.data(), lpv.size())) ||
+      (rc = dev_upload(h, &h->emb, d.emb, (size_t)T * de)) ||
+      (rc = dev_upload(h, &h->spe, d.spe, (size_t)T * d.d_spe)) ||
+      (rc = dev_upload(h, &h->w_d1, d.w_d1, (size_t)D)) ||
+      (rc = dev_upload(h, &h->w_out, d.w_out, (size_t)T * n)) ||
+      (rc = dev_upload(h, &h->b_out, d.b_out, (size_t)n)) ||
+      (rc = dev_upload(h, &h->hrow_off, hoff.data(), hoff.size())) ||
+      (rc = dev_upload(h, &h->hrow_idx, hidx.data(), hidx.size())) ||
+      (rc = dev_upload(h, &h->mask_off[0], moff[0].data(), moff[0].size())) ||
+      (rc = dev_upload(h, &h->mask_idx[0], midx[0].data(), midx[0].size())) ||
+      (rc = dev_upload(h, &h->mask_off[1], moff[1].data(), moff[1].size())) ||
+      (rc = dev_upload(h, &h->mask_idx[1], midx[1].data(), midx[1].size())) ||
+      (rc = dev_upload<int>(h, &h->d_err, nullptr, 1))) {
+    free_handle(h);
+    return rc;
+  }
+  if ((e = cudaMemset(h->d_err, 0, sizeof(int))) != cudaSuccess ||
+      (e = cudaHostAlloc(reinterpret_cast<void **>(&h->h_err), sizeof(int), cudaHostAllocDefault)) != cudaSuccess ||
+      (e = cudaEventCreateWithFlags(&h->ev, cudaEventDisableTiming)) != cudaSuccess) {
+    free_handle(h);
+    return cuda_fail(e, "create");
+  }
+  *h->h_err = 0;
+  *out = h;
+  return AECCT_OK;
+}
+
+static int collect_status(aecct_handle *h, bool block) {
+  if (!h->ev_pending) {
+    const int s = h->pending_status;
+    h->pending_status = AECCT_OK;
+    return s;
+  }
+  cudaError_t e = block ? cudaEventSynchronize(h->ev) : cudaEventQuery(h->ev);
+  if (e == cudaErrorNotReady) return AECCT_OK;
+  h->ev_pending = false;
+  if (e != cudaSuccess) return cuda_fail(e, "decode kernel");
+  if (*h->h_err) {
+    *h->h_err = 0;
+    cudaMemset(h->d_err, 0, sizeof(int));
+    g_last_error = "a device-side wait exceeded its limit";
+    return AECCT_ERR_TIMEOUT;
+  }
+  return AECCT_OK;
+}
+
+int aecct_decode(aecct_handle *h, const float *y_dev, int64_t B, uint8_t *bits_dev, uint8_t *syndrome_dev,
+                 float *logits_dev, void *cuda_stream) {
+  if (!h || B < 0) return AECCT_ERR_INVALID_ARG;
+  if (B == 0) return AECCT_OK;
+  if (!y_dev || !bits_dev) return AECCT_ERR_INVALID_ARG;
+  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+  const int prev = collect_status(h, false);
+  if (prev != AECCT_OK) return prev;
+  DecodeParams p = {};
+  p.n = h->n, p.k = h->k, p.T = h->T, p.m = h->m, p.n_layers = h->n_layers, p.h_first = h->h_first;
+  p.d_spe = h->d_spe, p.C = h->C, p.G = h->G;
+  p.B = B;
+  p.n_groups = (B + h->G - 1) / h->G;
+  p.n_clusters = static_cast<int>(p.n_groups < h->max_clusters ? p.n_groups : h->max_clusters);
+  p.y = y_dev, p.bits = bits_dev, p.syn = syndrome_dev, p.logits = logits_dev;
+  p.wstream = h->wstream, p.layer_bytes = h->layer_bytes, p.n_chunks = h->n_chunks;
+  std::memcpy(p.chunks, h->chunks, sizeof(p.chunks));
+  p.lparams = h->lparams, p.emb = h->emb, p.spe = h->spe, p.w_d1 = h->w_d1, p.b_d1 = h->b_d1;
+  p.w_out = h->w_out, p.b_out = h->b_out, p.hrow_off = h->hrow_off, p.hrow_idx = h->hrow_idx;
+  p.mask_off[0] = h->mask_off[0], p.mask_off[1] = h->mask_off[1];
+  p.mask_idx[0] = h->mask_idx[0], p.mask_idx[1] = h->mask_idx[1];
+  p.ln_eps = h->ln_eps, p.alpha_floor = h->alpha_floor, p.att_scale = h->att_scale;
+  p.cap_B = h->cap_B, p.cap_q = h->cap_q, p.cap_acc = h->cap_acc, p.cap_alpha = h->cap_alpha, p.cap_syn = h->cap_syn;
+  p.err = h->d_err, p.wait_limit = h->wait_limit;
+  cudaError_t e;
+  if (h->d == 32) e = launch_decode<32>(p, stream);
+  else if (h->d == 64) e = launch_decode<64>(p, stream);
+  else e = launch_decode<128>(p, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "decode launch");
+  if ((e = cudaMemcpyAsync(h->h_err, h->d_err, sizeof(int), cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
+    return cuda_fail(e, "status copy");
+  if ((e = cudaEventRecord(h->ev, stream)) != cudaSuccess) return cuda_fail(e, "event record");
+  h->ev_pending = true;
+  return AECCT_OK;
+}
+
+int aecct_synchronize(aecct_handle *h) {
+  if (!h) return AECCT_ERR_INVALID_ARG;
+  return collect_status(h, true);
+}
+
+int aecct_decode_host(aecct_handle *h, const float *y_host, int64_t B, uint8_t *bits_host, uint8_t *syndrome_host,
+                      float *logits_host, void *cuda_stream) {
+  if (!h || B < 0) return AECCT_ERR_INVALID_ARG;
+  if (B == 0) return AECCT_OK;
+  if (!y_host || !bits_host) return AECCT_ERR_INVALID_ARG;
+  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+  cudaError_t e;
+  if (B > h->stage_B) {
+    cudaFree(h->st_y), cudaFree(h->st_bits), cudaFree(h->st_syn), cudaFree(h->st_logits);
+    h->st_y = nullptr, h->st_bits = nullptr, h->st_syn = nullptr, h->st_logits = nullptr, h->stage_B = 0;
+    if ((e = cudaMalloc(&h->st_y, sizeof(float) * B * h->n)) != cudaSuccess ||
+        (e = cudaMalloc(&h->st_bits, (size_t)B * h->n)) != cudaSuccess ||
+        (e = cudaMalloc(&h->st_syn, (size_t)B * h->m)) != cudaSuccess ||
+        (e = cudaMalloc(&h->st_logits, sizeof(float) * B * h->n)) != cudaSuccess)
+      return e == cudaErrorMemoryAllocation ? AECCT_ERR_OUT_OF_MEMORY : cuda_fail(e, "staging");
+    h->stage_B = B;
+  }
+  if ((e = cudaMemcpyAsync(h->st_y, y_host, sizeof(float) * B * h->n, cudaMemcpyHostToDevice, stream)) != cudaSuccess)
+    return cuda_fail(e, "copy y");
+  int rc = aecct_decode(h, h->st_y, B, h->st_bits, syndrome_host ? h->st_syn : nullptr,
+                        logits_host ? h->st_logits : nullptr, cuda_stream);
+  if (rc) return rc;
+  if ((e = cudaMemcpyAsync(bits_host, h->st_bits, (size_t)B * h->n, cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
+    return cuda_fail(e, "copy bits");
+  if (syndrome_host &&
+      (e = cudaMemcpyAsync(syndrome_host, h->st_syn, (size_t)B * h->m, cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
+    return cuda_fail(e, "copy syndrome");
+  if (logits_host && (e = cudaMemcpyAsync(logits_host, h->st_logits, sizeof(float) * B * h->n,
+                                          cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
+    return cuda_fail(e, "copy logits");
+  if ((e = cudaStreamSynchronize(stream)) != cudaSuccess) return cuda_fail(e, "stream sync");
+  return collect_status(h, true);
+}
+
+int aecct_set_capture(aecct_handle *h, int64_t cap_B, int8_t *q_dev, int32_t *acc_dev, float *alpha_dev,
+                      uint8_t *syn_dev) {
+  if (!h || cap_B < 0) return AECCT_ERR_INVALID_ARG;
+  h->cap_B = cap_B;
+  h->cap_q = cap_B ? q_dev : nullptr;
+  h->cap_acc = cap_B ? acc_dev : nullptr;
+  h->cap_alpha = cap_B ? alpha_dev : nullptr;
+  h->cap_syn = cap_B ? syn_dev : nullptr;
+  return AECCT_OK;
+}
+
+int aecct_query(const aecct_handle *h, int32_t *cluster_ctas, int32_t *words_per_group, int32_t *max_clusters,
+                int32_t *threads_per_cta, int32_t *smem_bytes, int32_t *tmem_cols) {
+  if (!h) return AECCT_ERR_INVALID_ARG;
+  if (cluster_ctas) *cluster_ctas = h->C;
+  if (words_per_group) *words_per_group = h->G;
+  if (max_clusters) *max_clusters = h->max_clusters;
+  if (threads_per_cta) *threads_per_cta = kThreads;
+  const int sm = h->d == 32 ? SmemLayout<32>::kTotal : (h->d == 64 ? SmemLayout<64>::kTotal : SmemLayout<128>::kTotal);
+  if (smem_bytes) *smem_bytes = sm;
+  if (tmem_cols) *tmem_cols = 4 * h->d;
+  return AECCT_OK;
+}
+
+int aecct_destroy(aecct_handle *h) {
+  if (!h) return AECCT_ERR_INVALID_ARG;
+  if (h->ev_pending) cudaEventSynchronize(h->ev);
+  free_handle(h);
+  return AECCT_OK;
+}
+
+int aecct_selftest_mma(const int8_t *a_host, const int8_t *b_host, int32_t K, int32_t N, float *out_host) {
+  if (!a_host || !b_host || !out_host) return AECCT_ERR_INVALID_ARG;
+  if (K < 16 || K > 128 || K % 16 || N < 16 || N > 256 || N % 16) return AECCT_ERR_INVALID_ARG;
+  cudaError_t e = run_selftest_mma(a_host, b_host, K, N, out_host);
+  if (e == cudaErrorTimeout) return AECCT_ERR_TIMEOUT;
+  return e == cudaSuccess ? AECCT_OK : cuda_fail(e, "selftest mma");
+}
+
+int aecct_selftest_timeout(int64_t limit_cycles, int32_t *status_host) {
+  if (!status_host || limit_cycles <= 0) return AECCT_ERR_INVALID_ARG;
+  int st = -1;
+  cudaError_t e = run_selftest_timeout(limit_cycles, &st);
+  if (e != cudaSuccess) return cuda_fail(e, "selftest timeout");
+  *status_host = st == 1 ? AECCT_ERR_TIMEOUT : (st == 0 ? AECCT_OK : AECCT_ERR_CUDA);
+  return AECCT_OK;
+}
+
+}  // extern "C"

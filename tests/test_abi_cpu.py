@@ -1,0 +1,101 @@
+"""CPU-side checks of the C ABI: the library builds and loads, exports every function that
+include/aecct.h declares, packs weights in the documented 2-bit format, and rejects invalid
+model descriptions before touching a GPU."""
+import copy
+import os
+import re
+
+import numpy as np
+import pytest
+
+from paper_2410_05911_gb300 import aecct as A
+from paper_2410_05911_gb300 import inputs as I
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def header_functions():
+    text = open(os.path.join(ROOT, "include", "aecct.h")).read()
+    return sorted(set(re.findall(r"^\s*(?:int|const char \*)\s*(aecct_\w+)\s*\(", text, re.M)))
+
+
+def test_library_exports_every_declared_function():
+    L = A.load()
+    names = header_functions()
+    assert len(names) >= 11
+    for name in names:
+        assert hasattr(L, name), name
+    assert set(names) == set(A.EXPORTED_SYMBOLS)
+
+
+def test_status_strings():
+    assert A.status_string(0) == "ok"
+    assert "timed out" in A.status_string(A.AECCT_ERR_TIMEOUT)
+    assert A.status_string(-99) == "unknown status"
+
+
+def test_pack_ternary_layout():
+    t = np.array([[1, 0, -1, 1, 0, 0, 0, -1]], np.int8)
+    p = A.pack_ternary(t)
+    assert p.tolist() == [[0b01110001, 0b11000000]]
+    rng = np.random.default_rng(0)
+    t = rng.integers(-1, 2, (16, 64)).astype(np.int8)
+    p = A.pack_ternary(t)
+    codes = np.stack([(p >> (2 * s)) & 3 for s in range(4)], -1).reshape(16, 64)
+    back = np.where(codes == 1, 1, np.where(codes == 3, -1, 0))
+    assert (back == t).all() and not (codes == 2).any()
+    with pytest.raises(ValueError):
+        A.pack_ternary(np.array([[2, 0, 0, 0]], np.int8))
+
+
+def _status(model, **kw):
+    st, h = A.create_handle(model, **kw)
+    assert h is None or st == 0
+    return st
+
+
+@pytest.mark.parametrize("mutate,expected", [
+    (lambda m: setattr(m, "h_first", 9), A.AECCT_ERR_INVALID_ARG),
+    (lambda m: setattr(m, "h_first", -1), A.AECCT_ERR_INVALID_ARG),
+    (lambda m: setattr(m, "d_spe", 32), A.AECCT_ERR_INVALID_ARG),
+    (lambda m: setattr(m, "n_layers", 0), A.AECCT_ERR_INVALID_ARG),
+    (lambda m: setattr(m, "ln_eps", float("nan")), A.AECCT_ERR_INVALID_ARG),
+    (lambda m: setattr(m, "alpha_floor", 0.0), A.AECCT_ERR_INVALID_ARG),
+    (lambda m: m.H.__setitem__((0, 0), 2), A.AECCT_ERR_INVALID_ARG),
+    (lambda m: m.H.__setitem__((0, slice(None)), 0), A.AECCT_ERR_INVALID_ARG),
+    (lambda m: m.H.__setitem__((slice(None), 3), 0), A.AECCT_ERR_INVALID_ARG),
+    (lambda m: setattr(m, "activation", 7), A.AECCT_ERR_INVALID_ARG),
+    (lambda m: setattr(m, "activation", 1), A.AECCT_ERR_UNSUPPORTED),
+    (lambda m: setattr(m, "ffn_mult", 2), A.AECCT_ERR_UNSUPPORTED),
+])
+def test_create_rejects_invalid_descriptions(mutate, expected):
+    m = copy.deepcopy(I.workload_model("bch31_16"))
+    mutate(m)
+    assert _status(m) == expected
+
+
+def test_create_rejects_invalid_packed_code_and_shapes():
+    m = I.workload_model("bch31_16")
+    hm = A._HostModel(m)
+    hm.w_packed[5] = 0b00100000  # code 10 in slot 2
+    import ctypes
+    h = ctypes.c_void_p()
+    assert A.load().aecct_create(ctypes.byref(hm.desc), ctypes.byref(h)) == A.AECCT_ERR_INVALID_ARG
+    # valid but outside this build: d = 48 with 8 heads
+    code = I.make_code("bch31_16")
+    m48 = I.random_model(code, 48, 1, seed=3, d_spe=8)
+    assert _status(m48) == A.AECCT_ERR_UNSUPPORTED
+    # a cluster size that cannot hold one codeword
+    big = I.workload_model("ldpc384_192")
+    assert _status(big, cluster_ctas=2) == A.AECCT_ERR_INVALID_ARG
+    # NULL description / output pointer
+    assert A.load().aecct_create(None, ctypes.byref(h)) == A.AECCT_ERR_INVALID_ARG
+    assert A.load().aecct_create(ctypes.byref(hm.desc), None) == A.AECCT_ERR_INVALID_ARG
+
+
+def test_calls_on_null_handle():
+    L = A.load()
+    assert L.aecct_decode(None, None, 1, None, None, None, None) == A.AECCT_ERR_INVALID_ARG
+    assert L.aecct_synchronize(None) == A.AECCT_ERR_INVALID_ARG
+    assert L.aecct_destroy(None) == A.AECCT_ERR_INVALID_ARG
+    assert L.aecct_set_capture(None, 0, None, None, None, None) == A.AECCT_ERR_INVALID_ARG
