@@ -9,11 +9,9 @@ namespace aecct {
 
 constexpr int kRows = 128;          // token rows per CTA: one M = 128 tensor-core tile
 constexpr int kHeads = 8;           // this build: 8 attention heads
-constexpr int kEpiWarps = 16;       // CUDA-core warps: 4 TMEM lane quadrants x 4 column slices
+constexpr int kEpiWarps = 16;       // 4 TMEM lane quadrants x 4 column slices
 constexpr int kEpiThreads = kEpiWarps * 32;
-constexpr int kProducerWarp = 16;   // issues the bulk copies of weight chunks
-constexpr int kMmaWarp = 17;        // allocates TMEM and issues tcgen05.mma
-constexpr int kThreads = 18 * 32;
+constexpr int kThreads = kEpiThreads;  // thread 0 also streams weights and issues the MMAs
 constexpr int kMaxCluster = 8;
 constexpr uint32_t kStageBytes = 16384;  // one weight chunk: <= 128 rows x 64 K bf16
 constexpr int kMaxChunks = 32;           // weight chunks per block (QKV, O, FFN1, FFN2)
@@ -68,8 +66,13 @@ struct DecodeParams {
   const float *b_out;    // [n]
   const uint32_t *hrow_off;  // [m + 1] check i -> variables
   const uint16_t *hrow_idx;
-  const uint32_t *mask_off[2];  // [T + 1] token -> neighbour tokens, ascending; 0 = first ring, 1 = second
-  const uint16_t *mask_idx[2];
+  const uint16_t *perm;         // [T] row offset within a codeword -> token
+  const uint16_t *pos;          // [T] token -> row offset within its codeword
+  // HPSA neighbour lists, 0 = first ring, 1 = second ring.  mask_info[mk][t] = (start << 11) | count:
+  // the count row offsets of token t's neighbours (ascending token order) begin at mask_list[mk][start]
+  // and continue 8 per 16-byte entry (a list is padded to whole entries).
+  const uint32_t *mask_info[2];
+  const uint4 *mask_list[2];
   float ln_eps, alpha_floor, att_scale;
   // integer-core capture (device, optional)
   int64_t cap_B;
@@ -106,7 +109,7 @@ struct SmemLayout {
   static constexpr uint32_t kOffObits = kOffZ + 512;                  // decoded bits
   static constexpr uint32_t kOffBar = kOffObits + kOutBitsBytes;      // mbarriers
   static constexpr uint32_t kOffMisc = kOffBar + 256;                 // tmem base, abort flag, peer bases
-  static constexpr uint32_t kTotal = kOffMisc + 128;
+  static constexpr uint32_t kTotal = kOffMisc + 256;
   static constexpr uint32_t kTmemCols = 4u * D;
 };
 

@@ -8,6 +8,7 @@
 
 #include <cmath>
 #include <cstdlib>
+#include <algorithm>
 #include <cstring>
 #include <string>
 #include <vector>
@@ -40,8 +41,9 @@ struct aecct_handle {
   int n_chunks = 0;
   ChunkDesc chunks[kMaxChunks] = {};
   float *lparams = nullptr, *emb = nullptr, *spe = nullptr, *w_d1 = nullptr, *w_out = nullptr, *b_out = nullptr;
-  uint32_t *hrow_off = nullptr, *mask_off[2] = {nullptr, nullptr};
-  uint16_t *hrow_idx = nullptr, *mask_idx[2] = {nullptr, nullptr};
+  uint32_t *hrow_off = nullptr, *mask_info[2] = {nullptr, nullptr};
+  uint16_t *hrow_idx = nullptr, *mask_list[2] = {nullptr, nullptr};
+  uint16_t *perm = nullptr, *pos = nullptr;
   int *d_err = nullptr;
   int *h_err = nullptr;  // pinned
   cudaEvent_t ev = nullptr;
@@ -226,41 +228,76 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
       if (d.H[(size_t)i * n + j]) hidx.push_back(static_cast<uint16_t>(j));
     hoff[i + 1] = static_cast<uint32_t>(hidx.size());
   }
-  // ---- HPSA neighbour lists (Sec. 4.2): token t < n is variable t, token n + i is check i
-  std::vector<uint32_t> moff[2];
-  std::vector<uint16_t> midx[2];
-  for (int mk = 0; mk < 2; ++mk) moff[mk].assign(T + 1, 0);
-  std::vector<uint8_t> row(T);
-  for (int t = 0; t < T; ++t) {
-    // first ring: Tanner-graph neighbours
-    std::fill(row.begin(), row.end(), 0);
-    if (t < n) {
-      for (int i = 0; i < m; ++i)
-        if (d.H[(size_t)i * n + t]) row[n + i] = 1;
-    } else {
-      for (int j = 0; j < n; ++j)
-        if (d.H[(size_t)(t - n) * n + j]) row[j] = 1;
+  // ---- HPSA neighbour lists (Sec. 4.2): token t < n is variable t, token n + i is check i.
+  // First ring: Tanner-graph neighbours.  Second ring: same-type nodes at distance two, and the
+  // node itself.  Lists are in ascending token order (the order the softmax sums run in).
+  std::vector<std::vector<uint16_t>> nb[2];
+  nb[0].resize(T);
+  nb[1].resize(T);
+  {
+    std::vector<uint8_t> row(T);
+    for (int t = 0; t < T; ++t) {
+      std::fill(row.begin(), row.end(), 0);
+      if (t < n) {
+        for (int i = 0; i < m; ++i)
+          if (d.H[(size_t)i * n + t]) row[n + i] = 1;
+      } else {
+        for (int j = 0; j < n; ++j)
+          if (d.H[(size_t)(t - n) * n + j]) row[j] = 1;
+      }
+      for (int u = 0; u < T; ++u)
+        if (row[u]) nb[0][t].push_back(static_cast<uint16_t>(u));
+      std::fill(row.begin(), row.end(), 0);
+      if (t < n) {
+        for (int i = 0; i < m; ++i)
+          if (d.H[(size_t)i * n + t])
+            for (int j = 0; j < n; ++j)
+              if (d.H[(size_t)i * n + j]) row[j] = 1;
+      } else {
+        const int i0 = t - n;
+        for (int j = 0; j < n; ++j)
+          if (d.H[(size_t)i0 * n + j])
+            for (int i = 0; i < m; ++i)
+              if (d.H[(size_t)i * n + j]) row[n + i] = 1;
+      }
+      for (int u = 0; u < T; ++u)
+        if (row[u]) nb[1][t].push_back(static_cast<uint16_t>(u));
     }
-    for (int u = 0; u < T; ++u)
-      if (row[u]) midx[0].push_back(static_cast<uint16_t>(u));
-    moff[0][t + 1] = static_cast<uint32_t>(midx[0].size());
-    // second ring: same-type nodes at distance two, and the node itself
-    std::fill(row.begin(), row.end(), 0);
-    if (t < n) {
-      for (int i = 0; i < m; ++i)
-        if (d.H[(size_t)i * n + t])
-          for (int j = 0; j < n; ++j)
-            if (d.H[(size_t)i * n + j]) row[j] = 1;
-    } else {
-      const int i0 = t - n;
-      for (int j = 0; j < n; ++j)
-        if (d.H[(size_t)i0 * n + j])
-          for (int i = 0; i < m; ++i)
-            if (d.H[(size_t)i * n + j]) row[n + i] = 1;
+  }
+  // Rows of a codeword hold its tokens sorted by attention work (keys over the thread's first-ring
+  // and second-ring head), so the 32 rows of a warp loop over similar key counts.
+  std::vector<uint16_t> perm(T), pos(T);
+  {
+    std::vector<int> order(T);
+    for (int t = 0; t < T; ++t) order[t] = t;
+    const int hf = d.h_first, hs = d.heads - d.h_first;
+    auto work = [&](int t) {
+      const size_t a = hf > 0 ? nb[0][t].size() : 0, b = hs > 0 ? nb[1][t].size() : 0;
+      return (hf > 0 && hs > 0) ? a + b : (a + b) * 2;
+    };
+    std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return work(a) > work(b); });
+    for (int i = 0; i < T; ++i) {
+      perm[i] = static_cast<uint16_t>(order[i]);
+      pos[order[i]] = static_cast<uint16_t>(i);
     }
-    for (int u = 0; u < T; ++u)
-      if (row[u]) midx[1].push_back(static_cast<uint16_t>(u));
-    moff[1][t + 1] = static_cast<uint32_t>(midx[1].size());
+  }
+  // lists of row offsets, each padded to a multiple of 8 entries (one 16-byte load per 8 keys)
+  std::vector<uint32_t> minfo[2];
+  std::vector<uint16_t> mlist[2];
+  for (int mk = 0; mk < 2; ++mk) {
+    minfo[mk].assign(T, 0);
+    for (int t = 0; t < T; ++t) {
+      const size_t start = mlist[mk].size() / 8;
+      const size_t cnt = nb[mk][t].size();
+      if (cnt >= 2048 || start >= (1u << 21)) {
+        g_last_error = "neighbour list too long";
+        return AECCT_ERR_UNSUPPORTED;
+      }
+      minfo[mk][t] = static_cast<uint32_t>((start << 11) | cnt);
+      for (uint16_t u : nb[mk][t]) mlist[mk].push_back(pos[u]);
+      while (mlist[mk].size() % 8) mlist[mk].push_back(0);
+    }
+    if (mlist[mk].empty()) mlist[mk].assign(8, 0);
   }
 
   // ---- weights: 2-bit codes -> bf16 K-major core-matrix chunks, in the order the MMA consumes them
@@ -344,10 +381,12 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
       (rc = dev_upload(h, &h->b_out, d.b_out, (size_t)n)) ||
       (rc = dev_upload(h, &h->hrow_off, hoff.data(), hoff.size())) ||
       (rc = dev_upload(h, &h->hrow_idx, hidx.data(), hidx.size())) ||
-      (rc = dev_upload(h, &h->mask_off[0], moff[0].data(), moff[0].size())) ||
-      (rc = dev_upload(h, &h->mask_idx[0], midx[0].data(), midx[0].size())) ||
-      (rc = dev_upload(h, &h->mask_off[1], moff[1].data(), moff[1].size())) ||
-      (rc = dev_upload(h, &h->mask_idx[1], midx[1].data(), midx[1].size())) ||
+      (rc = dev_upload(h, &h->perm, perm.data(), perm.size())) ||
+      (rc = dev_upload(h, &h->pos, pos.data(), pos.size())) ||
+      (rc = dev_upload(h, &h->mask_info[0], minfo[0].data(), minfo[0].size())) ||
+      (rc = dev_upload(h, &h->mask_list[0], mlist[0].data(), mlist[0].size())) ||
+      (rc = dev_upload(h, &h->mask_info[1], minfo[1].data(), minfo[1].size())) ||
+      (rc = dev_upload(h, &h->mask_list[1], mlist[1].data(), mlist[1].size())) ||
       (rc = dev_upload<int>(h, &h->d_err, nullptr, 1))) {
     free_handle(h);
     return rc;
@@ -401,8 +440,10 @@ int aecct_decode(aecct_handle *h, const float *y_dev, int64_t B, uint8_t *bits_d
   std::memcpy(p.chunks, h->chunks, sizeof(p.chunks));
   p.lparams = h->lparams, p.emb = h->emb, p.spe = h->spe, p.w_d1 = h->w_d1, p.b_d1 = h->b_d1;
   p.w_out = h->w_out, p.b_out = h->b_out, p.hrow_off = h->hrow_off, p.hrow_idx = h->hrow_idx;
-  p.mask_off[0] = h->mask_off[0], p.mask_off[1] = h->mask_off[1];
-  p.mask_idx[0] = h->mask_idx[0], p.mask_idx[1] = h->mask_idx[1];
+  p.perm = h->perm, p.pos = h->pos;
+  p.mask_info[0] = h->mask_info[0], p.mask_info[1] = h->mask_info[1];
+  p.mask_list[0] = reinterpret_cast<const uint4 *>(h->mask_list[0]);
+  p.mask_list[1] = reinterpret_cast<const uint4 *>(h->mask_list[1]);
   p.ln_eps = h->ln_eps, p.alpha_floor = h->alpha_floor, p.att_scale = h->att_scale;
   p.cap_B = h->cap_B, p.cap_q = h->cap_q, p.cap_acc = h->cap_acc, p.cap_alpha = h->cap_alpha, p.cap_syn = h->cap_syn;
   p.err = h->d_err, p.wait_limit = h->wait_limit;

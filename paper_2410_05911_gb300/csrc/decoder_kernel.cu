@@ -150,6 +150,189 @@ struct RowRed {
   __device__ __forceinline__ float *slot(int s, int r) { return buf + (sel * 4 + s) * kRows + r; }
 };
 
+// 16-bit entry k of an index block (k known at compile time after unrolling)
+__device__ __forceinline__ int idx_at(const uint4 &w, int k) {
+  const uint32_t word = k < 2 ? w.x : (k < 4 ? w.y : (k < 6 ? w.z : w.w));
+  return static_cast<int>((k & 1) ? (word >> 16) : (word & 0xFFFFu));
+}
+
+// One (query, head) of HPSA (Sec. 4.2) over the neighbour rows described by `info` (see
+// DecodeParams::mask_info).  Two passes in the canonical order:
+// sigma_u = fma-chain(q . k_u) * scale, m = max sigma; p_u = 2^(sigma_u - m);
+// l = sum p_u and num = sum p_u v_u in ascending key order; A = num * (1 / l).
+// Keys come 8 per index load; U keys at a time have their loads issued together and their dot
+// products run as independent chains, while every sum keeps the sequential key order.
+template <int DH, int U, uint32_t STRIDE>
+__device__ __forceinline__ void hpsa_head(const float *q, uint32_t info, const uint4 *__restrict__ lists,
+                                          const uint64_t *kvgen, int rowbase, uint32_t hoff, float scale, float *A) {
+  const uint4 *lst = lists + (info >> 11);
+  const int cnt = static_cast<int>(info & 2047u);
+  auto keyptr = [&](int off) -> const float4 * {
+    const int ru = rowbase + off;
+    return reinterpret_cast<const float4 *>(kvgen[ru >> 7] + static_cast<uint32_t>(ru & 127) * STRIDE + hoff);
+  };
+  auto dotk = [&](const float4 *kk) -> float {
+    float dot = 0.0f;
+#pragma unroll
+    for (int i = 0; i < DH / 4; ++i) {
+      dot = __fmaf_rn(q[4 * i], kk[i].x, dot);
+      dot = __fmaf_rn(q[4 * i + 1], kk[i].y, dot);
+      dot = __fmaf_rn(q[4 * i + 2], kk[i].z, dot);
+      dot = __fmaf_rn(q[4 * i + 3], kk[i].w, dot);
+    }
+    return dot;
+  };
+  // pass 1: maximum score
+  float mx = -INFINITY;
+  for (int jb = 0; jb < cnt; jb += 8) {
+    const uint4 w = __ldg(lst + (jb >> 3));
+    if (jb + 8 <= cnt) {
+#pragma unroll
+      for (int k0 = 0; k0 < 8; k0 += U) {
+        float4 kk[U][DH / 4];
+#pragma unroll
+        for (int k = 0; k < U; ++k) {
+          const float4 *kp = keyptr(idx_at(w, k0 + k));
+#pragma unroll
+          for (int i = 0; i < DH / 4; ++i) kk[k][i] = kp[i];
+        }
+#pragma unroll
+        for (int k = 0; k < U; ++k) mx = fmaxf(mx, __fmul_rn(dotk(kk[k]), scale));
+      }
+    } else {
+      for (int k = 0; k < cnt - jb; ++k) {
+        const float4 *kp = keyptr(idx_at(w, k));
+        float4 kk[DH / 4];
+#pragma unroll
+        for (int i = 0; i < DH / 4; ++i) kk[i] = kp[i];
+        mx = fmaxf(mx, __fmul_rn(dotk(kk), scale));
+      }
+    }
+  }
+  // pass 2: probabilities, their sum and the weighted values, in key order
+  float lsum = 0.0f;
+  float num[DH];
+#pragma unroll
+  for (int i = 0; i < DH; ++i) num[i] = 0.0f;
+  auto accumulate = [&](float pr, const float4 *vv) {
+    lsum = __fadd_rn(lsum, pr);
+#pragma unroll
+    for (int i = 0; i < DH / 4; ++i) {
+      num[4 * i] = __fmaf_rn(pr, vv[i].x, num[4 * i]);
+      num[4 * i + 1] = __fmaf_rn(pr, vv[i].y, num[4 * i + 1]);
+      num[4 * i + 2] = __fmaf_rn(pr, vv[i].z, num[4 * i + 2]);
+      num[4 * i + 3] = __fmaf_rn(pr, vv[i].w, num[4 * i + 3]);
+    }
+  };
+  for (int jb = 0; jb < cnt; jb += 8) {
+    const uint4 w = __ldg(lst + (jb >> 3));
+    if (jb + 8 <= cnt) {
+#pragma unroll
+      for (int k0 = 0; k0 < 8; k0 += U) {
+        float4 kk[U][DH / 4], vv[U][DH / 4];
+#pragma unroll
+        for (int k = 0; k < U; ++k) {
+          const float4 *kp = keyptr(idx_at(w, k0 + k));
+#pragma unroll
+          for (int i = 0; i < DH / 4; ++i) kk[k][i] = kp[i];
+#pragma unroll
+          for (int i = 0; i < DH / 4; ++i) vv[k][i] = kp[DH / 4 + i];
+        }
+        float pr[U];
+#pragma unroll
+        for (int k = 0; k < U; ++k) pr[k] = exp2_series(__fsub_rn(__fmul_rn(dotk(kk[k]), scale), mx));
+#pragma unroll
+        for (int k = 0; k < U; ++k) accumulate(pr[k], vv[k]);
+      }
+    } else {
+      for (int k = 0; k < cnt - jb; ++k) {
+        const float4 *kp = keyptr(idx_at(w, k));
+        float4 kk[DH / 4], vv[DH / 4];
+#pragma unroll
+        for (int i = 0; i < DH / 4; ++i) kk[i] = kp[i];
+#pragma unroll
+        for (int i = 0; i < DH / 4; ++i) vv[i] = kp[DH / 4 + i];
+        accumulate(exp2_series(__fsub_rn(__fmul_rn(dotk(kk), scale), mx)), vv);
+      }
+    }
+  }
+  const float inv = __fdiv_rn(1.0f, lsum);
+#pragma unroll
+  for (int i = 0; i < DH; ++i) A[i] = __fmul_rn(num[i], inv);
+}
+
+// ------------------------------------------------------------------------------------------
+// weight streaming and tensor-core issue (run by thread 0 of each CTA)
+// ------------------------------------------------------------------------------------------
+// Weight chunks are consumed in a fixed sequence: for each group of codewords, for each block,
+// the block's chunks (QKV, then O, FFN1, FFN2).  Chunk i of the sequence uses ring stage i % S;
+// its copy completes phase i / S of full[stage], its MMAs release phase i / S of empty[stage].
+struct IssueState {
+  int64_t total;   // chunks this CTA consumes
+  int64_t issued;  // chunks whose copy has been started
+  int64_t used;    // chunks whose MMAs have been issued
+  uint32_t oph;    // parity of the next operand-ready phase
+};
+
+template <int D>
+__device__ __noinline__ void issue_copies(const DecodeParams &p, const Ctl &ctl, IssueState &st, int64_t limit,
+                                          uint32_t sb) {
+  using L = SmemLayout<D>;
+  constexpr int S = L::kStages;
+  const uint32_t bar_full = sb + L::kOffBar, bar_empty = bar_full + 8 * S;
+  if (limit > st.total) limit = st.total;
+  while (st.issued < limit) {
+    if (*ctl.abort) return;
+    const int s = static_cast<int>(st.issued % S);
+    if (st.issued >= S) wait_bar(ctl, bar_empty + 8 * s, static_cast<uint32_t>((st.issued / S - 1) & 1), false);
+    const int c = static_cast<int>(st.issued % p.n_chunks);
+    const int l = static_cast<int>((st.issued / p.n_chunks) % p.n_layers);
+    const uint32_t bytes = p.chunks[c].bytes;
+    mbar_arrive_expect_tx(bar_full + 8 * s, bytes);
+    bulk_g2s(sb + L::kOffW + s * kStageBytes, p.wstream + (size_t)l * p.layer_bytes + p.chunks[c].off, bytes,
+             bar_full + 8 * s);
+    ++st.issued;
+  }
+}
+
+// Wait until every warp has published the operand of GEMM `gemm`, issue its tcgen05.mma chain
+// (accumulators at TMEM column 0), signal the accumulator barrier, then prefetch the next chunks.
+template <int D>
+__device__ __noinline__ void issue_gemm(const DecodeParams &p, const Ctl &ctl, IssueState &st, int gemm, uint32_t sb,
+                                        uint32_t tmem) {
+  using L = SmemLayout<D>;
+  constexpr int S = L::kStages;
+  const uint32_t bar_full = sb + L::kOffBar, bar_empty = bar_full + 8 * S;
+  const uint32_t bar_op = bar_empty + 8 * S, bar_acc = bar_op + 8;
+  wait_bar(ctl, bar_op, st.oph, false);
+  st.oph ^= 1u;
+  tc_fence_after();
+  const uint32_t a_tile = (gemm == 3) ? (sb + L::kOffU) : (sb + L::kOffAop);
+  const uint32_t a_sbo = (gemm == 3) ? (4u * D / 8u) * 128u : (D / 8u) * 128u;
+  while (st.used < st.total) {
+    const int c = static_cast<int>(st.used % p.n_chunks);
+    const ChunkDesc ch = p.chunks[c];
+    if (ch.gemm != gemm) break;
+    issue_copies<D>(p, ctl, st, st.used + 1, sb);
+    const int s = static_cast<int>(st.used % S);
+    wait_bar(ctl, bar_full + 8 * s, static_cast<uint32_t>((st.used / S) & 1), false);
+    tc_fence_after();
+    const uint32_t b_tile = sb + L::kOffW + s * kStageBytes;
+    const uint32_t b_sbo = (ch.kcols / 8u) * 128u;
+    const uint32_t idesc = make_idesc_bf16(128, ch.nrows);
+    for (int ks = 0; ks < ch.kcols / 16; ++ks) {
+      const uint32_t kabs = ch.k0 + 16u * ks;
+      const uint64_t ad = make_sdesc(a_tile + (kabs / 8u) * 128u, 128u, a_sbo);
+      const uint64_t bd = make_sdesc(b_tile + ks * 256u, 128u, b_sbo);
+      mma_bf16(tmem + ch.n0, ad, bd, idesc, kabs > 0 ? 1u : 0u);
+    }
+    mma_commit(bar_empty + 8 * s);
+    ++st.used;
+  }
+  mma_commit(bar_acc);
+  issue_copies<D>(p, ctl, st, st.used + S, sb);
+}
+
 // ------------------------------------------------------------------------------------------
 // the kernel
 // ------------------------------------------------------------------------------------------
@@ -177,8 +360,8 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   const uint32_t bar_fin = bar_zf + 8;
   uint32_t *s_tmem = reinterpret_cast<uint32_t *>(smem + L::kOffMisc);
   volatile int *s_abort = reinterpret_cast<volatile int *>(smem + L::kOffMisc + 4);
-  uint32_t *s_kvpeer = reinterpret_cast<uint32_t *>(smem + L::kOffMisc + 8);  // [8]
-  uint32_t *s_zpeer = s_kvpeer + kMaxCluster;                                  // [8]
+  uint64_t *s_kvgen = reinterpret_cast<uint64_t *>(smem + L::kOffMisc + 8);  // [8] generic K/V bases per CTA
+  uint64_t *s_zgen = reinterpret_cast<uint64_t *>(smem + L::kOffMisc + 72);   // [8] generic z bases per CTA
 
   if (tid == 0) {
     for (int s = 0; s < S; ++s) {
@@ -193,13 +376,17 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
     mbar_init(bar_zf, p.C);
     mbar_init(bar_fin, 1);
     *s_abort = 0;
+    // generic base of the K/V and z areas of every CTA of the cluster: this CTA's own area through
+    // its plain shared-memory window, the others through the distributed shared window
     for (int c = 0; c < p.C; ++c) {
-      s_kvpeer[c] = mapa_cluster(sb + L::kOffU, c);
-      s_zpeer[c] = mapa_cluster(sb + L::kOffZ, c);
+      const bool own = c == static_cast<int>(crank);
+      s_kvgen[c] = own ? reinterpret_cast<uint64_t>(smem + L::kOffU) : mapa_generic(smem + L::kOffU, c);
+      s_zgen[c] = own ? reinterpret_cast<uint64_t>(smem + L::kOffZ) : mapa_generic(smem + L::kOffZ, c);
     }
     fence_mbar_init_cluster();
   }
-  if (warp == kMmaWarp) {
+  __syncwarp();  // warp 0 reconverges before its warp-collective TMEM allocation
+  if (warp == 0) {
     tmem_alloc(smem_u32(s_tmem), L::kTmemCols);
     tmem_relinquish();
   }
@@ -209,73 +396,14 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   const uint32_t tmem = *s_tmem;
   const Ctl ctl{s_abort, p.err, p.wait_limit};
 
-  if (warp == kProducerWarp) {
-    // ------------------------------------------------------------ weight-chunk producer
-    if (lane == 0) {
-      int stage = 0;
-      uint32_t eph = 0;
-      bool issued[S];
-      uint32_t fpar[S];
-#pragma unroll
-      for (int s = 0; s < S; ++s) issued[s] = false, fpar[s] = 0;
-      for (int64_t gi = cluster_id; gi < p.n_groups; gi += p.n_clusters) {
-        for (int l = 0; l < p.n_layers; ++l) {
-          const uint8_t *lw = p.wstream + (size_t)l * p.layer_bytes;
-          for (int c = 0; c < p.n_chunks; ++c) {
-            if (*s_abort) goto producer_done;
-            wait_bar(ctl, bar_empty + 8 * stage, eph ^ 1u, false);
-            const uint32_t bytes = p.chunks[c].bytes;
-            mbar_arrive_expect_tx(bar_full + 8 * stage, bytes);
-            bulk_g2s(sb + L::kOffW + stage * kStageBytes, lw + p.chunks[c].off, bytes, bar_full + 8 * stage);
-            issued[stage] = true;
-            fpar[stage] = eph;
-            if (++stage == S) stage = 0, eph ^= 1u;
-          }
-        }
-      }
-    producer_done:
-      for (int s = 0; s < S; ++s)
-        if (issued[s]) wait_bar_drain(ctl, bar_full + 8 * s, fpar[s]);
-    }
-  } else if (warp == kMmaWarp) {
-    // ------------------------------------------------------------ tensor-core issuer
-    if (lane == 0) {
-      int stage = 0;
-      uint32_t fph = 0, oph = 0;
-      for (int64_t gi = cluster_id; gi < p.n_groups; gi += p.n_clusters) {
-        if (*s_abort) break;
-        for (int l = 0; l < p.n_layers; ++l) {
-          int c = 0;
-          for (int gemm = 0; gemm < 4; ++gemm) {
-            wait_bar(ctl, bar_op, oph, false);
-            oph ^= 1u;
-            tc_fence_after();
-            const uint32_t a_tile = (gemm == 3) ? (sb + L::kOffU) : (sb + L::kOffAop);
-            const uint32_t a_sbo = (gemm == 3) ? (4u * D / 8u) * 128u : (D / 8u) * 128u;
-            for (; c < p.n_chunks && p.chunks[c].gemm == gemm; ++c) {
-              const ChunkDesc ch = p.chunks[c];
-              wait_bar(ctl, bar_full + 8 * stage, fph, false);
-              tc_fence_after();
-              const uint32_t b_tile = sb + L::kOffW + stage * kStageBytes;
-              const uint32_t b_sbo = (ch.kcols / 8u) * 128u;
-              const uint32_t idesc = make_idesc_bf16(128, ch.nrows);
-              for (int ks = 0; ks < ch.kcols / 16; ++ks) {
-                const uint32_t kabs = ch.k0 + 16u * ks;
-                const uint64_t ad = make_sdesc(a_tile + (kabs / 8u) * 128u, 128u, a_sbo);
-                const uint64_t bd = make_sdesc(b_tile + ks * 256u, 128u, b_sbo);
-                mma_bf16(tmem + ch.n0, ad, bd, idesc, kabs > 0 ? 1u : 0u);
-              }
-              mma_commit(bar_empty + 8 * stage);
-              if (++stage == S) stage = 0, fph ^= 1u;
-            }
-            mma_commit(bar_acc);
-          }
-        }
-      }
-      mma_commit(bar_fin);
-      wait_bar_drain(ctl, bar_fin, 0);
-    }
-  } else {
+  IssueState ist{0, 0, 0, 0};
+  if (tid == 0) {
+    const int64_t my_groups = (p.n_groups - cluster_id + p.n_clusters - 1) / p.n_clusters;
+    ist.total = my_groups * p.n_layers * p.n_chunks;
+    issue_copies<D>(p, ctl, ist, S, sb);
+  }
+  __syncwarp();
+  {
     // ------------------------------------------------------------ CUDA-core warps
     const int qd = warp & 3, sl = warp >> 2;
     const int r = 32 * qd + lane;
@@ -308,11 +436,14 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
       red.sel ^= 1;
       return a;
     };
-    auto signal_op = [&]() {
+    // publish this warp's part of the operand of `gemm`; thread 0 then issues the GEMM
+    auto signal_op = [&](int gemm) {
       tc_fence_before();  // this thread's TMEM reads are ordered before the MMA the arrive releases
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) mbar_arrive(bar_op);
+      if (tid == 0) issue_gemm<D>(p, ctl, ist, gemm, sb, tmem);
+      __syncwarp();  // warp 0 waits for its issuing lane before any warp-collective instruction
     };
     auto cluster_arrive = [&](uint32_t bar) {
       // all 512 CUDA-core threads of this CTA are past their accesses: tell every CTA
@@ -321,6 +452,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         fence_acq_rel_cluster();
         for (int c = 0; c < p.C; ++c) mbar_arrive_cluster(mapa_cluster(bar, c));
       }
+      __syncwarp();
     };
     auto wait_acc = [&]() {
       wait_bar(ctl, bar_acc, acc_ph, false);
@@ -332,7 +464,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
       if (named_bar_or(5, kEpiThreads, *s_abort != 0)) break;
       const int rho = static_cast<int>(crank) * kRows + r;
       const int g = rho / T;
-      const int t = rho - g * T;
+      const int t = __ldg(p.perm + (rho - g * T));  // token held by this row (rows are ordered by attention work)
       const int64_t b = gi * p.G + g;
       const bool row_cw = g < p.G;
       const bool valid = row_cw && b < p.B;
@@ -400,7 +532,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           capture_q(0, 0, qv, sl * XS, XS, alpha_in);
         }
       }
-      signal_op();
+      signal_op(0);
 
       for (int l = 0; l < p.n_layers; ++l) {
         const float *lp = p.lparams + (size_t)l * LP::stride(D);
@@ -459,56 +591,11 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           for (int i = 0; i < DH; ++i) A[hh][i] = 0.0f;
           if (row_cw) {
             const int mk = (e < p.h_first) ? 0 : 1;
-            const uint32_t beg = __ldg(p.mask_off[mk] + t), end = __ldg(p.mask_off[mk] + t + 1);
-            const uint16_t *idx = p.mask_idx[mk];
-            const int rowbase = g * T;
-            const uint32_t hoff = e * (8 * DH);
-            float mx = -INFINITY;
-            for (uint32_t j = beg; j < end; ++j) {
-              const int ru = rowbase + __ldg(idx + j);
-              const uint32_t a = s_kvpeer[ru >> 7] + (ru & 127) * L::kKvStride + hoff;
-              float dot = 0.0f;
-#pragma unroll
-              for (int i = 0; i < DH; i += 4) {
-                const float4 kk = ld_cluster_f32x4(a + 4 * i);
-                dot = __fmaf_rn(q[i], kk.x, dot);
-                dot = __fmaf_rn(q[i + 1], kk.y, dot);
-                dot = __fmaf_rn(q[i + 2], kk.z, dot);
-                dot = __fmaf_rn(q[i + 3], kk.w, dot);
-              }
-              mx = fmaxf(mx, __fmul_rn(dot, p.att_scale));
-            }
-            float lsum = 0.0f;
-            float num[DH];
-#pragma unroll
-            for (int i = 0; i < DH; ++i) num[i] = 0.0f;
-            for (uint32_t j = beg; j < end; ++j) {
-              const int ru = rowbase + __ldg(idx + j);
-              const uint32_t a = s_kvpeer[ru >> 7] + (ru & 127) * L::kKvStride + hoff;
-              float dot = 0.0f;
-#pragma unroll
-              for (int i = 0; i < DH; i += 4) {
-                const float4 kk = ld_cluster_f32x4(a + 4 * i);
-                dot = __fmaf_rn(q[i], kk.x, dot);
-                dot = __fmaf_rn(q[i + 1], kk.y, dot);
-                dot = __fmaf_rn(q[i + 2], kk.z, dot);
-                dot = __fmaf_rn(q[i + 3], kk.w, dot);
-              }
-              const float pr = exp2_series(__fsub_rn(__fmul_rn(dot, p.att_scale), mx));
-              lsum = __fadd_rn(lsum, pr);
-#pragma unroll
-              for (int i = 0; i < DH; i += 4) {
-                const float4 vv = ld_cluster_f32x4(a + 4 * (DH + i));
-                num[i] = __fmaf_rn(pr, vv.x, num[i]);
-                num[i + 1] = __fmaf_rn(pr, vv.y, num[i + 1]);
-                num[i + 2] = __fmaf_rn(pr, vv.z, num[i + 2]);
-                num[i + 3] = __fmaf_rn(pr, vv.w, num[i + 3]);
-              }
-            }
-            const float inv = __fdiv_rn(1.0f, lsum);
-#pragma unroll
-            for (int i = 0; i < DH; ++i) A[hh][i] = __fmul_rn(num[i], inv);
+            constexpr int U = (DH >= 16) ? 2 : 4;
+            hpsa_head<DH, U, L::kKvStride>(q, __ldg(p.mask_info[mk] + t), p.mask_list[mk], s_kvgen, g * T,
+                                           e * (8 * DH), p.att_scale, A[hh]);
           }
+          __syncwarp();  // lanes leave their key loops at different times; reconverge before tcgen05.ld
 #pragma unroll
           for (int i = 0; i < DH; ++i) amax = fmaxf(amax, fabsf(A[hh][i]));
         }
@@ -528,7 +615,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             if (cap) capture_q(l, 1, qv, e * DH, DH, alpha_in);
           }
         }
-        signal_op();
+        signal_op(1);
         cluster_arrive(bar_kvf);  // this CTA no longer reads any K/V of this block
 
         // ---------------- S6: O projection + residual + LayerNorm (Sec. 5, Post-LN)
@@ -566,7 +653,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             capture_q(l, 2, qv, sl * XS, XS, alpha_in);
           }
         }
-        signal_op();
+        signal_op(2);
 
         // ---------------- S7: FFN1 + ReLU (Sec. 4 item 4), Quant(u) -> FFN2 operand
         wait_acc();
@@ -614,7 +701,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             if (cap) capture_q(l, 3, qv, c0, 32, alpha_in);
           }
         }
-        signal_op();
+        signal_op(3);
 
         // ---------------- S8: FFN2 + residual + LayerNorm
         wait_acc();
@@ -649,7 +736,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             for (int j = 0; j < XS; ++j) qv[j] = q_code(x[j], rr);
             capture_q(l + 1, 0, qv, sl * XS, XS, alpha_in);
           }
-          signal_op();
+          signal_op(0);
         }
       }
 
@@ -679,8 +766,8 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           float acc = 0.0f;
           const int rb0 = gg * T;
           for (int tt = 0; tt < T; ++tt) {
-            const int ru = rb0 + tt;
-            const float zt = ld_cluster_f32(s_zpeer[ru >> 7] + (ru & 127) * 4);
+            const int ru = rb0 + __ldg(p.pos + tt);
+            const float zt = *reinterpret_cast<const float *>(s_zgen[ru >> 7] + static_cast<uint32_t>(ru & 127) * 4u);
             acc = __fmaf_rn(__ldg(p.w_out + tt * n + j), zt, acc);
           }
           const float eps = __fadd_rn(acc, __ldg(p.b_out + j));
@@ -709,10 +796,18 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   }
 
   // ------------------------------------------------------------ teardown
+  if (tid == 0) {
+    // every MMA and every weight copy this CTA started must have landed before TMEM and the
+    // shared memory go away
+    mma_commit(bar_fin);
+    wait_bar_drain(ctl, bar_fin, 0);
+    for (int64_t i = ist.issued - S; i < ist.issued; ++i)
+      if (i >= 0) wait_bar_drain(ctl, bar_full + 8 * static_cast<int>(i % S), static_cast<uint32_t>((i / S) & 1));
+  }
   tc_fence_before();
   __syncwarp();
   cluster_sync_all();
-  if (warp == kMmaWarp) {
+  if (warp == 0) {
     __syncwarp();
     tc_fence_after();
     tmem_dealloc(tmem, L::kTmemCols);
