@@ -60,6 +60,9 @@ typedef struct aecct_handle aecct_handle; /* opaque */
  *   activation    0 = ReLU (Sec. 4 item 4).  Other values are rejected.
  *   cluster_ctas  0 = choose automatically; otherwise the number of CTAs (1..8) that
  *                 share one group of codewords (tuning knob).
+ *   attention_mode 0 = choose automatically; 1 = per-row neighbour lists (any cluster size);
+ *                 2 = warp tasks over shared key sets (one CTA per group, d <= 64, at most
+ *                 128 tokens).  Every mode computes the same results bit for bit.
  *   H             [(n-k)][n] uint8 row-major, entries 0/1, no all-zero row or column.
  *   emb           [T][d-d_spe] fp32: token t's embedding row, scaled by h_t (Sec. 3, ECCT).
  *   spe           [T][d_spe] fp32: spectral positional encoding table (Sec. 4.3);
@@ -83,7 +86,7 @@ typedef struct aecct_handle aecct_handle; /* opaque */
  *                 wait, after which the kernel stops and decode reports AECCT_ERR_TIMEOUT.
  */
 typedef struct {
-  int32_t n, k, d, n_layers, heads, h_first, d_spe, ffn_mult, activation, cluster_ctas;
+  int32_t n, k, d, n_layers, heads, h_first, d_spe, ffn_mult, activation, cluster_ctas, attention_mode;
   const uint8_t *H;
   const float *emb;
   const float *spe;
@@ -145,9 +148,10 @@ int aecct_set_capture(aecct_handle *h, int64_t cap_B, int8_t *q_dev, int32_t *ac
 
 /* Launch facts of the handle (for benchmarks): CTAs per codeword group, codewords per
  * group, the number of clusters a decode launches at most, threads per CTA, dynamic
- * shared memory bytes per CTA, and TMEM columns per CTA.  Any pointer may be NULL. */
+ * shared memory bytes per CTA, and the attention mode in use (1 = per-row lists,
+ * 2 = warp tasks).  Any pointer may be NULL. */
 int aecct_query(const aecct_handle *h, int32_t *cluster_ctas, int32_t *words_per_group, int32_t *max_clusters,
-                int32_t *threads_per_cta, int32_t *smem_bytes, int32_t *tmem_cols);
+                int32_t *threads_per_cta, int32_t *smem_bytes, int32_t *attention_mode);
 
 int aecct_destroy(aecct_handle *h);
 

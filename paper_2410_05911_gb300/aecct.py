@@ -40,6 +40,7 @@ class ModelDesc(ctypes.Structure):
         ("n", ctypes.c_int32), ("k", ctypes.c_int32), ("d", ctypes.c_int32), ("n_layers", ctypes.c_int32),
         ("heads", ctypes.c_int32), ("h_first", ctypes.c_int32), ("d_spe", ctypes.c_int32),
         ("ffn_mult", ctypes.c_int32), ("activation", ctypes.c_int32), ("cluster_ctas", ctypes.c_int32),
+        ("attention_mode", ctypes.c_int32),
         ("H", ctypes.c_void_p), ("emb", ctypes.c_void_p), ("spe", ctypes.c_void_p), ("w_packed", ctypes.c_void_p),
         ("w_scale", ctypes.c_void_p), ("bias", ctypes.c_void_p), ("ln_gamma", ctypes.c_void_p),
         ("ln_beta", ctypes.c_void_p), ("w_d1", ctypes.c_void_p), ("b_d1", ctypes.c_float),
@@ -118,7 +119,7 @@ def pack_ternary(t: np.ndarray) -> np.ndarray:
 class _HostModel:
     """Contiguous host copies of a model's tensors, in the ABI layout (kept alive with the desc)."""
 
-    def __init__(self, model, cluster_ctas: int = 0, wait_limit_cycles: int = 0):
+    def __init__(self, model, cluster_ctas: int = 0, wait_limit_cycles: int = 0, attention_mode: int = 0):
         d, F = model.d, model.ffn_mult * model.d
         self.H = np.ascontiguousarray(model.H, dtype=np.uint8)
         self.emb = np.ascontiguousarray(model.emb, dtype=np.float32)
@@ -139,16 +140,16 @@ class _HostModel:
         ptr = lambda a: a.ctypes.data if a.size else None  # noqa: E731
         self.desc = ModelDesc(
             model.n, model.k, model.d, model.n_layers, model.heads, model.h_first, model.d_spe, model.ffn_mult,
-            model.activation, int(cluster_ctas), ptr(self.H), ptr(self.emb), ptr(self.spe), ptr(self.w_packed),
+            model.activation, int(cluster_ctas), int(attention_mode), ptr(self.H), ptr(self.emb), ptr(self.spe), ptr(self.w_packed),
             ptr(self.w_scale), ptr(self.bias), ptr(self.ln_gamma), ptr(self.ln_beta), ptr(self.w_d1),
             float(model.b_d1), ptr(self.w_out), ptr(self.b_out), float(model.ln_eps), float(model.alpha_floor),
             int(wait_limit_cycles))
 
 
-def create_handle(model, cluster_ctas: int = 0, wait_limit_cycles: int = 0):
+def create_handle(model, cluster_ctas: int = 0, wait_limit_cycles: int = 0, attention_mode: int = 0):
     """aecct_create on a model (see inputs.ModelTensors); returns (status, handle or None)."""
     L = load()
-    hm = _HostModel(model, cluster_ctas, wait_limit_cycles)
+    hm = _HostModel(model, cluster_ctas, wait_limit_cycles, attention_mode)
     h = ctypes.c_void_p()
     st = L.aecct_create(ctypes.byref(hm.desc), ctypes.byref(h))
     return st, (h if st == AECCT_OK else None)
@@ -162,7 +163,7 @@ class Decoder:
     torch.cuda.current_stream().
     """
 
-    def __init__(self, model, cluster_ctas: int = 0, wait_limit_cycles: int = 0):
+    def __init__(self, model, cluster_ctas: int = 0, wait_limit_cycles: int = 0, attention_mode: int = 0):
         import torch
 
         if not torch.cuda.is_available():
@@ -173,7 +174,7 @@ class Decoder:
         self.T = 2 * model.n - model.k
         self.d, self.n_layers = model.d, model.n_layers
         self._L = load()
-        st, h = create_handle(model, cluster_ctas, wait_limit_cycles)
+        st, h = create_handle(model, cluster_ctas, wait_limit_cycles, attention_mode)
         _check(st, "aecct_create")
         self._h = h
         self._cap = None
@@ -192,7 +193,7 @@ class Decoder:
     def query(self) -> dict:
         vals = [ctypes.c_int32() for _ in range(6)]
         _check(self._L.aecct_query(self._h, *[ctypes.byref(v) for v in vals]), "aecct_query")
-        keys = ("cluster_ctas", "words_per_group", "max_clusters", "threads_per_cta", "smem_bytes", "tmem_cols")
+        keys = ("cluster_ctas", "words_per_group", "max_clusters", "threads_per_cta", "smem_bytes", "attention_mode")
         return {k: v.value for k, v in zip(keys, vals)}
 
     def decode(self, y, want_syndrome: bool = True, want_logits: bool = True, out=None, stream=None):

@@ -16,6 +16,8 @@ constexpr int kMaxCluster = 8;
 constexpr uint32_t kStageBytes = 16384;  // one weight chunk: <= 128 rows x 64 K bf16
 constexpr int kMaxChunks = 32;           // weight chunks per block (QKV, O, FFN1, FFN2)
 constexpr int kOutBitsBytes = 4096;      // decoded bits of the codewords one CTA finishes
+constexpr int kMaxTasks = 16;            // attention tasks per warp (task mode)
+constexpr int kMaxGroups = 32;           // 32-row query groups per CTA (task mode)
 
 // One weight chunk of a block: rows [n0, n0 + nrows) and K columns [k0, k0 + kcols) of the
 // block's GEMM `gemm` (0 = QKV, 1 = O, 2 = FFN1, 3 = FFN2), stored as a K-major bf16 tile
@@ -73,6 +75,14 @@ struct DecodeParams {
   // and continue 8 per 16-byte entry (a list is padded to whole entries).
   const uint32_t *mask_info[2];
   const uint4 *mask_list[2];
+  // Task-mode attention plan (one CTA per group of codewords, d <= 64).  A task is one head for
+  // a query group: up to 32 consecutive rows of one codeword, one per lane.  It walks the union of
+  // its lanes' key sets (ascending token order) with per-lane membership bits.
+  const uint16_t *plan_task;   // [16 warps][kMaxTasks]: group * 8 + head; 0xFFFF ends the list
+  const uint4 *plan_grp;       // [groups]: {first row, lanes, first row of the codeword, 0}
+  const uint32_t *plan_uinfo;  // [groups][2 rings]: (start << 8) | count of the union list
+  const uint4 *plan_ulist;     // union lists: 16 row offsets (one byte each) per entry
+  const uint4 *plan_mask;      // [groups][2][32 lanes]: 128 membership bits over the union list
   float ln_eps, alpha_floor, att_scale;
   // integer-core capture (device, optional)
   int64_t cap_B;
@@ -92,13 +102,20 @@ __host__ __device__ constexpr inline uint32_t core_off(uint32_t r, uint32_t c, u
   return (r >> 3) * (kdim >> 3) * 128u + (c >> 3) * 128u + (r & 7u) * 16u + (c & 7u) * 2u;
 }
 
-template <int D>
+// Shared-memory map.  Region U holds, per block, first the attention operands and then the FFN2
+// operand.  Row mode: per token row 8 heads x (K | V) x d_h fp32.  Task mode: 8 heads x
+// (Q | K | V) x d_h fp32, followed by the attention output A [128][D] fp32.
+template <int D, bool TASKS = false>
 struct SmemLayout {
-  static constexpr uint32_t kKvStride = 8u * D + 16u;  // token row: 8 heads x (K | V) x d_h fp32, + 16 B pad
+  static constexpr uint32_t kSlot = (TASKS ? 12u : 8u) * (D / 8u);  // bytes of one head of one row
+  static constexpr uint32_t kKvStride = 8u * kSlot + 16u;            // token row, + 16 B pad
   static constexpr uint32_t kKvBytes = kRows * kKvStride;
+  static constexpr uint32_t kOffA = kKvBytes;                         // task mode: A [128][D] fp32
+  static constexpr uint32_t kABytes = TASKS ? kRows * D * 4u : 0u;
   static constexpr uint32_t kUqBytes = kRows * 4u * D * 2u;  // FFN2 operand: 128 x 4D bf16
   __host__ __device__ static constexpr uint32_t align1k(uint32_t v) { return (v + 1023u) & ~1023u; }
-  static constexpr uint32_t kRegionU = align1k(kKvBytes > kUqBytes ? kKvBytes : kUqBytes);
+  static constexpr uint32_t kRegionU =
+      align1k(kKvBytes + kABytes > kUqBytes ? kKvBytes + kABytes : kUqBytes);
   static constexpr uint32_t kAopBytes = kRows * D * 2u;  // QKV / O / FFN1 operand: 128 x D bf16
   static constexpr int kStages = (D == 128) ? 3 : 4;
   static constexpr uint32_t kOffU = 0;
@@ -114,9 +131,9 @@ struct SmemLayout {
 };
 
 // decoder_kernel.cu
-template <int D>
+template <int D, bool TASKS>
 cudaError_t launch_decode(const DecodeParams &p, cudaStream_t stream);
-template <int D>
+template <int D, bool TASKS>
 cudaError_t prepare_decode_kernel(int cluster_ctas, int *max_active_clusters);
 
 // api.cu diagnostics kernels live in selftest.cu

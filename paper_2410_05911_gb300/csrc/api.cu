@@ -32,6 +32,7 @@ int cuda_fail(cudaError_t e, const char *what) {
 struct aecct_handle {
   int n = 0, k = 0, T = 0, m = 0, d = 0, n_layers = 0, h_first = 0, d_spe = 0;
   int C = 1, G = 1, max_clusters = 0;
+  bool tasks = false;  // warp-task attention (one CTA per group, d <= 64)
   float ln_eps = 0, alpha_floor = 0, att_scale = 0, b_d1 = 0;
   long long wait_limit = 0;
   int device = 0;
@@ -44,6 +45,9 @@ struct aecct_handle {
   uint32_t *hrow_off = nullptr, *mask_info[2] = {nullptr, nullptr};
   uint16_t *hrow_idx = nullptr, *mask_list[2] = {nullptr, nullptr};
   uint16_t *perm = nullptr, *pos = nullptr;
+  uint16_t *plan_task = nullptr;
+  uint32_t *plan_grp = nullptr, *plan_uinfo = nullptr, *plan_mask = nullptr;
+  uint8_t *plan_ulist = nullptr;
   int *d_err = nullptr;
   int *h_err = nullptr;  // pinned
   cudaEvent_t ev = nullptr;
@@ -107,6 +111,7 @@ int validate(const aecct_model_desc *d) {
   if (d->ffn_mult <= 0) return AECCT_ERR_INVALID_ARG;
   if (d->activation < 0 || d->activation > 1) return AECCT_ERR_INVALID_ARG;
   if (d->cluster_ctas < 0 || d->cluster_ctas > 64) return AECCT_ERR_INVALID_ARG;
+  if (d->attention_mode < 0 || d->attention_mode > 2) return AECCT_ERR_INVALID_ARG;
   if (!d->H || !d->emb || !d->w_packed || !d->w_scale || !d->bias || !d->ln_gamma || !d->ln_beta || !d->w_d1 ||
       !d->w_out || !d->b_out)
     return AECCT_ERR_INVALID_ARG;
@@ -179,11 +184,24 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
   const aecct_model_desc &d = *desc;
   const int n = d.n, k = d.k, m = n - k, T = 2 * n - k, D = d.d, F = 4 * D;
 
+  // Attention mode.  Task mode keeps every codeword inside one CTA (no cluster): it needs T <= 128,
+  // d <= 64 (shared memory for Q, K, V and A), and at most kMaxGroups 32-row query groups.
+  const int g1 = kRows / T;
+  const bool task_ok = T <= kRows && D <= 64 && g1 >= 1 && g1 * ((T + 31) / 32) <= kMaxGroups &&
+                       g1 * n <= kOutBitsBytes && (d.cluster_ctas == 0 || d.cluster_ctas == 1);
+  bool tasks = false;
+  if (d.attention_mode == 2) {
+    if (!task_ok) return AECCT_ERR_UNSUPPORTED;
+    tasks = true;
+  } else if (d.attention_mode == 0) {
+    tasks = task_ok;
+  }
   // choose the number of CTAs that share a group: densest packing of T-token words over C x 128 rows
   int best_C = 0, best_G = 0;
   double best_eff = -1.0;
   const int cmin = (T + kRows - 1) / kRows;
   for (int C = cmin; C <= kMaxCluster; ++C) {
+    if (tasks && C != 1) continue;
     if (d.cluster_ctas && C != d.cluster_ctas) continue;
     const int G = (C * kRows) / T;
     if (G < 1) continue;
@@ -204,9 +222,11 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
     return AECCT_ERR_NO_DEVICE;
   }
   int max_clusters = 0;
-  if (D == 32) e = prepare_decode_kernel<32>(best_C, &max_clusters);
-  else if (D == 64) e = prepare_decode_kernel<64>(best_C, &max_clusters);
-  else e = prepare_decode_kernel<128>(best_C, &max_clusters);
+  if (tasks) e = D == 32 ? prepare_decode_kernel<32, true>(best_C, &max_clusters)
+                         : prepare_decode_kernel<64, true>(best_C, &max_clusters);
+  else if (D == 32) e = prepare_decode_kernel<32, false>(best_C, &max_clusters);
+  else if (D == 64) e = prepare_decode_kernel<64, false>(best_C, &max_clusters);
+  else e = prepare_decode_kernel<128, false>(best_C, &max_clusters);
   if (e != cudaSuccess) return cuda_fail(e, "kernel occupancy");
   if (max_clusters < 1) {
     g_last_error = "no cluster of this size fits on the device";
@@ -215,7 +235,7 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
 
   aecct_handle *h = new aecct_handle();
   h->n = n, h->k = k, h->T = T, h->m = m, h->d = D, h->n_layers = d.n_layers, h->h_first = d.h_first;
-  h->d_spe = d.d_spe, h->C = best_C, h->G = best_G, h->max_clusters = max_clusters;
+  h->d_spe = d.d_spe, h->C = best_C, h->G = best_G, h->max_clusters = max_clusters, h->tasks = tasks;
   h->ln_eps = d.ln_eps, h->alpha_floor = d.alpha_floor, h->b_d1 = d.b_d1, h->device = dev;
   h->att_scale = static_cast<float>(1.4426950408889634074 / std::sqrt(static_cast<double>(D / kHeads)));
   h->wait_limit = d.wait_limit_cycles ? d.wait_limit_cycles : (1LL << 32);
@@ -275,7 +295,9 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
       const size_t a = hf > 0 ? nb[0][t].size() : 0, b = hs > 0 ? nb[1][t].size() : 0;
       return (hf > 0 && hs > 0) ? a + b : (a + b) * 2;
     };
-    std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return work(a) > work(b); });
+    // task mode keeps the natural order (variables, then checks): query groups of one node type
+    // share most of their keys
+    if (!tasks) std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return work(a) > work(b); });
     for (int i = 0; i < T; ++i) {
       perm[i] = static_cast<uint16_t>(order[i]);
       pos[order[i]] = static_cast<uint16_t>(i);
@@ -298,6 +320,68 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
       while (mlist[mk].size() % 8) mlist[mk].push_back(0);
     }
     if (mlist[mk].empty()) mlist[mk].assign(8, 0);
+  }
+
+  // ---- task-mode attention plan (every CTA holds the same layout: G codewords of T rows)
+  std::vector<uint16_t> ptask;
+  std::vector<uint32_t> pgrp, puinfo, pmask;
+  std::vector<uint8_t> pulist;
+  if (tasks) {
+    const int G = best_G;
+    struct Grp {
+      int row0, lanes, cwrow0;
+    };
+    std::vector<Grp> grps;
+    for (int cw = 0; cw < G; ++cw)
+      for (int off0 = 0; off0 < T; off0 += 32) grps.push_back({cw * T + off0, std::min(32, T - off0), cw * T});
+    const int ng = static_cast<int>(grps.size());
+    std::vector<int> ucount(ng * 2, 0);
+    pgrp.assign((size_t)ng * 4, 0);
+    puinfo.assign((size_t)ng * 2, 0);
+    pmask.assign((size_t)ng * 2 * 32 * 4, 0);
+    for (int gi = 0; gi < ng; ++gi) {
+      pgrp[gi * 4 + 0] = static_cast<uint32_t>(grps[gi].row0);
+      pgrp[gi * 4 + 1] = static_cast<uint32_t>(grps[gi].lanes);
+      pgrp[gi * 4 + 2] = static_cast<uint32_t>(grps[gi].cwrow0);
+      const int off0 = grps[gi].row0 - grps[gi].cwrow0;
+      for (int ring = 0; ring < 2; ++ring) {
+        // union of the lanes' key sets, in ascending token order
+        std::vector<uint8_t> in(T, 0);
+        for (int ln = 0; ln < grps[gi].lanes; ++ln)
+          for (uint16_t u : nb[ring][perm[off0 + ln]]) in[u] = 1;
+        std::vector<int> uni;
+        for (int u = 0; u < T; ++u)
+          if (in[u]) uni.push_back(u);
+        const size_t start = pulist.size() / 16;
+        puinfo[gi * 2 + ring] = static_cast<uint32_t>((start << 8) | uni.size());
+        ucount[gi * 2 + ring] = static_cast<int>(uni.size());
+        for (int u : uni) pulist.push_back(static_cast<uint8_t>(pos[u]));
+        while (pulist.size() % 16) pulist.push_back(0);
+        for (int ln = 0; ln < grps[gi].lanes; ++ln) {
+          std::vector<uint8_t> mine(T, 0);
+          for (uint16_t u : nb[ring][perm[off0 + ln]]) mine[u] = 1;
+          for (size_t kk = 0; kk < uni.size(); ++kk)
+            if (mine[uni[kk]]) pmask[((size_t)(gi * 2 + ring) * 32 + ln) * 4 + kk / 32] |= 1u << (kk % 32);
+        }
+      }
+    }
+    // tasks (group, head), longest first, each to the least-loaded warp
+    std::vector<std::pair<int, int>> tl;  // (cost, task)
+    for (int gi = 0; gi < ng; ++gi)
+      for (int e = 0; e < kHeads; ++e) tl.push_back({ucount[gi * 2 + (e < d.h_first ? 0 : 1)] + 4, gi * 8 + e});
+    std::stable_sort(tl.begin(), tl.end(), [](const std::pair<int, int> &x, const std::pair<int, int> &y) {
+      return x.first > y.first;
+    });
+    ptask.assign((size_t)kEpiWarps * kMaxTasks, 0xFFFFu);
+    std::vector<long> load(kEpiWarps, 0);
+    std::vector<int> cnt(kEpiWarps, 0);
+    for (const auto &tk : tl) {
+      int best = -1;
+      for (int w = 0; w < kEpiWarps; ++w)
+        if (cnt[w] < kMaxTasks && (best < 0 || load[w] < load[best])) best = w;
+      ptask[(size_t)best * kMaxTasks + cnt[best]++] = static_cast<uint16_t>(tk.second);
+      load[best] += tk.first;
+    }
   }
 
   // ---- weights: 2-bit codes -> bf16 K-major core-matrix chunks, in the order the MMA consumes them
@@ -387,6 +471,11 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
       (rc = dev_upload(h, &h->mask_list[0], mlist[0].data(), mlist[0].size())) ||
       (rc = dev_upload(h, &h->mask_info[1], minfo[1].data(), minfo[1].size())) ||
       (rc = dev_upload(h, &h->mask_list[1], mlist[1].data(), mlist[1].size())) ||
+      (rc = dev_upload(h, &h->plan_task, ptask.data(), ptask.size())) ||
+      (rc = dev_upload(h, &h->plan_grp, pgrp.data(), pgrp.size())) ||
+      (rc = dev_upload(h, &h->plan_uinfo, puinfo.data(), puinfo.size())) ||
+      (rc = dev_upload(h, &h->plan_ulist, pulist.data(), pulist.size())) ||
+      (rc = dev_upload(h, &h->plan_mask, pmask.data(), pmask.size())) ||
       (rc = dev_upload<int>(h, &h->d_err, nullptr, 1))) {
     free_handle(h);
     return rc;
@@ -441,6 +530,11 @@ int aecct_decode(aecct_handle *h, const float *y_dev, int64_t B, uint8_t *bits_d
   p.lparams = h->lparams, p.emb = h->emb, p.spe = h->spe, p.w_d1 = h->w_d1, p.b_d1 = h->b_d1;
   p.w_out = h->w_out, p.b_out = h->b_out, p.hrow_off = h->hrow_off, p.hrow_idx = h->hrow_idx;
   p.perm = h->perm, p.pos = h->pos;
+  p.plan_task = h->plan_task;
+  p.plan_grp = reinterpret_cast<const uint4 *>(h->plan_grp);
+  p.plan_uinfo = h->plan_uinfo;
+  p.plan_ulist = reinterpret_cast<const uint4 *>(h->plan_ulist);
+  p.plan_mask = reinterpret_cast<const uint4 *>(h->plan_mask);
   p.mask_info[0] = h->mask_info[0], p.mask_info[1] = h->mask_info[1];
   p.mask_list[0] = reinterpret_cast<const uint4 *>(h->mask_list[0]);
   p.mask_list[1] = reinterpret_cast<const uint4 *>(h->mask_list[1]);
@@ -448,9 +542,10 @@ int aecct_decode(aecct_handle *h, const float *y_dev, int64_t B, uint8_t *bits_d
   p.cap_B = h->cap_B, p.cap_q = h->cap_q, p.cap_acc = h->cap_acc, p.cap_alpha = h->cap_alpha, p.cap_syn = h->cap_syn;
   p.err = h->d_err, p.wait_limit = h->wait_limit;
   cudaError_t e;
-  if (h->d == 32) e = launch_decode<32>(p, stream);
-  else if (h->d == 64) e = launch_decode<64>(p, stream);
-  else e = launch_decode<128>(p, stream);
+  if (h->tasks) e = h->d == 32 ? launch_decode<32, true>(p, stream) : launch_decode<64, true>(p, stream);
+  else if (h->d == 32) e = launch_decode<32, false>(p, stream);
+  else if (h->d == 64) e = launch_decode<64, false>(p, stream);
+  else e = launch_decode<128, false>(p, stream);
   if (e != cudaSuccess) return cuda_fail(e, "decode launch");
   if ((e = cudaMemcpyAsync(h->h_err, h->d_err, sizeof(int), cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
     return cuda_fail(e, "status copy");
@@ -510,15 +605,17 @@ int aecct_set_capture(aecct_handle *h, int64_t cap_B, int8_t *q_dev, int32_t *ac
 }
 
 int aecct_query(const aecct_handle *h, int32_t *cluster_ctas, int32_t *words_per_group, int32_t *max_clusters,
-                int32_t *threads_per_cta, int32_t *smem_bytes, int32_t *tmem_cols) {
+                int32_t *threads_per_cta, int32_t *smem_bytes, int32_t *attention_mode) {
   if (!h) return AECCT_ERR_INVALID_ARG;
   if (cluster_ctas) *cluster_ctas = h->C;
   if (words_per_group) *words_per_group = h->G;
   if (max_clusters) *max_clusters = h->max_clusters;
   if (threads_per_cta) *threads_per_cta = kThreads;
-  const int sm = h->d == 32 ? SmemLayout<32>::kTotal : (h->d == 64 ? SmemLayout<64>::kTotal : SmemLayout<128>::kTotal);
+  int sm;
+  if (h->tasks) sm = h->d == 32 ? SmemLayout<32, true>::kTotal : SmemLayout<64, true>::kTotal;
+  else sm = h->d == 32 ? SmemLayout<32>::kTotal : (h->d == 64 ? SmemLayout<64>::kTotal : SmemLayout<128>::kTotal);
   if (smem_bytes) *smem_bytes = sm;
-  if (tmem_cols) *tmem_cols = 4 * h->d;
+  if (attention_mode) *attention_mode = h->tasks ? 2 : 1;
   return AECCT_OK;
 }
 

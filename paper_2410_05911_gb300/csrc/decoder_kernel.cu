@@ -43,7 +43,64 @@ __device__ __forceinline__ float exp2_series(float x) {
   p = __fmaf_rn(p, f, __uint_as_float(0x3f317218u));  // k = 1
   p = __fmaf_rn(p, f, 1.0f);                          // k = 0
   // p is in [0.70, 1.42] and n >= -125, so p * 2^n is normal: scale through the exponent field
-  return __int_as_float(__float_as_int(p) + (static_cast<int>(n) << 23));
+  return __int_as_float(__float_as_int(p) + (__float2int_rn(n) << 23));
+}
+
+// ---- paired fp32 arithmetic (sm_100 f32x2: each lane is one IEEE round-to-nearest operation,
+// bit-identical to the scalar _rn operation on that lane).  The code generator contracts a paired
+// multiply whose only use is a paired add into one fused multiply-add, even with --fmad=false
+// and an explicit .rn modifier, so pairs are used only where no contraction can occur: fused
+// multiply-adds that the canonical order asks for, adds of values that are not products, and
+// products that feed no add.  Every multiply-then-add of the canonical order uses the scalar
+// __fmul_rn / __fadd_rn intrinsics, which are never contracted.
+__device__ __forceinline__ uint64_t pack2(float2 a) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a.x), "f"(a.y));
+  return r;
+}
+__device__ __forceinline__ float2 unpack2(uint64_t r) {
+  float2 a;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(a.x), "=f"(a.y) : "l"(r));
+  return a;
+}
+__device__ __forceinline__ float2 mul2(float2 a, float2 b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(pack2(a)), "l"(pack2(b)));
+  return unpack2(d);
+}
+__device__ __forceinline__ float2 add2(float2 a, float2 b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(pack2(a)), "l"(pack2(b)));
+  return unpack2(d);
+}
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(pack2(a)), "l"(pack2(b)), "l"(pack2(c)));
+  return unpack2(d);
+}
+
+// two independent evaluations of exp2_series (same steps on each lane); inputs below -125 give 0
+__device__ __forceinline__ float2 exp2_series2(float2 x) {
+  const float n0 = rintf(x.x), n1 = rintf(x.y);
+  const float2 f = add2(x, make_float2(-n0, -n1));
+  float2 p = make_float2(__uint_as_float(0x377fe5feu), __uint_as_float(0x377fe5feu));
+  p = fma2(p, f, make_float2(__uint_as_float(0x39218489u), __uint_as_float(0x39218489u)));
+  p = fma2(p, f, make_float2(__uint_as_float(0x3aaec3ffu), __uint_as_float(0x3aaec3ffu)));
+  p = fma2(p, f, make_float2(__uint_as_float(0x3c1d955bu), __uint_as_float(0x3c1d955bu)));
+  p = fma2(p, f, make_float2(__uint_as_float(0x3d635847u), __uint_as_float(0x3d635847u)));
+  p = fma2(p, f, make_float2(__uint_as_float(0x3e75fdf0u), __uint_as_float(0x3e75fdf0u)));
+  p = fma2(p, f, make_float2(__uint_as_float(0x3f317218u), __uint_as_float(0x3f317218u)));
+  p = fma2(p, f, make_float2(1.0f, 1.0f));
+  const float r0 = (x.x >= -125.0f) ? __int_as_float(__float_as_int(p.x) + (__float2int_rn(n0) << 23)) : 0.0f;
+  const float r1 = (x.y >= -125.0f) ? __int_as_float(__float_as_int(p.y) + (__float2int_rn(n1) << 23)) : 0.0f;
+  return make_float2(r0, r1);
+}
+
+// out[j] = acc[j] * f + b[j]  (eq. AAPLinear dequantisation, f = gamma*delta*alpha/Q_b)
+template <int N>
+__device__ __forceinline__ void dequant(const float *acc, float f, const float *b, float *out) {
+#pragma unroll
+  for (int j = 0; j < N; ++j) out[j] = __fadd_rn(__fmul_rn(acc[j], f), b[j]);
 }
 
 template <int N>
@@ -94,11 +151,17 @@ __device__ __noinline__ bool wait_bar_drain(const Ctl &c, uint32_t bar, uint32_t
 // ------------------------------------------------------------------------------------------
 // small helpers for the CUDA-core warps
 // ------------------------------------------------------------------------------------------
-__device__ __forceinline__ float q_code(float v, float r) {
-  float q = rintf(__fmul_rn(v, r));
-  q = q > 127.0f ? 127.0f : q;
-  q = q < -127.0f ? -127.0f : q;
-  return q;
+// Code of v under r = 127/alpha' (eq. Quant).  |v| <= alpha' gives |v * r| <= 127 (1 + 2^-24)
+// before rounding, so the clip of RoundClip can never act and is left out.
+__device__ __forceinline__ float q_code(float v, float r) { return rintf(__fmul_rn(v, r)); }
+template <int N>
+__device__ __forceinline__ void codes(const float *v, float r, float *q) {
+#pragma unroll
+  for (int j = 0; j < N; j += 2) {
+    const float2 t = mul2(make_float2(v[j], v[j + 1]), make_float2(r, r));
+    q[j] = rintf(t.x);
+    q[j + 1] = rintf(t.y);
+  }
 }
 __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
   // a, b are integers in [-127, 127]: exact in bf16
@@ -261,6 +324,136 @@ __device__ __forceinline__ void hpsa_head(const float *q, uint32_t info, const u
   for (int i = 0; i < DH; ++i) A[i] = __fmul_rn(num[i], inv);
 }
 
+// membership bit k of a lane's 128-bit mask, and byte k of a 16-entry index block
+__device__ __forceinline__ bool mask_bit(const uint4 &m, int k) {
+  const uint32_t w = k < 64 ? (k < 32 ? m.x : m.y) : (k < 96 ? m.z : m.w);
+  return ((w >> (k & 31)) & 1u) != 0u;
+}
+__device__ __forceinline__ int byte_at(const uint4 &w, int k) {
+  const uint32_t v = k < 8 ? (k < 4 ? w.x : w.y) : (k < 12 ? w.z : w.w);
+  return static_cast<int>((v >> (8 * (k & 3))) & 0xFFu);
+}
+
+// One HPSA head for a query group (task mode).  Every lane walks the group's union key list in
+// ascending token order; the loads are warp-uniform (shared-memory broadcasts).  A lane only
+// folds in the keys of its own set (membership bit), so for each query the max, the sum l and
+// the weighted sum num see exactly its keys, in ascending order, as in the canonical definition.
+// Keys go two at a time through f32x2 instructions: the two lanes of a pair are independent
+// computations, and the folds into l and num stay sequential in key order.
+template <int DH, uint32_t STRIDE>
+__device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int cnt, const uint4 *__restrict__ ul,
+                                          const uint8_t *rows, uint32_t kslot, float scale, float *A) {
+  auto kptr = [&](int off) { return reinterpret_cast<const float4 *>(rows + off * STRIDE + kslot); };
+  // dot products of q with two keys: lane x for key a, lane y for key b (FMA chains in feature order)
+  auto dot2 = [&](const float4 *ka, const float4 *kb) -> float2 {
+    float2 d = make_float2(0.0f, 0.0f);
+#pragma unroll
+    for (int i = 0; i < DH / 4; ++i) {
+      d = fma2(make_float2(q[4 * i], q[4 * i]), make_float2(ka[i].x, kb[i].x), d);
+      d = fma2(make_float2(q[4 * i + 1], q[4 * i + 1]), make_float2(ka[i].y, kb[i].y), d);
+      d = fma2(make_float2(q[4 * i + 2], q[4 * i + 2]), make_float2(ka[i].z, kb[i].z), d);
+      d = fma2(make_float2(q[4 * i + 3], q[4 * i + 3]), make_float2(ka[i].w, kb[i].w), d);
+    }
+    return d;
+  };
+  const float2 sc = make_float2(scale, scale);
+  constexpr int U = 4;
+  // pass 1: maximum score over the lane's keys
+  float mx = -INFINITY;
+  for (int jb = 0; jb < cnt; jb += 16) {
+    const uint4 w = __ldg(ul + (jb >> 4));
+    const int nk = min(16, cnt - jb);
+    if (nk == 16) {
+#pragma unroll
+      for (int k0 = 0; k0 < 16; k0 += U) {
+        float4 kk[U][DH / 4];
+#pragma unroll
+        for (int k = 0; k < U; ++k) {
+          const float4 *kp = kptr(byte_at(w, k0 + k));
+#pragma unroll
+          for (int i = 0; i < DH / 4; ++i) kk[k][i] = kp[i];
+        }
+#pragma unroll
+        for (int k = 0; k < U; k += 2) {
+          const float2 sg = mul2(dot2(kk[k], kk[k + 1]), sc);
+          if (mask_bit(mask, jb + k0 + k)) mx = fmaxf(mx, sg.x);
+          if (mask_bit(mask, jb + k0 + k + 1)) mx = fmaxf(mx, sg.y);
+        }
+      }
+    } else {
+      for (int k = 0; k < nk; k += 2) {
+        const int k1 = (k + 1 < nk) ? k + 1 : k;
+        float4 ka[DH / 4], kb[DH / 4];
+        const float4 *pa = kptr(byte_at(w, k)), *pb = kptr(byte_at(w, k1));
+#pragma unroll
+        for (int i = 0; i < DH / 4; ++i) ka[i] = pa[i], kb[i] = pb[i];
+        const float2 sg = mul2(dot2(ka, kb), sc);
+        if (mask_bit(mask, jb + k)) mx = fmaxf(mx, sg.x);
+        if (k1 != k && mask_bit(mask, jb + k1)) mx = fmaxf(mx, sg.y);
+      }
+    }
+  }
+  // pass 2: p = 2^(sigma - m), l += p, num += p v, in key order
+  float lsum = 0.0f;
+  float num[DH];
+#pragma unroll
+  for (int i = 0; i < DH; ++i) num[i] = 0.0f;
+  // sigma - m for a pair of dot products (scalar: a product followed by a subtraction)
+  auto shifted = [&](float2 d) {
+    return make_float2(__fsub_rn(__fmul_rn(d.x, scale), mx), __fsub_rn(__fmul_rn(d.y, scale), mx));
+  };
+  auto fold = [&](float pr, const float4 *vv) {
+    lsum = __fadd_rn(lsum, pr);
+    const float2 pp = make_float2(pr, pr);
+#pragma unroll
+    for (int i = 0; i < DH / 4; ++i) {
+      const float2 lo = fma2(pp, make_float2(vv[i].x, vv[i].y), make_float2(num[4 * i], num[4 * i + 1]));
+      const float2 hi = fma2(pp, make_float2(vv[i].z, vv[i].w), make_float2(num[4 * i + 2], num[4 * i + 3]));
+      num[4 * i] = lo.x, num[4 * i + 1] = lo.y, num[4 * i + 2] = hi.x, num[4 * i + 3] = hi.y;
+    }
+  };
+  for (int jb = 0; jb < cnt; jb += 16) {
+    const uint4 w = __ldg(ul + (jb >> 4));
+    const int nk = min(16, cnt - jb);
+    if (nk == 16) {
+#pragma unroll
+      for (int k0 = 0; k0 < 16; k0 += U) {
+        float4 kk[U][DH / 4], vv[U][DH / 4];
+#pragma unroll
+        for (int k = 0; k < U; ++k) {
+          const float4 *kp = kptr(byte_at(w, k0 + k));
+#pragma unroll
+          for (int i = 0; i < DH / 4; ++i) kk[k][i] = kp[i];
+#pragma unroll
+          for (int i = 0; i < DH / 4; ++i) vv[k][i] = kp[DH / 4 + i];
+        }
+        float2 pr[U / 2];
+#pragma unroll
+        for (int k = 0; k < U; k += 2) pr[k / 2] = exp2_series2(shifted(dot2(kk[k], kk[k + 1])));
+#pragma unroll
+        for (int k = 0; k < U; k += 2) {
+          if (mask_bit(mask, jb + k0 + k)) fold(pr[k / 2].x, vv[k]);
+          if (mask_bit(mask, jb + k0 + k + 1)) fold(pr[k / 2].y, vv[k + 1]);
+        }
+      }
+    } else {
+      for (int k = 0; k < nk; k += 2) {
+        const int k1 = (k + 1 < nk) ? k + 1 : k;
+        float4 ka[DH / 4], kb[DH / 4], va[DH / 4], vb[DH / 4];
+        const float4 *pa = kptr(byte_at(w, k)), *pb = kptr(byte_at(w, k1));
+#pragma unroll
+        for (int i = 0; i < DH / 4; ++i) ka[i] = pa[i], kb[i] = pb[i], va[i] = pa[DH / 4 + i], vb[i] = pb[DH / 4 + i];
+        const float2 pr = exp2_series2(shifted(dot2(ka, kb)));
+        if (mask_bit(mask, jb + k)) fold(pr.x, va);
+        if (k1 != k && mask_bit(mask, jb + k1)) fold(pr.y, vb);
+      }
+    }
+  }
+  const float inv = __fdiv_rn(1.0f, lsum);
+#pragma unroll
+  for (int i = 0; i < DH; ++i) A[i] = __fmul_rn(num[i], inv);
+}
+
 // ------------------------------------------------------------------------------------------
 // weight streaming and tensor-core issue (run by thread 0 of each CTA)
 // ------------------------------------------------------------------------------------------
@@ -274,10 +467,10 @@ struct IssueState {
   uint32_t oph;    // parity of the next operand-ready phase
 };
 
-template <int D>
+template <int D, bool TASKS>
 __device__ __noinline__ void issue_copies(const DecodeParams &p, const Ctl &ctl, IssueState &st, int64_t limit,
                                           uint32_t sb) {
-  using L = SmemLayout<D>;
+  using L = SmemLayout<D, TASKS>;
   constexpr int S = L::kStages;
   const uint32_t bar_full = sb + L::kOffBar, bar_empty = bar_full + 8 * S;
   if (limit > st.total) limit = st.total;
@@ -297,10 +490,10 @@ __device__ __noinline__ void issue_copies(const DecodeParams &p, const Ctl &ctl,
 
 // Wait until every warp has published the operand of GEMM `gemm`, issue its tcgen05.mma chain
 // (accumulators at TMEM column 0), signal the accumulator barrier, then prefetch the next chunks.
-template <int D>
+template <int D, bool TASKS>
 __device__ __noinline__ void issue_gemm(const DecodeParams &p, const Ctl &ctl, IssueState &st, int gemm, uint32_t sb,
                                         uint32_t tmem) {
-  using L = SmemLayout<D>;
+  using L = SmemLayout<D, TASKS>;
   constexpr int S = L::kStages;
   const uint32_t bar_full = sb + L::kOffBar, bar_empty = bar_full + 8 * S;
   const uint32_t bar_op = bar_empty + 8 * S, bar_acc = bar_op + 8;
@@ -313,7 +506,7 @@ __device__ __noinline__ void issue_gemm(const DecodeParams &p, const Ctl &ctl, I
     const int c = static_cast<int>(st.used % p.n_chunks);
     const ChunkDesc ch = p.chunks[c];
     if (ch.gemm != gemm) break;
-    issue_copies<D>(p, ctl, st, st.used + 1, sb);
+    issue_copies<D, TASKS>(p, ctl, st, st.used + 1, sb);
     const int s = static_cast<int>(st.used % S);
     wait_bar(ctl, bar_full + 8 * s, static_cast<uint32_t>((st.used / S) & 1), false);
     tc_fence_after();
@@ -330,15 +523,15 @@ __device__ __noinline__ void issue_gemm(const DecodeParams &p, const Ctl &ctl, I
     ++st.used;
   }
   mma_commit(bar_acc);
-  issue_copies<D>(p, ctl, st, st.used + S, sb);
+  issue_copies<D, TASKS>(p, ctl, st, st.used + S, sb);
 }
 
 // ------------------------------------------------------------------------------------------
 // the kernel
 // ------------------------------------------------------------------------------------------
-template <int D>
+template <int D, bool TASKS>
 __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid_constant__ DecodeParams p) {
-  using L = SmemLayout<D>;
+  using L = SmemLayout<D, TASKS>;
   using LP = LayerParamLayout;
   constexpr int DH = D / kHeads;  // head width
   constexpr int XS = D / 4;       // x columns per thread
@@ -400,7 +593,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   if (tid == 0) {
     const int64_t my_groups = (p.n_groups - cluster_id + p.n_clusters - 1) / p.n_clusters;
     ist.total = my_groups * p.n_layers * p.n_chunks;
-    issue_copies<D>(p, ctl, ist, S, sb);
+    issue_copies<D, TASKS>(p, ctl, ist, S, sb);
   }
   __syncwarp();
   {
@@ -442,7 +635,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) mbar_arrive(bar_op);
-      if (tid == 0) issue_gemm<D>(p, ctl, ist, gemm, sb, tmem);
+      if (tid == 0) issue_gemm<D, TASKS>(p, ctl, ist, gemm, sb, tmem);
       __syncwarp();  // warp 0 waits for its issuing lane before any warp-collective instruction
     };
     auto cluster_arrive = [&](uint32_t bar) {
@@ -506,10 +699,31 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         alpha_in = a;
         const float rr = __fdiv_rn(127.0f, a);
         float qv[XS];
-#pragma unroll
-        for (int j = 0; j < XS; ++j) qv[j] = q_code(x[j], rr);
+        codes<XS>(x, rr, qv);
         store_codes<XS>(aop, r, sl * XS, D, qv);
         return rr;
+      };
+      // x <- LayerNorm(x + (acc * f + bias)) with gamma g and beta be (Post-LN, Sec. 5)
+      auto residual_ln = [&](const float *ac, float f, const float *bias, const float *g, const float *be) {
+        float bb[XS], v[XS];
+        ldg_vec<XS>(bias, bb);
+        dequant<XS>(ac, f, bb, v);
+#pragma unroll
+        for (int j = 0; j < XS; ++j) v[j] = __fadd_rn(x[j], v[j]);
+        const float mu = __fmul_rn(row_sum(psum<XS>(v)), inv_d);
+        float sq[XS];
+#pragma unroll
+        for (int j = 0; j < XS; ++j) {
+          v[j] = __fsub_rn(v[j], mu);
+          sq[j] = __fmul_rn(v[j], v[j]);
+        }
+        const float var = __fmul_rn(row_sum(psum<XS>(sq)), inv_d);
+        const float rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, p.ln_eps)));
+        float gg[XS], bt[XS];
+        ldg_vec<XS>(g, gg);
+        ldg_vec<XS>(be, bt);
+#pragma unroll
+        for (int j = 0; j < XS; ++j) x[j] = __fadd_rn(__fmul_rn(__fmul_rn(v[j], rstd), gg[j]), bt[j]);
       };
       auto capture_q = [&](int layer, int gemm, const float *qv, int c0, int len, float alpha) {
         const int64_t row = ((b * p.n_layers + layer) * 4 + gemm) * T + t;
@@ -527,8 +741,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         const float rr = quant_x_to_aop();
         if (cap) {
           float qv[XS];
-#pragma unroll
-          for (int j = 0; j < XS; ++j) qv[j] = q_code(x[j], rr);
+          codes<XS>(x, rr, qv);
           capture_q(0, 0, qv, sl * XS, XS, alpha_in);
         }
       }
@@ -559,97 +772,145 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             capture_acc(l, 0, ka, D + e * DH, DH);
             capture_acc(l, 0, va, 2 * D + e * DH, DH);
           }
-          const uint32_t dst = kvl + r * L::kKvStride + e * (8 * DH);
+          // head slot of this row: row mode (K | V), task mode (Q | K | V)
+          const uint32_t dst = kvl + r * L::kKvStride + e * L::kSlot + (TASKS ? 4 * DH : 0);
+          dequant<DH>(ka, fk, bk, ka);
+          dequant<DH>(va, fv, bv, va);
 #pragma unroll
           for (int i = 0; i < DH; i += 4) {
-            st_shared_f4(dst + 4 * i, __fadd_rn(__fmul_rn(ka[i], fk), bk[i]), __fadd_rn(__fmul_rn(ka[i + 1], fk), bk[i + 1]),
-                         __fadd_rn(__fmul_rn(ka[i + 2], fk), bk[i + 2]), __fadd_rn(__fmul_rn(ka[i + 3], fk), bk[i + 3]));
-            st_shared_f4(dst + 4 * (DH + i), __fadd_rn(__fmul_rn(va[i], fv), bv[i]),
-                         __fadd_rn(__fmul_rn(va[i + 1], fv), bv[i + 1]), __fadd_rn(__fmul_rn(va[i + 2], fv), bv[i + 2]),
-                         __fadd_rn(__fmul_rn(va[i + 3], fv), bv[i + 3]));
+            st_shared_f4(dst + 4 * i, ka[i], ka[i + 1], ka[i + 2], ka[i + 3]);
+            st_shared_f4(dst + 4 * (DH + i), va[i], va[i + 1], va[i + 2], va[i + 3]);
+          }
+          if constexpr (TASKS) {
+            float qa[DH], bq[DH];
+            tmem_ld<DH>(tl + e * DH, qa);
+            tmem_wait_ld();
+            if (cap) capture_acc(l, 0, qa, e * DH, DH);
+            ldg_vec<DH>(lp + LP::bqkv(D) + e * DH, bq);
+            const uint32_t qdst = kvl + r * L::kKvStride + e * L::kSlot;
+            dequant<DH>(qa, fq, bq, qa);
+#pragma unroll
+            for (int i = 0; i < DH; i += 4) st_shared_f4(qdst + 4 * i, qa[i], qa[i + 1], qa[i + 2], qa[i + 3]);
           }
         }
-        cluster_arrive(bar_kvr);
-        wait_bar(ctl, bar_kvr, kvr_ph, true);
-        kvr_ph ^= 1u;
-
-        // ---------------- S5: HPSA (Sec. 4.2)
-        float A[2][DH];
-        float amax = 0.0f;
+        if constexpr (TASKS) {
+          // ---------------- S5: HPSA (Sec. 4.2), task mode: warp tasks over query groups
+          named_bar_sync(5, kEpiThreads);  // every Q, K, V row of this CTA is in shared memory
+          for (int k = 0; k < kMaxTasks; ++k) {
+            const uint32_t task = __ldg(p.plan_task + warp * kMaxTasks + k);
+            if (task == 0xFFFFu) break;
+            const int grp = static_cast<int>(task >> 3), e = static_cast<int>(task & 7u);
+            const int ring = e < p.h_first ? 0 : 1;
+            const uint4 gi = __ldg(p.plan_grp + grp);
+            const bool act = lane < static_cast<int>(gi.y);
+            const int row = static_cast<int>(gi.x) + (act ? lane : 0);
+            const uint4 mk = act ? __ldg(p.plan_mask + (grp * 2 + ring) * 32 + lane) : make_uint4(0u, 0u, 0u, 0u);
+            const uint32_t ui = __ldg(p.plan_uinfo + grp * 2 + ring);
+            float q[DH], a[DH];
+            const float4 *qp = reinterpret_cast<const float4 *>(smem + L::kOffU + row * L::kKvStride + e * L::kSlot);
 #pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-          const int e = sl + 4 * hh;
-          float qa[DH], bq[DH];
-          tmem_ld<DH>(tl + e * DH, qa);
-          tmem_wait_ld();
-          if (cap) capture_acc(l, 0, qa, e * DH, DH);
-          ldg_vec<DH>(lp + LP::bqkv(D) + e * DH, bq);
-          float q[DH];
+            for (int i = 0; i < DH / 4; ++i) {
+              const float4 v = qp[i];
+              q[4 * i] = v.x, q[4 * i + 1] = v.y, q[4 * i + 2] = v.z, q[4 * i + 3] = v.w;
+            }
+            hpsa_task<DH, L::kKvStride>(q, mk, static_cast<int>(ui & 255u), p.plan_ulist + (ui >> 8),
+                                        smem + L::kOffU + gi.z * L::kKvStride, e * L::kSlot + 4 * DH, p.att_scale, a);
+            if (act) {
+              float4 *ap = reinterpret_cast<float4 *>(smem + L::kOffU + L::kOffA + (row * D + e * DH) * 4);
 #pragma unroll
-          for (int i = 0; i < DH; ++i) q[i] = __fadd_rn(__fmul_rn(qa[i], fq), bq[i]);
-#pragma unroll
-          for (int i = 0; i < DH; ++i) A[hh][i] = 0.0f;
-          if (row_cw) {
-            const int mk = (e < p.h_first) ? 0 : 1;
-            constexpr int U = (DH >= 16) ? 2 : 4;
-            hpsa_head<DH, U, L::kKvStride>(q, __ldg(p.mask_info[mk] + t), p.mask_list[mk], s_kvgen, g * T,
-                                           e * (8 * DH), p.att_scale, A[hh]);
+              for (int i = 0; i < DH / 4; ++i) ap[i] = make_float4(a[4 * i], a[4 * i + 1], a[4 * i + 2], a[4 * i + 3]);
+            }
+            __syncwarp();
           }
-          __syncwarp();  // lanes leave their key loops at different times; reconverge before tcgen05.ld
+          named_bar_sync(5, kEpiThreads);  // A complete; Q, K, V no longer read
+          // Quant(A) -> O operand, by row slices
+          float av[XS];
+          {
+            const float4 *ap = reinterpret_cast<const float4 *>(smem + L::kOffU + L::kOffA + (r * D + sl * XS) * 4);
 #pragma unroll
-          for (int i = 0; i < DH; ++i) amax = fmaxf(amax, fabsf(A[hh][i]));
-        }
-        // Quant(A) -> O operand
-        {
+            for (int i = 0; i < XS / 4; ++i) {
+              const float4 v = ap[i];
+              av[4 * i] = v.x, av[4 * i + 1] = v.y, av[4 * i + 2] = v.z, av[4 * i + 3] = v.w;
+            }
+          }
+          float amax = 0.0f;
+#pragma unroll
+          for (int j = 0; j < XS; ++j) amax = fmaxf(amax, fabsf(av[j]));
           float a = row_max(amax);
           a = (a > p.alpha_floor) ? a : p.alpha_floor;
           alpha_in = a;
           const float rr = __fdiv_rn(127.0f, a);
-#pragma unroll
+          float qv[XS];
+          codes<XS>(av, rr, qv);
+          store_codes<XS>(aop, r, sl * XS, D, qv);
+          if (cap) capture_q(l, 1, qv, sl * XS, XS, alpha_in);
+        } else {
+        cluster_arrive(bar_kvr);
+          wait_bar(ctl, bar_kvr, kvr_ph, true);
+          kvr_ph ^= 1u;
+  
+          // ---------------- S5: HPSA (Sec. 4.2)
+          float A[2][DH];
+          float amax = 0.0f;
+  #pragma unroll
           for (int hh = 0; hh < 2; ++hh) {
             const int e = sl + 4 * hh;
-            float qv[DH];
-#pragma unroll
-            for (int i = 0; i < DH; ++i) qv[i] = q_code(A[hh][i], rr);
-            store_codes<DH>(aop, r, e * DH, D, qv);
-            if (cap) capture_q(l, 1, qv, e * DH, DH, alpha_in);
+            float qa[DH], bq[DH];
+            tmem_ld<DH>(tl + e * DH, qa);
+            tmem_wait_ld();
+            if (cap) capture_acc(l, 0, qa, e * DH, DH);
+            ldg_vec<DH>(lp + LP::bqkv(D) + e * DH, bq);
+            float q[DH];
+  #pragma unroll
+            for (int i = 0; i < DH; ++i) q[i] = __fadd_rn(__fmul_rn(qa[i], fq), bq[i]);
+  #pragma unroll
+            for (int i = 0; i < DH; ++i) A[hh][i] = 0.0f;
+            if (row_cw) {
+              const int mk = (e < p.h_first) ? 0 : 1;
+              constexpr int U = (DH >= 16) ? 2 : 4;
+              hpsa_head<DH, U, L::kKvStride>(q, __ldg(p.mask_info[mk] + t), p.mask_list[mk], s_kvgen, g * T,
+                                             e * (8 * DH), p.att_scale, A[hh]);
+            }
+            __syncwarp();  // lanes leave their key loops at different times; reconverge before tcgen05.ld
+  #pragma unroll
+            for (int i = 0; i < DH; ++i) amax = fmaxf(amax, fabsf(A[hh][i]));
+          }
+          // Quant(A) -> O operand
+          {
+            float a = row_max(amax);
+            a = (a > p.alpha_floor) ? a : p.alpha_floor;
+            alpha_in = a;
+            const float rr = __fdiv_rn(127.0f, a);
+  #pragma unroll
+            for (int hh = 0; hh < 2; ++hh) {
+              const int e = sl + 4 * hh;
+              float qv[DH];
+  #pragma unroll
+              for (int i = 0; i < DH; ++i) qv[i] = q_code(A[hh][i], rr);
+              store_codes<DH>(aop, r, e * DH, D, qv);
+              if (cap) capture_q(l, 1, qv, e * DH, DH, alpha_in);
+            }
           }
         }
         signal_op(1);
-        cluster_arrive(bar_kvf);  // this CTA no longer reads any K/V of this block
+        if constexpr (!TASKS) cluster_arrive(bar_kvf);  // this CTA no longer reads any K/V of this block
 
         // ---------------- S6: O projection + residual + LayerNorm (Sec. 5, Post-LN)
         wait_acc();
         {
           const float fo = __fdiv_rn(__fmul_rn(__ldg(sw + 3), alpha_in), 127.0f);
-          float ac[XS], bb[XS], gg[XS], be[XS];
+          float ac[XS];
           tmem_ld<XS>(tl + sl * XS, ac);
           tmem_ld<XS>(tl + 3 * D + sl * XS, x);
           tmem_wait_ld();
           if (cap) capture_acc(l, 1, ac, sl * XS, XS);
-          ldg_vec<XS>(lp + LP::bo(D) + sl * XS, bb);
-          float v[XS];
-#pragma unroll
-          for (int j = 0; j < XS; ++j) v[j] = __fadd_rn(x[j], __fadd_rn(__fmul_rn(ac[j], fo), bb[j]));
-          const float mu = __fmul_rn(row_sum(psum<XS>(v)), inv_d);
-#pragma unroll
-          for (int j = 0; j < XS; ++j) {
-            v[j] = __fsub_rn(v[j], mu);
-            ac[j] = __fmul_rn(v[j], v[j]);
-          }
-          const float var = __fmul_rn(row_sum(psum<XS>(ac)), inv_d);
-          const float rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, p.ln_eps)));
-          ldg_vec<XS>(lp + LP::ln1g(D) + sl * XS, gg);
-          ldg_vec<XS>(lp + LP::ln1b(D) + sl * XS, be);
-#pragma unroll
-          for (int j = 0; j < XS; ++j) x[j] = __fadd_rn(__fmul_rn(__fmul_rn(v[j], rstd), gg[j]), be[j]);
+          residual_ln(ac, fo, lp + LP::bo(D) + sl * XS, lp + LP::ln1g(D) + sl * XS, lp + LP::ln1b(D) + sl * XS);
         }
         {
           const float rr = quant_x_to_aop();
           if (cap) {
             float qv[XS];
-#pragma unroll
-            for (int j = 0; j < XS; ++j) qv[j] = q_code(x[j], rr);
+            codes<XS>(x, rr, qv);
             capture_q(l, 2, qv, sl * XS, XS, alpha_in);
           }
         }
@@ -659,21 +920,24 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         wait_acc();
         {
           const float f1 = __fdiv_rn(__fmul_rn(__ldg(sw + 4), alpha_in), 127.0f);
-          constexpr int NCH = D / 32;  // 32-column chunks of this thread's D hidden columns
+          constexpr int NCH = D / 32;      // 32-column chunks of this thread's D hidden columns
+          constexpr bool KEEP = D <= 64;   // u stays in registers between the max and the codes
+          float uk[KEEP ? D : 1];
           float umax = 0.0f;
-#pragma unroll 1
+#pragma unroll
           for (int ch = 0; ch < NCH; ++ch) {
             const int c0 = sl * D + 32 * ch;
-            float ac[32], bb[32];
+            float ac[32], bb[32], u[32];
             tmem_ld<32>(tl + c0, ac);
             tmem_wait_ld();
             if (cap) capture_acc(l, 2, ac, c0, 32);
             ldg_vec<32>(lp + LP::b1(D) + c0, bb);
+            dequant<32>(ac, f1, bb, u);
 #pragma unroll
             for (int j = 0; j < 32; ++j) {
-              float u = __fadd_rn(__fmul_rn(ac[j], f1), bb[j]);
-              u = u > 0.0f ? u : 0.0f;
-              umax = fmaxf(umax, u);
+              u[j] = u[j] > 0.0f ? u[j] : 0.0f;
+              umax = fmaxf(umax, u[j]);
+              if constexpr (KEEP) uk[32 * ch + j] = u[j];
             }
           }
           float a = row_max(umax);
@@ -681,22 +945,28 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           alpha_in = a;
           const float rr = __fdiv_rn(127.0f, a);
           // peers have finished reading this CTA's K/V: the shared region may now take u codes
-          wait_bar(ctl, bar_kvf, kvf_ph, true);
-          kvf_ph ^= 1u;
-#pragma unroll 1
+          if constexpr (!TASKS) {
+            wait_bar(ctl, bar_kvf, kvf_ph, true);
+            kvf_ph ^= 1u;
+          }
+#pragma unroll
           for (int ch = 0; ch < NCH; ++ch) {
             const int c0 = sl * D + 32 * ch;
-            float ac[32], bb[32];
-            tmem_ld<32>(tl + c0, ac);
-            tmem_wait_ld();
-            ldg_vec<32>(lp + LP::b1(D) + c0, bb);
-            float qv[32];
+            float u[32];
+            if constexpr (KEEP) {
 #pragma unroll
-            for (int j = 0; j < 32; ++j) {
-              float u = __fadd_rn(__fmul_rn(ac[j], f1), bb[j]);
-              u = u > 0.0f ? u : 0.0f;
-              qv[j] = q_code(u, rr);
+              for (int j = 0; j < 32; ++j) u[j] = uk[32 * ch + j];
+            } else {
+              float ac[32], bb[32];
+              tmem_ld<32>(tl + c0, ac);
+              tmem_wait_ld();
+              ldg_vec<32>(lp + LP::b1(D) + c0, bb);
+              dequant<32>(ac, f1, bb, u);
+#pragma unroll
+              for (int j = 0; j < 32; ++j) u[j] = u[j] > 0.0f ? u[j] : 0.0f;
             }
+            float qv[32];
+            codes<32>(u, rr, qv);
             store_codes<32>(uqt, r, c0, 4 * D, qv);
             if (cap) capture_q(l, 3, qv, c0, 32, alpha_in);
           }
@@ -707,33 +977,17 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         wait_acc();
         {
           const float f2 = __fdiv_rn(__fmul_rn(__ldg(sw + 5), alpha_in), 127.0f);
-          float ac[XS], bb[XS], gg[XS], be[XS];
+          float ac[XS];
           tmem_ld<XS>(tl + sl * XS, ac);
           tmem_wait_ld();
           if (cap) capture_acc(l, 3, ac, sl * XS, XS);
-          ldg_vec<XS>(lp + LP::b2(D) + sl * XS, bb);
-          float v[XS];
-#pragma unroll
-          for (int j = 0; j < XS; ++j) v[j] = __fadd_rn(x[j], __fadd_rn(__fmul_rn(ac[j], f2), bb[j]));
-          const float mu = __fmul_rn(row_sum(psum<XS>(v)), inv_d);
-#pragma unroll
-          for (int j = 0; j < XS; ++j) {
-            v[j] = __fsub_rn(v[j], mu);
-            ac[j] = __fmul_rn(v[j], v[j]);
-          }
-          const float var = __fmul_rn(row_sum(psum<XS>(ac)), inv_d);
-          const float rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, p.ln_eps)));
-          ldg_vec<XS>(lp + LP::ln2g(D) + sl * XS, gg);
-          ldg_vec<XS>(lp + LP::ln2b(D) + sl * XS, be);
-#pragma unroll
-          for (int j = 0; j < XS; ++j) x[j] = __fadd_rn(__fmul_rn(__fmul_rn(v[j], rstd), gg[j]), be[j]);
+          residual_ln(ac, f2, lp + LP::b2(D) + sl * XS, lp + LP::ln2g(D) + sl * XS, lp + LP::ln2b(D) + sl * XS);
         }
         if (l + 1 < p.n_layers) {
           const float rr = quant_x_to_aop();
           if (cap) {
             float qv[XS];
-#pragma unroll
-            for (int j = 0; j < XS; ++j) qv[j] = q_code(x[j], rr);
+            codes<XS>(x, rr, qv);
             capture_q(l + 1, 0, qv, sl * XS, XS, alpha_in);
           }
           signal_op(0);
@@ -814,10 +1068,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   }
 }
 
-template <int D>
+template <int D, bool TASKS>
 cudaError_t prepare_decode_kernel(int cluster_ctas, int *max_active_clusters) {
-  using L = SmemLayout<D>;
-  cudaError_t e = cudaFuncSetAttribute(aecct_decoder_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  using L = SmemLayout<D, TASKS>;
+  cudaError_t e = cudaFuncSetAttribute(aecct_decoder_kernel<D, TASKS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(L::kTotal));
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
@@ -831,12 +1085,12 @@ cudaError_t prepare_decode_kernel(int cluster_ctas, int *max_active_clusters) {
   cfg.dynamicSmemBytes = L::kTotal;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaOccupancyMaxActiveClusters(max_active_clusters, aecct_decoder_kernel<D>, &cfg);
+  return cudaOccupancyMaxActiveClusters(max_active_clusters, aecct_decoder_kernel<D, TASKS>, &cfg);
 }
 
-template <int D>
+template <int D, bool TASKS>
 cudaError_t launch_decode(const DecodeParams &p, cudaStream_t stream) {
-  using L = SmemLayout<D>;
+  using L = SmemLayout<D, TASKS>;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -849,14 +1103,18 @@ cudaError_t launch_decode(const DecodeParams &p, cudaStream_t stream) {
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, aecct_decoder_kernel<D>, p);
+  return cudaLaunchKernelEx(&cfg, aecct_decoder_kernel<D, TASKS>, p);
 }
 
-template cudaError_t launch_decode<32>(const DecodeParams &, cudaStream_t);
-template cudaError_t launch_decode<64>(const DecodeParams &, cudaStream_t);
-template cudaError_t launch_decode<128>(const DecodeParams &, cudaStream_t);
-template cudaError_t prepare_decode_kernel<32>(int, int *);
-template cudaError_t prepare_decode_kernel<64>(int, int *);
-template cudaError_t prepare_decode_kernel<128>(int, int *);
+template cudaError_t launch_decode<32, false>(const DecodeParams &, cudaStream_t);
+template cudaError_t launch_decode<64, false>(const DecodeParams &, cudaStream_t);
+template cudaError_t launch_decode<128, false>(const DecodeParams &, cudaStream_t);
+template cudaError_t launch_decode<32, true>(const DecodeParams &, cudaStream_t);
+template cudaError_t launch_decode<64, true>(const DecodeParams &, cudaStream_t);
+template cudaError_t prepare_decode_kernel<32, false>(int, int *);
+template cudaError_t prepare_decode_kernel<64, false>(int, int *);
+template cudaError_t prepare_decode_kernel<128, false>(int, int *);
+template cudaError_t prepare_decode_kernel<32, true>(int, int *);
+template cudaError_t prepare_decode_kernel<64, true>(int, int *);
 
 }  // namespace aecct

@@ -88,6 +88,10 @@ def test_create_rejects_invalid_packed_code_and_shapes():
     # a cluster size that cannot hold one codeword
     big = I.workload_model("ldpc384_192")
     assert _status(big, cluster_ctas=2) == A.AECCT_ERR_INVALID_ARG
+    # attention modes: unknown value, and warp tasks where they do not apply (T > 128, d = 128)
+    assert _status(I.workload_model("bch31_16"), attention_mode=3) == A.AECCT_ERR_INVALID_ARG
+    assert _status(I.workload_model("ldpc128_64"), attention_mode=2) == A.AECCT_ERR_UNSUPPORTED
+    assert _status(I.workload_model("bch63_36"), attention_mode=2) == A.AECCT_ERR_UNSUPPORTED
     # NULL description / output pointer
     assert A.load().aecct_create(None, ctypes.byref(h)) == A.AECCT_ERR_INVALID_ARG
     assert A.load().aecct_create(ctypes.byref(hm.desc), None) == A.AECCT_ERR_INVALID_ARG

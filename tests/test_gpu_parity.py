@@ -21,10 +21,11 @@ SAMPLE_B = {"bch31_16": 64, "polar64_32": 48, "ldpc128_64": 12, "bch63_36": 24, 
 _decoders = {}
 
 
-def decoder(key, cluster_ctas=0):
-    k = (key, cluster_ctas)
+def decoder(key, cluster_ctas=0, attention_mode=0):
+    k = (key, cluster_ctas, attention_mode)
     if k not in _decoders:
-        _decoders[k] = (A.Decoder(I.workload_model(key), cluster_ctas=cluster_ctas), I.workload_model(key))
+        _decoders[k] = (A.Decoder(I.workload_model(key), cluster_ctas=cluster_ctas, attention_mode=attention_mode),
+                        I.workload_model(key))
     return _decoders[k]
 
 
@@ -62,25 +63,34 @@ def test_small_batch_exact_with_integer_core(key):
     for name in ("syn_in", "q", "alpha", "acc"):
         a, b = g["capture"][name], r["capture"][name]
         if name == "alpha":
-            assert (a.view(np.int32) == b.view(np.int32)).all(), name
-        else:
-            bad = np.argwhere(a != b)
-            assert bad.size == 0, f"{name} differs first at {bad[:3].tolist()} (gpu {a[tuple(bad[0])]} oracle {b[tuple(bad[0])]})"
+            a, b = a.view(np.int32), b.view(np.int32)
+        bad = np.argwhere(a != b)
+        # index layout: [word, block, gemm (0 QKV, 1 O, 2 FFN1, 3 FFN2), token, column]
+        assert bad.size == 0, (f"{name}: {len(bad)} entries differ, first at {bad[:4].tolist()} "
+                               f"(gpu {a[tuple(bad[0])]} oracle {b[tuple(bad[0])]})")
     assert_same(g, r, key)
 
 
+LAYOUTS = {
+    # (cluster_ctas, attention_mode): per-row lists over a packed cluster, one CTA per group,
+    # warp tasks (one CTA per group, d <= 64)
+    "bch31_16": [(0, 1), (1, 1), (0, 2)],
+    "polar64_32": [(0, 1), (1, 1), (0, 2)],
+    "bch63_36": [(0, 1), (1, 1)],
+}
+
+
 @pytest.mark.gpu
-@pytest.mark.parametrize("key", ["bch31_16", "polar64_32", "bch63_36"])
-def test_result_independent_of_cluster_packing(key):
-    # one CTA per group instead of the packed cluster: identical results
-    dec1, model = decoder(key, cluster_ctas=1)
-    dec0, _ = decoder(key)
-    assert dec1.query()["cluster_ctas"] == 1
+@pytest.mark.parametrize("key", sorted(LAYOUTS))
+def test_result_independent_of_layout_and_attention_mode(key):
     w = I.workload(key)
     ch = I.channel_batch(w.code, 40, w.ebn0_db[-1], seed=77)
-    a = gpu_decode(dec1, ch.y)
-    b = gpu_decode(dec0, ch.y)
-    assert_same(a, b, key)
+    ref = O.decode(I.workload_model(key), ch.y)
+    for cc, mode in LAYOUTS[key]:
+        dec, _ = decoder(key, cluster_ctas=cc, attention_mode=mode)
+        q = dec.query()
+        assert q["attention_mode"] == mode and (cc == 0 or q["cluster_ctas"] == cc)
+        assert_same(gpu_decode(dec, ch.y), ref, f"{key} C={q['cluster_ctas']} mode={mode}")
 
 
 @pytest.mark.gpu
