@@ -324,11 +324,7 @@ __device__ __forceinline__ void hpsa_head(const float *q, uint32_t info, const u
   for (int i = 0; i < DH; ++i) A[i] = __fmul_rn(num[i], inv);
 }
 
-// membership bit k of a lane's 128-bit mask, and byte k of a 16-entry index block
-__device__ __forceinline__ bool mask_bit(const uint4 &m, int k) {
-  const uint32_t w = k < 64 ? (k < 32 ? m.x : m.y) : (k < 96 ? m.z : m.w);
-  return ((w >> (k & 31)) & 1u) != 0u;
-}
+// byte k of a 16-entry index block
 __device__ __forceinline__ int byte_at(const uint4 &w, int k) {
   const uint32_t v = k < 8 ? (k < 4 ? w.x : w.y) : (k < 12 ? w.z : w.w);
   return static_cast<int>((v >> (8 * (k & 3))) & 0xFFu);
@@ -358,10 +354,16 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
   };
   const float2 sc = make_float2(scale, scale);
   constexpr int U = 4;
+  // membership bits of a 16-key block (jb is a multiple of 16)
+  auto segment = [&](int jb) -> uint32_t {
+    const uint32_t word = jb < 64 ? (jb < 32 ? mask.x : mask.y) : (jb < 96 ? mask.z : mask.w);
+    return word >> (jb & 16);
+  };
   // pass 1: maximum score over the lane's keys
   float mx = -INFINITY;
   for (int jb = 0; jb < cnt; jb += 16) {
     const uint4 w = __ldg(ul + (jb >> 4));
+    const uint32_t seg = segment(jb);
     const int nk = min(16, cnt - jb);
     if (nk == 16) {
 #pragma unroll
@@ -376,8 +378,8 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
 #pragma unroll
         for (int k = 0; k < U; k += 2) {
           const float2 sg = mul2(dot2(kk[k], kk[k + 1]), sc);
-          if (mask_bit(mask, jb + k0 + k)) mx = fmaxf(mx, sg.x);
-          if (mask_bit(mask, jb + k0 + k + 1)) mx = fmaxf(mx, sg.y);
+          if (((seg >> (k0 + k)) & 1u)) mx = fmaxf(mx, sg.x);
+          if (((seg >> (k0 + k + 1)) & 1u)) mx = fmaxf(mx, sg.y);
         }
       }
     } else {
@@ -388,8 +390,8 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
 #pragma unroll
         for (int i = 0; i < DH / 4; ++i) ka[i] = pa[i], kb[i] = pb[i];
         const float2 sg = mul2(dot2(ka, kb), sc);
-        if (mask_bit(mask, jb + k)) mx = fmaxf(mx, sg.x);
-        if (k1 != k && mask_bit(mask, jb + k1)) mx = fmaxf(mx, sg.y);
+        if (((seg >> k) & 1u)) mx = fmaxf(mx, sg.x);
+        if (k1 != k && ((seg >> k1) & 1u)) mx = fmaxf(mx, sg.y);
       }
     }
   }
@@ -414,6 +416,7 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
   };
   for (int jb = 0; jb < cnt; jb += 16) {
     const uint4 w = __ldg(ul + (jb >> 4));
+    const uint32_t seg = segment(jb);
     const int nk = min(16, cnt - jb);
     if (nk == 16) {
 #pragma unroll
@@ -432,8 +435,8 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
         for (int k = 0; k < U; k += 2) pr[k / 2] = exp2_series2(shifted(dot2(kk[k], kk[k + 1])));
 #pragma unroll
         for (int k = 0; k < U; k += 2) {
-          if (mask_bit(mask, jb + k0 + k)) fold(pr[k / 2].x, vv[k]);
-          if (mask_bit(mask, jb + k0 + k + 1)) fold(pr[k / 2].y, vv[k + 1]);
+          if (((seg >> (k0 + k)) & 1u)) fold(pr[k / 2].x, vv[k]);
+          if (((seg >> (k0 + k + 1)) & 1u)) fold(pr[k / 2].y, vv[k + 1]);
         }
       }
     } else {
@@ -444,8 +447,8 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
 #pragma unroll
         for (int i = 0; i < DH / 4; ++i) ka[i] = pa[i], kb[i] = pb[i], va[i] = pa[DH / 4 + i], vb[i] = pb[DH / 4 + i];
         const float2 pr = exp2_series2(shifted(dot2(ka, kb)));
-        if (mask_bit(mask, jb + k)) fold(pr.x, va);
-        if (k1 != k && mask_bit(mask, jb + k1)) fold(pr.y, vb);
+        if (((seg >> k) & 1u)) fold(pr.x, va);
+        if (k1 != k && ((seg >> k1) & 1u)) fold(pr.y, vb);
       }
     }
   }
@@ -460,36 +463,50 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
 // Weight chunks are consumed in a fixed sequence: for each group of codewords, for each block,
 // the block's chunks (QKV, then O, FFN1, FFN2).  Chunk i of the sequence uses ring stage i % S;
 // its copy completes phase i / S of full[stage], its MMAs release phase i / S of empty[stage].
+// Positions advance incrementally (no integer division on the issuing thread).
 struct IssueState {
   int64_t total;   // chunks this CTA consumes
   int64_t issued;  // chunks whose copy has been started
   int64_t used;    // chunks whose MMAs have been issued
+  int cs, cc, cl;  // next copy: ring stage, chunk of the block, block
+  uint32_t cround; // next copy: number of completed passes over the ring
+  int ms, mc;      // next MMA: ring stage, chunk of the block
+  uint32_t mround; // next MMA: passes over the ring
   uint32_t oph;    // parity of the next operand-ready phase
+  uint32_t aph;    // parity of the next accumulator-ready phase
 };
 
+// Start the copy of the next chunk into its ring stage (waiting for the stage's previous MMAs).
 template <int D, bool TASKS>
-__device__ __noinline__ void issue_copies(const DecodeParams &p, const Ctl &ctl, IssueState &st, int64_t limit,
-                                          uint32_t sb) {
+__device__ __forceinline__ void copy_next(const DecodeParams &p, const Ctl &ctl, IssueState &st, uint32_t sb) {
   using L = SmemLayout<D, TASKS>;
   constexpr int S = L::kStages;
   const uint32_t bar_full = sb + L::kOffBar, bar_empty = bar_full + 8 * S;
-  if (limit > st.total) limit = st.total;
-  while (st.issued < limit) {
+  if (st.cround > 0) wait_bar(ctl, bar_empty + 8 * st.cs, (st.cround - 1u) & 1u, false);
+  const uint32_t bytes = p.chunks[st.cc].bytes;
+  mbar_arrive_expect_tx(bar_full + 8 * st.cs, bytes);
+  bulk_g2s(sb + L::kOffW + st.cs * kStageBytes, p.wstream + (size_t)st.cl * p.layer_bytes + p.chunks[st.cc].off,
+           bytes, bar_full + 8 * st.cs);
+  ++st.issued;
+  if (++st.cs == S) st.cs = 0, ++st.cround;
+  if (++st.cc == p.n_chunks) {
+    st.cc = 0;
+    if (++st.cl == p.n_layers) st.cl = 0;
+  }
+}
+
+// Keep up to S chunks in flight ahead of the MMAs.
+template <int D, bool TASKS>
+__device__ __noinline__ void issue_copies(const DecodeParams &p, const Ctl &ctl, IssueState &st, uint32_t sb) {
+  constexpr int S = SmemLayout<D, TASKS>::kStages;
+  while (st.issued < st.total && st.issued < st.used + S) {
     if (*ctl.abort) return;
-    const int s = static_cast<int>(st.issued % S);
-    if (st.issued >= S) wait_bar(ctl, bar_empty + 8 * s, static_cast<uint32_t>((st.issued / S - 1) & 1), false);
-    const int c = static_cast<int>(st.issued % p.n_chunks);
-    const int l = static_cast<int>((st.issued / p.n_chunks) % p.n_layers);
-    const uint32_t bytes = p.chunks[c].bytes;
-    mbar_arrive_expect_tx(bar_full + 8 * s, bytes);
-    bulk_g2s(sb + L::kOffW + s * kStageBytes, p.wstream + (size_t)l * p.layer_bytes + p.chunks[c].off, bytes,
-             bar_full + 8 * s);
-    ++st.issued;
+    copy_next<D, TASKS>(p, ctl, st, sb);
   }
 }
 
 // Wait until every warp has published the operand of GEMM `gemm`, issue its tcgen05.mma chain
-// (accumulators at TMEM column 0), signal the accumulator barrier, then prefetch the next chunks.
+// (accumulators at TMEM column 0), wait for its completion, then prefetch the next chunks.
 template <int D, bool TASKS>
 __device__ __noinline__ void issue_gemm(const DecodeParams &p, const Ctl &ctl, IssueState &st, int gemm, uint32_t sb,
                                         uint32_t tmem) {
@@ -503,14 +520,12 @@ __device__ __noinline__ void issue_gemm(const DecodeParams &p, const Ctl &ctl, I
   const uint32_t a_tile = (gemm == 3) ? (sb + L::kOffU) : (sb + L::kOffAop);
   const uint32_t a_sbo = (gemm == 3) ? (4u * D / 8u) * 128u : (D / 8u) * 128u;
   while (st.used < st.total) {
-    const int c = static_cast<int>(st.used % p.n_chunks);
-    const ChunkDesc ch = p.chunks[c];
+    const ChunkDesc ch = p.chunks[st.mc];
     if (ch.gemm != gemm) break;
-    issue_copies<D, TASKS>(p, ctl, st, st.used + 1, sb);
-    const int s = static_cast<int>(st.used % S);
-    wait_bar(ctl, bar_full + 8 * s, static_cast<uint32_t>((st.used / S) & 1), false);
+    if (st.issued == st.used) copy_next<D, TASKS>(p, ctl, st, sb);
+    wait_bar(ctl, bar_full + 8 * st.ms, st.mround & 1u, false);
     tc_fence_after();
-    const uint32_t b_tile = sb + L::kOffW + s * kStageBytes;
+    const uint32_t b_tile = sb + L::kOffW + st.ms * kStageBytes;
     const uint32_t b_sbo = (ch.kcols / 8u) * 128u;
     const uint32_t idesc = make_idesc_bf16(128, ch.nrows);
     for (int ks = 0; ks < ch.kcols / 16; ++ks) {
@@ -519,11 +534,18 @@ __device__ __noinline__ void issue_gemm(const DecodeParams &p, const Ctl &ctl, I
       const uint64_t bd = make_sdesc(b_tile + ks * 256u, 128u, b_sbo);
       mma_bf16(tmem + ch.n0, ad, bd, idesc, kabs > 0 ? 1u : 0u);
     }
-    mma_commit(bar_empty + 8 * s);
+    mma_commit(bar_empty + 8 * st.ms);
     ++st.used;
+    if (++st.ms == S) st.ms = 0, ++st.mround;
+    if (++st.mc == p.n_chunks) st.mc = 0;
   }
   mma_commit(bar_acc);
-  issue_copies<D, TASKS>(p, ctl, st, st.used + S, sb);
+  // the issuing thread alone waits for the accumulators; the other threads of the CTA wait in a
+  // named barrier (no spinning), which this thread joins after the wait
+  wait_bar(ctl, bar_acc, st.aph, false);
+  st.aph ^= 1u;
+  // every MMA so far is complete, so the stages they read are free: prefetch the next chunks
+  issue_copies<D, TASKS>(p, ctl, st, sb);
 }
 
 // ------------------------------------------------------------------------------------------
@@ -589,11 +611,11 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   const uint32_t tmem = *s_tmem;
   const Ctl ctl{s_abort, p.err, p.wait_limit};
 
-  IssueState ist{0, 0, 0, 0};
+  IssueState ist{};
   if (tid == 0) {
     const int64_t my_groups = (p.n_groups - cluster_id + p.n_clusters - 1) / p.n_clusters;
     ist.total = my_groups * p.n_layers * p.n_chunks;
-    issue_copies<D, TASKS>(p, ctl, ist, S, sb);
+    issue_copies<D, TASKS>(p, ctl, ist, sb);
   }
   __syncwarp();
   {
@@ -611,7 +633,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
     const int T = p.T, n = p.n, m = p.m, de = D - p.d_spe;
     const int W4 = 4 * D;
     const float inv_d = 1.0f / static_cast<float>(D);
-    uint32_t acc_ph = 0, kvr_ph = 0, kvf_ph = 0, zr_ph = 0;
+    uint32_t kvr_ph = 0, kvf_ph = 0, zr_ph = 0, zf_ph = 0;
     int64_t z_uses = 0;
 
     // reduce one value per row over the 4 slices: max or pairwise sum ((s0+s1)+(s2+s3))
@@ -647,10 +669,18 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
       }
       __syncwarp();
     };
+    // accumulators of the last GEMM are complete once thread 0 (which waited for them inside
+    // issue_gemm) reaches this barrier
     auto wait_acc = [&]() {
-      wait_bar(ctl, bar_acc, acc_ph, false);
-      acc_ph ^= 1u;
+      named_bar_sync(5, kEpiThreads);
       tc_fence_after();
+    };
+    // wait for a cluster-wide phase: thread 0 waits on the mbarrier, the others in a named barrier
+    auto cluster_wait = [&](uint32_t bar, uint32_t &ph) {
+      if (tid == 0) wait_bar(ctl, bar, ph, true);
+      ph ^= 1u;
+      __syncwarp();
+      named_bar_sync(5, kEpiThreads);
     };
 
     for (int64_t gi = cluster_id; gi < p.n_groups; gi += p.n_clusters) {
@@ -846,8 +876,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           if (cap) capture_q(l, 1, qv, sl * XS, XS, alpha_in);
         } else {
         cluster_arrive(bar_kvr);
-          wait_bar(ctl, bar_kvr, kvr_ph, true);
-          kvr_ph ^= 1u;
+          cluster_wait(bar_kvr, kvr_ph);
   
           // ---------------- S5: HPSA (Sec. 4.2)
           float A[2][DH];
@@ -945,10 +974,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           alpha_in = a;
           const float rr = __fdiv_rn(127.0f, a);
           // peers have finished reading this CTA's K/V: the shared region may now take u codes
-          if constexpr (!TASKS) {
-            wait_bar(ctl, bar_kvf, kvf_ph, true);
-            kvf_ph ^= 1u;
-          }
+          if constexpr (!TASKS) cluster_wait(bar_kvf, kvf_ph);
 #pragma unroll
           for (int ch = 0; ch < NCH; ++ch) {
             const int c0 = sl * D + 32 * ch;
@@ -1001,13 +1027,12 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
 #pragma unroll
         for (int j = 0; j < XS; ++j) wv[j] = __fmul_rn(x[j], wv[j]);
         const float z = __fadd_rn(row_sum(psum<XS>(wv)), p.b_d1);
-        if (z_uses > 0) wait_bar(ctl, bar_zf, static_cast<uint32_t>((z_uses - 1) & 1), true);
+        if (z_uses > 0) cluster_wait(bar_zf, zf_ph);
         ++z_uses;
         if (sl == 0) zbuf[r] = z;
       }
       cluster_arrive(bar_zr);
-      wait_bar(ctl, bar_zr, zr_ph, true);
-      zr_ph ^= 1u;
+      cluster_wait(bar_zr, zr_ph);
       // ---------------- S10: decisions x_hat = y * eps, decoded-word syndrome
       {
         const int n_local = (p.G - static_cast<int>(crank) + p.C - 1) / p.C;  // groups g = crank + C*i
