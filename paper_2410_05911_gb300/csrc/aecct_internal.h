@@ -11,7 +11,7 @@ constexpr int kRows = 128;          // token rows per CTA: one M = 128 tensor-co
 constexpr int kHeads = 8;           // this build: 8 attention heads
 constexpr int kEpiWarps = 16;       // 4 TMEM lane quadrants x 4 column slices
 constexpr int kEpiThreads = kEpiWarps * 32;
-constexpr int kThreads = kEpiThreads;  // thread 0 also streams weights and issues the MMAs
+constexpr int kThreads = kEpiThreads;  // warp 0 also streams weights and issues the MMAs
 constexpr int kMaxCluster = 8;
 constexpr uint32_t kStageBytes = 16384;  // one weight chunk: <= 128 rows x 64 K bf16
 constexpr int kMaxChunks = 32;           // weight chunks per block (QKV, O, FFN1, FFN2)
@@ -104,18 +104,15 @@ __host__ __device__ constexpr inline uint32_t core_off(uint32_t r, uint32_t c, u
 
 // Shared-memory map.  Region U holds, per block, first the attention operands and then the FFN2
 // operand.  Row mode: per token row 8 heads x (K | V) x d_h fp32.  Task mode: 8 heads x
-// (Q | K | V) x d_h fp32, followed by the attention output A [128][D] fp32.
+// (Q | K | V) x d_h fp32; the attention output of a (row, head) then replaces its Q.
 template <int D, bool TASKS = false>
 struct SmemLayout {
   static constexpr uint32_t kSlot = (TASKS ? 12u : 8u) * (D / 8u);  // bytes of one head of one row
   static constexpr uint32_t kKvStride = 8u * kSlot + 16u;            // token row, + 16 B pad
   static constexpr uint32_t kKvBytes = kRows * kKvStride;
-  static constexpr uint32_t kOffA = kKvBytes;                         // task mode: A [128][D] fp32
-  static constexpr uint32_t kABytes = TASKS ? kRows * D * 4u : 0u;
   static constexpr uint32_t kUqBytes = kRows * 4u * D * 2u;  // FFN2 operand: 128 x 4D bf16
   __host__ __device__ static constexpr uint32_t align1k(uint32_t v) { return (v + 1023u) & ~1023u; }
-  static constexpr uint32_t kRegionU =
-      align1k(kKvBytes + kABytes > kUqBytes ? kKvBytes + kABytes : kUqBytes);
+  static constexpr uint32_t kRegionU = align1k(kKvBytes > kUqBytes ? kKvBytes : kUqBytes);
   static constexpr uint32_t kAopBytes = kRows * D * 2u;  // QKV / O / FFN1 operand: 128 x D bf16
   static constexpr int kStages = (D == 128) ? 3 : 4;
   static constexpr uint32_t kOffU = 0;
@@ -125,8 +122,8 @@ struct SmemLayout {
   static constexpr uint32_t kOffZ = kOffRed + 4096;                   // 128 floats
   static constexpr uint32_t kOffObits = kOffZ + 512;                  // decoded bits
   static constexpr uint32_t kOffBar = kOffObits + kOutBitsBytes;      // mbarriers
-  static constexpr uint32_t kOffMisc = kOffBar + 256;                 // tmem base, abort flag, peer bases
-  static constexpr uint32_t kTotal = kOffMisc + 256;
+  static constexpr uint32_t kOffMisc = kOffBar + 256;  // tmem base, abort flag, peer bases, issue table
+  static constexpr uint32_t kTotal = kOffMisc + 1024;
   static constexpr uint32_t kTmemCols = 4u * D;
 };
 

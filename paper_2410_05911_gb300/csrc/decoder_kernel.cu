@@ -118,12 +118,12 @@ struct Ctl {
   long long limit;
 };
 
-// Bounded mbarrier wait.  Returns false (and raises the CTA abort flag plus the device
-// error word) when the phase does not complete within `limit` SM cycles; once the abort
+// Bounded mbarrier wait (wait_bar).  Returns false (and raises the CTA abort flag plus the
+// device error word) when the phase does not complete within `limit` SM cycles; once the abort
 // flag is up every later wait returns false at once so the kernel drains without blocking.
-__device__ __noinline__ bool wait_bar(const Ctl &c, uint32_t bar, uint32_t parity, bool cluster_scope) {
-  if (*c.abort) return false;
-  if (cluster_scope ? mbar_try_wait_acq_cluster(bar, parity) : mbar_try_wait(bar, parity)) return true;
+// The polling loop is out of line; the first test is inline (a call saves registers to local
+// memory, which misses the small L1 left beside the shared-memory carve-out).
+__device__ __noinline__ bool wait_bar_slow(const Ctl c, uint32_t bar, uint32_t parity, bool cluster_scope) {
   const long long t0 = clock64();
   while (true) {
     for (int i = 0; i < 32; ++i)
@@ -136,8 +136,19 @@ __device__ __noinline__ bool wait_bar(const Ctl &c, uint32_t bar, uint32_t parit
     }
   }
 }
+__device__ __forceinline__ bool wait_bar(const Ctl c, uint32_t bar, uint32_t parity, bool cluster_scope) {
+  if (*c.abort) return false;
+  if (cluster_scope ? mbar_try_wait_acq_cluster(bar, parity) : mbar_try_wait(bar, parity)) return true;
+  return wait_bar_slow(c, bar, parity, cluster_scope);
+}
+// The same wait for a whole converged warp: lane 0 polls, the result goes to every lane.
+__device__ __forceinline__ bool wait_bar_warp(const Ctl c, uint32_t bar, uint32_t parity, bool cluster_scope) {
+  bool ok = true;
+  if ((threadIdx.x & 31) == 0) ok = wait_bar(c, bar, parity, cluster_scope);
+  return __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+}
 // Teardown wait: ignores the abort flag (used to drain copies / MMAs in flight), still bounded.
-__device__ __noinline__ bool wait_bar_drain(const Ctl &c, uint32_t bar, uint32_t parity) {
+__device__ __noinline__ bool wait_bar_drain(const Ctl c, uint32_t bar, uint32_t parity) {
   const long long t0 = clock64();
   while (!mbar_try_wait(bar, parity)) {
     if (clock64() - t0 > c.limit) {
@@ -458,12 +469,25 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
 }
 
 // ------------------------------------------------------------------------------------------
-// weight streaming and tensor-core issue (run by thread 0 of each CTA)
+// weight streaming and tensor-core issue (run by warp 0 of each CTA)
 // ------------------------------------------------------------------------------------------
 // Weight chunks are consumed in a fixed sequence: for each group of codewords, for each block,
 // the block's chunks (QKV, then O, FFN1, FFN2).  Chunk i of the sequence uses ring stage i % S;
 // its copy completes phase i / S of full[stage], its MMAs release phase i / S of empty[stage].
-// Positions advance incrementally (no integer division on the issuing thread).
+// Positions advance incrementally (no integer division on the issuing warp).
+
+// What the issuing warp reads for every chunk, copied once into shared memory.
+struct IssueTable {
+  ChunkDesc chunks[kMaxChunks];
+  const uint8_t *wstream;
+  uint32_t layer_bytes;
+  int n_chunks;
+  int n_layers;
+  int pad;
+};
+
+// Progress of the weight-chunk ring and of the MMA chain.  Warp 0 issues both; every lane of it
+// holds the same copy of this state.
 struct IssueState {
   int64_t total;   // chunks this CTA consumes
   int64_t issued;  // chunks whose copy has been started
@@ -478,15 +502,14 @@ struct IssueState {
 
 // Start the copy of the next chunk into its ring stage (waiting for the stage's previous MMAs).
 template <int D, bool TASKS>
-__device__ __forceinline__ void copy_next(const DecodeParams &p, const Ctl &ctl, IssueState &st, uint32_t sb) {
+__device__ __forceinline__ void copy_next(const IssueTable &p, const Ctl ctl, IssueState &st, uint32_t sb) {
   using L = SmemLayout<D, TASKS>;
   constexpr int S = L::kStages;
   const uint32_t bar_full = sb + L::kOffBar, bar_empty = bar_full + 8 * S;
-  if (st.cround > 0) wait_bar(ctl, bar_empty + 8 * st.cs, (st.cround - 1u) & 1u, false);
-  const uint32_t bytes = p.chunks[st.cc].bytes;
-  mbar_arrive_expect_tx(bar_full + 8 * st.cs, bytes);
-  bulk_g2s(sb + L::kOffW + st.cs * kStageBytes, p.wstream + (size_t)st.cl * p.layer_bytes + p.chunks[st.cc].off,
-           bytes, bar_full + 8 * st.cs);
+  if (st.cround > 0) wait_bar_warp(ctl, bar_empty + 8 * st.cs, (st.cround - 1u) & 1u, false);
+  const ChunkDesc &ch = p.chunks[st.cc];
+  bulk_g2s_expect_warp(sb + L::kOffW + st.cs * kStageBytes, p.wstream + (size_t)st.cl * p.layer_bytes + ch.off,
+                       ch.bytes, bar_full + 8 * st.cs);
   ++st.issued;
   if (++st.cs == S) st.cs = 0, ++st.cround;
   if (++st.cc == p.n_chunks) {
@@ -495,26 +518,36 @@ __device__ __forceinline__ void copy_next(const DecodeParams &p, const Ctl &ctl,
   }
 }
 
-// Keep up to S chunks in flight ahead of the MMAs.
+// Keep up to S chunks in flight ahead of the MMAs (whole warp 0).
 template <int D, bool TASKS>
-__device__ __noinline__ void issue_copies(const DecodeParams &p, const Ctl &ctl, IssueState &st, uint32_t sb) {
+__device__ __forceinline__ void issue_copies_reg(const IssueTable &p, const Ctl ctl, IssueState &st, uint32_t sb) {
   constexpr int S = SmemLayout<D, TASKS>::kStages;
   while (st.issued < st.total && st.issued < st.used + S) {
     if (*ctl.abort) return;
     copy_next<D, TASKS>(p, ctl, st, sb);
   }
 }
-
-// Wait until every warp has published the operand of GEMM `gemm`, issue its tcgen05.mma chain
-// (accumulators at TMEM column 0), wait for its completion, then prefetch the next chunks.
+// The issue state lives in shared memory between calls (a local-memory copy would miss the small
+// L1 left beside the shared-memory carve-out); each call works on a register copy.
 template <int D, bool TASKS>
-__device__ __noinline__ void issue_gemm(const DecodeParams &p, const Ctl &ctl, IssueState &st, int gemm, uint32_t sb,
+__device__ __forceinline__ void issue_copies(const IssueTable &p, const Ctl ctl, IssueState *sst, uint32_t sb) {
+  IssueState st = *sst;
+  issue_copies_reg<D, TASKS>(p, ctl, st, sb);
+  *sst = st;
+}
+
+// Whole warp 0: wait until every warp has published the operand of GEMM `gemm`, issue its
+// tcgen05.mma chain (accumulators at TMEM column 0), wait for its completion, then prefetch the
+// next chunks.
+template <int D, bool TASKS>
+__device__ __forceinline__ void issue_gemm(const IssueTable &p, const Ctl ctl, IssueState *sst, int gemm, uint32_t sb,
                                         uint32_t tmem) {
   using L = SmemLayout<D, TASKS>;
+  IssueState st = *sst;
   constexpr int S = L::kStages;
   const uint32_t bar_full = sb + L::kOffBar, bar_empty = bar_full + 8 * S;
   const uint32_t bar_op = bar_empty + 8 * S, bar_acc = bar_op + 8;
-  wait_bar(ctl, bar_op, st.oph, false);
+  wait_bar_warp(ctl, bar_op, st.oph, false);
   st.oph ^= 1u;
   tc_fence_after();
   const uint32_t a_tile = (gemm == 3) ? (sb + L::kOffU) : (sb + L::kOffAop);
@@ -523,7 +556,7 @@ __device__ __noinline__ void issue_gemm(const DecodeParams &p, const Ctl &ctl, I
     const ChunkDesc ch = p.chunks[st.mc];
     if (ch.gemm != gemm) break;
     if (st.issued == st.used) copy_next<D, TASKS>(p, ctl, st, sb);
-    wait_bar(ctl, bar_full + 8 * st.ms, st.mround & 1u, false);
+    wait_bar_warp(ctl, bar_full + 8 * st.ms, st.mround & 1u, false);
     tc_fence_after();
     const uint32_t b_tile = sb + L::kOffW + st.ms * kStageBytes;
     const uint32_t b_sbo = (ch.kcols / 8u) * 128u;
@@ -532,20 +565,21 @@ __device__ __noinline__ void issue_gemm(const DecodeParams &p, const Ctl &ctl, I
       const uint32_t kabs = ch.k0 + 16u * ks;
       const uint64_t ad = make_sdesc(a_tile + (kabs / 8u) * 128u, 128u, a_sbo);
       const uint64_t bd = make_sdesc(b_tile + ks * 256u, 128u, b_sbo);
-      mma_bf16(tmem + ch.n0, ad, bd, idesc, kabs > 0 ? 1u : 0u);
+      mma_bf16_warp(tmem + ch.n0, ad, bd, idesc, kabs > 0 ? 1u : 0u);
     }
-    mma_commit(bar_empty + 8 * st.ms);
+    mma_commit_warp(bar_empty + 8 * st.ms);
     ++st.used;
     if (++st.ms == S) st.ms = 0, ++st.mround;
     if (++st.mc == p.n_chunks) st.mc = 0;
   }
-  mma_commit(bar_acc);
-  // the issuing thread alone waits for the accumulators; the other threads of the CTA wait in a
-  // named barrier (no spinning), which this thread joins after the wait
-  wait_bar(ctl, bar_acc, st.aph, false);
+  mma_commit_warp(bar_acc);
+  // warp 0 alone waits for the accumulators; the other warps of the CTA wait in a named barrier
+  // (no spinning), which warp 0 joins after the wait
+  wait_bar_warp(ctl, bar_acc, st.aph, false);
   st.aph ^= 1u;
   // every MMA so far is complete, so the stages they read are free: prefetch the next chunks
-  issue_copies<D, TASKS>(p, ctl, st, sb);
+  issue_copies_reg<D, TASKS>(p, ctl, st, sb);
+  *sst = st;
 }
 
 // ------------------------------------------------------------------------------------------
@@ -577,6 +611,9 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   volatile int *s_abort = reinterpret_cast<volatile int *>(smem + L::kOffMisc + 4);
   uint64_t *s_kvgen = reinterpret_cast<uint64_t *>(smem + L::kOffMisc + 8);  // [8] generic K/V bases per CTA
   uint64_t *s_zgen = reinterpret_cast<uint64_t *>(smem + L::kOffMisc + 72);   // [8] generic z bases per CTA
+  IssueTable *s_itab = reinterpret_cast<IssueTable *>(smem + L::kOffMisc + 256);
+  IssueState *s_ist = reinterpret_cast<IssueState *>(smem + L::kOffMisc + 256 + sizeof(IssueTable));
+  static_assert(256 + sizeof(IssueTable) + sizeof(IssueState) <= L::kTotal - L::kOffMisc, "misc area too small");
 
   if (tid == 0) {
     for (int s = 0; s < S; ++s) {
@@ -591,6 +628,11 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
     mbar_init(bar_zf, p.C);
     mbar_init(bar_fin, 1);
     *s_abort = 0;
+    for (int c = 0; c < kMaxChunks; ++c) s_itab->chunks[c] = p.chunks[c];
+    s_itab->wstream = p.wstream;
+    s_itab->layer_bytes = p.layer_bytes;
+    s_itab->n_chunks = p.n_chunks;
+    s_itab->n_layers = p.n_layers;
     // generic base of the K/V and z areas of every CTA of the cluster: this CTA's own area through
     // its plain shared-memory window, the others through the distributed shared window
     for (int c = 0; c < p.C; ++c) {
@@ -611,13 +653,15 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   const uint32_t tmem = *s_tmem;
   const Ctl ctl{s_abort, p.err, p.wait_limit};
 
-  IssueState ist{};
-  if (tid == 0) {
-    const int64_t my_groups = (p.n_groups - cluster_id + p.n_clusters - 1) / p.n_clusters;
-    ist.total = my_groups * p.n_layers * p.n_chunks;
-    issue_copies<D, TASKS>(p, ctl, ist, sb);
+  if (warp == 0) {
+    if (lane == 0) {
+      IssueState st{};
+      st.total = (p.n_groups - cluster_id + p.n_clusters - 1) / p.n_clusters * p.n_layers * p.n_chunks;
+      *s_ist = st;
+    }
+    __syncwarp();
+    issue_copies<D, TASKS>(*s_itab, ctl, s_ist, sb);
   }
-  __syncwarp();
   {
     // ------------------------------------------------------------ CUDA-core warps
     const int qd = warp & 3, sl = warp >> 2;
@@ -651,14 +695,14 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
       red.sel ^= 1;
       return a;
     };
-    // publish this warp's part of the operand of `gemm`; thread 0 then issues the GEMM
+    // publish this warp's part of the operand of `gemm`; warp 0 then issues the GEMM
     auto signal_op = [&](int gemm) {
       tc_fence_before();  // this thread's TMEM reads are ordered before the MMA the arrive releases
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) mbar_arrive(bar_op);
-      if (tid == 0) issue_gemm<D, TASKS>(p, ctl, ist, gemm, sb, tmem);
-      __syncwarp();  // warp 0 waits for its issuing lane before any warp-collective instruction
+      __syncwarp();
+      if (warp == 0) issue_gemm<D, TASKS>(*s_itab, ctl, s_ist, gemm, sb, tmem);
     };
     auto cluster_arrive = [&](uint32_t bar) {
       // all 512 CUDA-core threads of this CTA are past their accesses: tell every CTA
@@ -669,7 +713,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
       }
       __syncwarp();
     };
-    // accumulators of the last GEMM are complete once thread 0 (which waited for them inside
+    // accumulators of the last GEMM are complete once warp 0 (which waited for them inside
     // issue_gemm) reaches this barrier
     auto wait_acc = [&]() {
       named_bar_sync(5, kEpiThreads);
@@ -846,7 +890,8 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             hpsa_task<DH, L::kKvStride>(q, mk, static_cast<int>(ui & 255u), p.plan_ulist + (ui >> 8),
                                         smem + L::kOffU + gi.z * L::kKvStride, e * L::kSlot + 4 * DH, p.att_scale, a);
             if (act) {
-              float4 *ap = reinterpret_cast<float4 *>(smem + L::kOffU + L::kOffA + (row * D + e * DH) * 4);
+              // A of (row, head e) replaces Q of (row, head e): this task was its only reader
+              float4 *ap = reinterpret_cast<float4 *>(smem + L::kOffU + row * L::kKvStride + e * L::kSlot);
 #pragma unroll
               for (int i = 0; i < DH / 4; ++i) ap[i] = make_float4(a[4 * i], a[4 * i + 1], a[4 * i + 2], a[4 * i + 3]);
             }
@@ -854,13 +899,17 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           }
           named_bar_sync(5, kEpiThreads);  // A complete; Q, K, V no longer read
           // Quant(A) -> O operand, by row slices
+          // columns [sl XS, sl XS + XS) are heads 2 sl and 2 sl + 1, in their Q slots
           float av[XS];
-          {
-            const float4 *ap = reinterpret_cast<const float4 *>(smem + L::kOffU + L::kOffA + (r * D + sl * XS) * 4);
 #pragma unroll
-            for (int i = 0; i < XS / 4; ++i) {
+          for (int hh = 0; hh < 2; ++hh) {
+            const float4 *ap =
+                reinterpret_cast<const float4 *>(smem + L::kOffU + r * L::kKvStride + (2 * sl + hh) * L::kSlot);
+#pragma unroll
+            for (int i = 0; i < DH / 4; ++i) {
               const float4 v = ap[i];
-              av[4 * i] = v.x, av[4 * i + 1] = v.y, av[4 * i + 2] = v.z, av[4 * i + 3] = v.w;
+              av[hh * DH + 4 * i] = v.x, av[hh * DH + 4 * i + 1] = v.y;
+              av[hh * DH + 4 * i + 2] = v.z, av[hh * DH + 4 * i + 3] = v.w;
             }
           }
           float amax = 0.0f;
@@ -1075,16 +1124,20 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   }
 
   // ------------------------------------------------------------ teardown
-  if (tid == 0) {
+  if (warp == 0) {
     // every MMA and every weight copy this CTA started must have landed before TMEM and the
     // shared memory go away
-    mma_commit(bar_fin);
-    wait_bar_drain(ctl, bar_fin, 0);
-    for (int64_t i = ist.issued - S; i < ist.issued; ++i)
-      if (i >= 0) wait_bar_drain(ctl, bar_full + 8 * static_cast<int>(i % S), static_cast<uint32_t>((i / S) & 1));
+    __syncwarp();
+    mma_commit_warp(bar_fin);
+    if (lane == 0) {
+      wait_bar_drain(ctl, bar_fin, 0);
+      const int64_t issued = s_ist->issued;
+      for (int64_t i = issued - S; i < issued; ++i)
+        if (i >= 0) wait_bar_drain(ctl, bar_full + 8 * static_cast<int>(i % S), static_cast<uint32_t>((i / S) & 1));
+    }
+    __syncwarp();
   }
   tc_fence_before();
-  __syncwarp();
   cluster_sync_all();
   if (warp == 0) {
     __syncwarp();
@@ -1099,6 +1152,18 @@ cudaError_t prepare_decode_kernel(int cluster_ctas, int *max_active_clusters) {
   cudaError_t e = cudaFuncSetAttribute(aecct_decoder_kernel<D, TASKS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(L::kTotal));
   if (e != cudaSuccess) return e;
+  // ask for the smallest shared-memory carve-out that holds one CTA (1 KB of it is reserved by
+  // the system): the rest of the 256 KB unified array stays L1 for spills and parameter loads
+  int dev = 0, smem_sm = 0;
+  if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+  if ((e = cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev)) != cudaSuccess)
+    return e;
+  if (smem_sm > 0) {
+    const int pct = static_cast<int>((100ll * (L::kTotal + 1024) + smem_sm - 1) / smem_sm);
+    e = cudaFuncSetAttribute(aecct_decoder_kernel<D, TASKS>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                             pct > 100 ? 100 : pct);
+    if (e != cudaSuccess) return e;
+  }
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
