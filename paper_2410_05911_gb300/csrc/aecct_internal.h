@@ -13,8 +13,6 @@ constexpr int kEpiWarps = 16;       // 4 TMEM lane quadrants x 4 column slices
 constexpr int kEpiThreads = kEpiWarps * 32;
 constexpr int kThreads = kEpiThreads;  // warp 0 also streams weights and issues the MMAs
 constexpr int kMaxCluster = 8;
-constexpr uint32_t kStageBytes = 16384;  // one weight chunk: <= 128 rows x 64 K bf16
-constexpr int kMaxChunks = 32;           // weight chunks per block (QKV, O, FFN1, FFN2)
 constexpr int kOutBitsBytes = 4096;      // decoded bits of the codewords one CTA finishes
 constexpr int kMaxTasks = 16;            // attention tasks per warp (task mode)
 constexpr int kMaxGroups = 32;           // 32-row query groups per CTA (task mode)
@@ -25,8 +23,65 @@ constexpr int kMaxGroups = 32;           // 32-row query groups per CTA (task mo
 struct ChunkDesc {
   uint32_t off;
   uint32_t bytes;
-  uint16_t gemm, n0, nrows, k0, kcols, pad;
+  int gemm, n0, nrows, k0, kcols;
 };
+
+// The fixed order in which a block's weights stream through shared memory, for model width D.
+// GEMM g has N_g output rows and K_g inputs: QKV (3D, D), O (D, D), FFN1 (4D, D), FFN2 (D, 4D).
+// D = 32 and 64: one chunk per GEMM (N <= 256 is a single tcgen05.mma shape), two stages of the
+// largest GEMM.  D = 128: 128 x 64 chunks, three 16 KB stages.  A block has kCPL chunks; kCPL is
+// a multiple of 2 kStages, so chunk p of any block uses stage p % kStages and completes phase
+// parity (p / kStages) & 1 of that stage's barriers, whatever block it belongs to.
+template <int D>
+struct WeightSchedule {
+  static constexpr int kStages = (D == 128) ? 3 : 2;
+  static constexpr uint32_t kStageBytes = (D == 32) ? 8192u : (D == 64) ? 32768u : 16384u;
+  __host__ __device__ static constexpr int gemm_n(int g) { return g == 0 ? 3 * D : (g == 2 ? 4 * D : D); }
+  __host__ __device__ static constexpr int gemm_k(int g) { return g == 3 ? 4 * D : D; }
+  __host__ __device__ static constexpr int tile_n(int g) { return D == 128 ? 128 : gemm_n(g); }
+  __host__ __device__ static constexpr int tile_k(int g) { return D == 128 ? 64 : gemm_k(g); }
+  __host__ __device__ static constexpr int count(int g) {
+    return ((gemm_n(g) + tile_n(g) - 1) / tile_n(g)) * (gemm_k(g) / tile_k(g));
+  }
+  __host__ __device__ static constexpr int first(int g) {
+    int f = 0;
+    for (int h = 0; h < g; ++h) f += count(h);
+    return f;
+  }
+  static constexpr int kCPL = first(4);  // chunks per block
+  __host__ __device__ static constexpr ChunkDesc chunk(int p) {
+    int g = 0;
+    while (g < 3 && p >= first(g + 1)) ++g;
+    const int j = p - first(g), kt = gemm_k(g) / tile_k(g);
+    const int n0 = (j / kt) * tile_n(g), k0 = (j % kt) * tile_k(g);
+    const int nrows = (gemm_n(g) - n0) < tile_n(g) ? (gemm_n(g) - n0) : tile_n(g);
+    uint32_t off = 0;
+    for (int q = 0; q < p; ++q) off += chunk_bytes(q);
+    return ChunkDesc{off, static_cast<uint32_t>(nrows * tile_k(g) * 2), g, n0, nrows, k0, tile_k(g)};
+  }
+  __host__ __device__ static constexpr uint32_t chunk_bytes(int p) {
+    int g = 0;
+    while (g < 3 && p >= first(g + 1)) ++g;
+    const int j = p - first(g), kt = gemm_k(g) / tile_k(g);
+    const int n0 = (j / kt) * tile_n(g);
+    const int nrows = (gemm_n(g) - n0) < tile_n(g) ? (gemm_n(g) - n0) : tile_n(g);
+    return static_cast<uint32_t>(nrows * tile_k(g) * 2);
+  }
+  static constexpr uint32_t kLayerBytes = chunk(kCPL - 1).off + chunk_bytes(kCPL - 1);
+};
+// the tcgen05.mma shape rules (M = 128: 16 <= N <= 256, N % 16 == 0) and the stage sizes
+template <int D>
+__host__ __device__ constexpr bool schedule_ok() {
+  using W = WeightSchedule<D>;
+  if (W::kCPL % (2 * W::kStages) != 0) return false;
+  for (int p = 0; p < W::kCPL; ++p) {
+    const ChunkDesc c = W::chunk(p);
+    if (c.nrows < 16 || c.nrows > 256 || c.nrows % 16 != 0 || c.kcols % 16 != 0) return false;
+    if (c.bytes > W::kStageBytes || c.off % 16 != 0) return false;
+  }
+  return true;
+}
+static_assert(schedule_ok<32>() && schedule_ok<64>() && schedule_ok<128>(), "weight schedule");
 
 // Per-block parameter vector layout (floats), D = model width.
 struct LayerParamLayout {
@@ -55,10 +110,8 @@ struct DecodeParams {
   uint8_t *syn;
   float *logits;
   // model (device)
-  const uint8_t *wstream;  // bf16 weight chunks, block after block
-  uint32_t layer_bytes;
-  int n_chunks;
-  ChunkDesc chunks[kMaxChunks];
+  const uint8_t *wstream;  // bf16 weight chunks in WeightSchedule<D> order, block after block
+  uint32_t layer_bytes;    // WeightSchedule<D>::kLayerBytes
   const float *lparams;  // [n_layers][LayerParamLayout::stride(D)]
   const float *emb;      // [T][D - d_spe]
   const float *spe;      // [T][d_spe]
@@ -114,7 +167,8 @@ struct SmemLayout {
   __host__ __device__ static constexpr uint32_t align1k(uint32_t v) { return (v + 1023u) & ~1023u; }
   static constexpr uint32_t kRegionU = align1k(kKvBytes > kUqBytes ? kKvBytes : kUqBytes);
   static constexpr uint32_t kAopBytes = kRows * D * 2u;  // QKV / O / FFN1 operand: 128 x D bf16
-  static constexpr int kStages = (D == 128) ? 3 : 4;
+  static constexpr int kStages = WeightSchedule<D>::kStages;
+  static constexpr uint32_t kStageBytes = WeightSchedule<D>::kStageBytes;
   static constexpr uint32_t kOffU = 0;
   static constexpr uint32_t kOffAop = kRegionU;
   static constexpr uint32_t kOffW = align1k(kOffAop + kAopBytes);
@@ -122,8 +176,8 @@ struct SmemLayout {
   static constexpr uint32_t kOffZ = kOffRed + 4096;                   // 128 floats
   static constexpr uint32_t kOffObits = kOffZ + 512;                  // decoded bits
   static constexpr uint32_t kOffBar = kOffObits + kOutBitsBytes;      // mbarriers
-  static constexpr uint32_t kOffMisc = kOffBar + 256;  // tmem base, abort flag, peer bases, issue table
-  static constexpr uint32_t kTotal = kOffMisc + 1024;
+  static constexpr uint32_t kOffMisc = kOffBar + 256;  // tmem base, abort flag, peer bases, copy count
+  static constexpr uint32_t kTotal = kOffMisc + 256;
   static constexpr uint32_t kTmemCols = 4u * D;
 };
 

@@ -40,7 +40,7 @@ struct aecct_handle {
   uint8_t *wstream = nullptr;
   uint32_t layer_bytes = 0;
   int n_chunks = 0;
-  ChunkDesc chunks[kMaxChunks] = {};
+  ChunkDesc chunks[32] = {};  // WeightSchedule<d> order
   float *lparams = nullptr, *emb = nullptr, *spe = nullptr, *w_d1 = nullptr, *w_out = nullptr, *b_out = nullptr;
   uint32_t *hrow_off = nullptr, *mask_info[2] = {nullptr, nullptr};
   uint16_t *hrow_idx = nullptr, *mask_list[2] = {nullptr, nullptr};
@@ -156,6 +156,18 @@ inline int8_t tern(uint8_t code) { return code == 1 ? 1 : (code == 3 ? -1 : 0); 
 struct Gemm {
   int N, K;
 };
+
+// the chunks of one block in the order the kernel streams them (WeightSchedule<D>)
+template <int D>
+int schedule_chunks_t(ChunkDesc *out) {
+  using W = WeightSchedule<D>;
+  static_assert(W::kCPL <= 32, "chunk table");
+  for (int c = 0; c < W::kCPL; ++c) out[c] = W::chunk(c);
+  return W::kCPL;
+}
+int schedule_chunks(int D, ChunkDesc *out) {
+  return D == 32 ? schedule_chunks_t<32>(out) : D == 64 ? schedule_chunks_t<64>(out) : schedule_chunks_t<128>(out);
+}
 
 }  // namespace
 
@@ -386,25 +398,8 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
 
   // ---- weights: 2-bit codes -> bf16 K-major core-matrix chunks, in the order the MMA consumes them
   const Gemm gemms[4] = {{3 * D, D}, {D, D}, {F, D}, {D, F}};
-  int nch = 0;
-  uint32_t off = 0;
-  for (int g = 0; g < 4; ++g) {
-    const int KB = gemms[g].K < 64 ? gemms[g].K : 64;
-    for (int n0 = 0; n0 < gemms[g].N; n0 += 128) {
-      const int NB = (gemms[g].N - n0) < 128 ? (gemms[g].N - n0) : 128;
-      for (int k0 = 0; k0 < gemms[g].K; k0 += KB) {
-        ChunkDesc &c = h->chunks[nch++];
-        c.off = off;
-        c.bytes = static_cast<uint32_t>(NB * KB * 2);
-        c.gemm = static_cast<uint16_t>(g);
-        c.n0 = static_cast<uint16_t>(n0);
-        c.nrows = static_cast<uint16_t>(NB);
-        c.k0 = static_cast<uint16_t>(k0);
-        c.kcols = static_cast<uint16_t>(KB);
-        off += c.bytes;
-      }
-    }
-  }
+  const int nch = schedule_chunks(D, h->chunks);
+  const uint32_t off = h->chunks[nch - 1].off + h->chunks[nch - 1].bytes;
   h->n_chunks = nch;
   h->layer_bytes = off;
   std::vector<uint16_t> ws((size_t)d.n_layers * off / 2, 0);
@@ -525,8 +520,7 @@ int aecct_decode(aecct_handle *h, const float *y_dev, int64_t B, uint8_t *bits_d
   p.n_groups = (B + h->G - 1) / h->G;
   p.n_clusters = static_cast<int>(p.n_groups < h->max_clusters ? p.n_groups : h->max_clusters);
   p.y = y_dev, p.bits = bits_dev, p.syn = syndrome_dev, p.logits = logits_dev;
-  p.wstream = h->wstream, p.layer_bytes = h->layer_bytes, p.n_chunks = h->n_chunks;
-  std::memcpy(p.chunks, h->chunks, sizeof(p.chunks));
+  p.wstream = h->wstream, p.layer_bytes = h->layer_bytes;
   p.lparams = h->lparams, p.emb = h->emb, p.spe = h->spe, p.w_d1 = h->w_d1, p.b_d1 = h->b_d1;
   p.w_out = h->w_out, p.b_out = h->b_out, p.hrow_off = h->hrow_off, p.hrow_idx = h->hrow_idx;
   p.perm = h->perm, p.pos = h->pos;

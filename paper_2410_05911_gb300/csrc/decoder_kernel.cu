@@ -14,10 +14,11 @@
 //          Quant -> MMA FFN2 -> dequant + residual + LayerNorm
 //   S9/S10 (Sec. 3)        output head, hard decisions, syndrome of the decoded word
 //
-// Warp roles (576 threads): warps 0-15 do all CUDA-core work; thread (warp w, lane i) owns
-// token row 32*(w%4) + i (the TMEM lane quadrant its warp may read) and column slice w/4;
-// warp 16 streams weight chunks from global memory into a ring of shared-memory stages
-// with the bulk-copy (TMA) engine; warp 17 issues the tensor-core MMAs.
+// Warp roles (512 threads): warps 0-15 do all CUDA-core work; thread (warp w, lane i) owns
+// token row 32*(w%4) + i (the TMEM lane quadrant its warp may read) and column slice w/4.
+// Between its CUDA-core steps, warp 0 also streams the block weights from global memory into
+// a ring of shared-memory stages with the bulk-copy (TMA) engine and issues the tensor-core
+// MMAs, in a compile-time schedule (WeightSchedule).
 //
 // Every floating-point step uses one fixed order of IEEE fp32 operations (explicit _rn
 // intrinsics, pairwise feature sums, two-pass base-2 softmax with a Taylor-series exp2), so
@@ -471,117 +472,101 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
 // ------------------------------------------------------------------------------------------
 // weight streaming and tensor-core issue (run by warp 0 of each CTA)
 // ------------------------------------------------------------------------------------------
-// Weight chunks are consumed in a fixed sequence: for each group of codewords, for each block,
-// the block's chunks (QKV, then O, FFN1, FFN2).  Chunk i of the sequence uses ring stage i % S;
-// its copy completes phase i / S of full[stage], its MMAs release phase i / S of empty[stage].
-// Positions advance incrementally (no integer division on the issuing warp).
-
-// What the issuing warp reads for every chunk, copied once into shared memory.
-struct IssueTable {
-  ChunkDesc chunks[kMaxChunks];
-  const uint8_t *wstream;
-  uint32_t layer_bytes;
-  int n_chunks;
-  int n_layers;
-  int pad;
-};
-
-// Progress of the weight-chunk ring and of the MMA chain.  Warp 0 issues both; every lane of it
-// holds the same copy of this state.
-struct IssueState {
-  int64_t total;   // chunks this CTA consumes
-  int64_t issued;  // chunks whose copy has been started
-  int64_t used;    // chunks whose MMAs have been issued
-  int cs, cc, cl;  // next copy: ring stage, chunk of the block, block
-  uint32_t cround; // next copy: number of completed passes over the ring
-  int ms, mc;      // next MMA: ring stage, chunk of the block
-  uint32_t mround; // next MMA: passes over the ring
-  uint32_t oph;    // parity of the next operand-ready phase
-  uint32_t aph;    // parity of the next accumulator-ready phase
-};
-
-// Start the copy of the next chunk into its ring stage (waiting for the stage's previous MMAs).
+// Chunk p of a block lives in stage p % S and completes phase parity (p / S) & 1 of full[stage]
+// (and, D = 128, of empty[stage]); the operand-ready and accumulator-ready barriers complete one
+// phase per GEMM, four per block, so GEMM g always waits for parity g & 1.  Everything the issue
+// path computes is therefore a compile-time constant or a warp-uniform base address, and the
+// tcgen05 instructions take their operands straight from uniform registers.
 template <int D, bool TASKS>
-__device__ __forceinline__ void copy_next(const IssueTable &p, const Ctl ctl, IssueState &st, uint32_t sb) {
+struct Issuer {
   using L = SmemLayout<D, TASKS>;
-  constexpr int S = L::kStages;
-  const uint32_t bar_full = sb + L::kOffBar, bar_empty = bar_full + 8 * S;
-  if (st.cround > 0) wait_bar_warp(ctl, bar_empty + 8 * st.cs, (st.cround - 1u) & 1u, false);
-  const ChunkDesc &ch = p.chunks[st.cc];
-  bulk_g2s_expect_warp(sb + L::kOffW + st.cs * kStageBytes, p.wstream + (size_t)st.cl * p.layer_bytes + ch.off,
-                       ch.bytes, bar_full + 8 * st.cs);
-  ++st.issued;
-  if (++st.cs == S) st.cs = 0, ++st.cround;
-  if (++st.cc == p.n_chunks) {
-    st.cc = 0;
-    if (++st.cl == p.n_layers) st.cl = 0;
-  }
-}
+  using W = WeightSchedule<D>;
+  static constexpr int S = W::kStages;
+  static constexpr int CPL = W::kCPL;
+  // some GEMM has more chunks than stages (D = 128): every chunk then releases its stage through
+  // empty[stage], so that chunk p always completes phase parity (p / S) & 1 there
+  static constexpr bool kRefillInGemm =
+      W::count(0) > S || W::count(1) > S || W::count(2) > S || W::count(3) > S;
+  uint32_t sb, tmem;
+  Ctl ctl;
+  uint32_t *n_issued;  // copies started so far (read by the teardown drain)
 
-// Keep up to S chunks in flight ahead of the MMAs (whole warp 0).
-template <int D, bool TASKS>
-__device__ __forceinline__ void issue_copies_reg(const IssueTable &p, const Ctl ctl, IssueState &st, uint32_t sb) {
-  constexpr int S = SmemLayout<D, TASKS>::kStages;
-  while (st.issued < st.total && st.issued < st.used + S) {
-    if (*ctl.abort) return;
-    copy_next<D, TASKS>(p, ctl, st, sb);
-  }
-}
-// The issue state lives in shared memory between calls (a local-memory copy would miss the small
-// L1 left beside the shared-memory carve-out); each call works on a register copy.
-template <int D, bool TASKS>
-__device__ __forceinline__ void issue_copies(const IssueTable &p, const Ctl ctl, IssueState *sst, uint32_t sb) {
-  IssueState st = *sst;
-  issue_copies_reg<D, TASKS>(p, ctl, st, sb);
-  *sst = st;
-}
+  __device__ __forceinline__ uint32_t bar_full(int s) const { return sb + L::kOffBar + 8 * s; }
+  __device__ __forceinline__ uint32_t bar_empty(int s) const { return sb + L::kOffBar + 8 * (S + s); }
+  __device__ __forceinline__ uint32_t bar_op() const { return sb + L::kOffBar + 16 * S; }
+  __device__ __forceinline__ uint32_t bar_acc() const { return sb + L::kOffBar + 16 * S + 8; }
 
-// Whole warp 0: wait until every warp has published the operand of GEMM `gemm`, issue its
-// tcgen05.mma chain (accumulators at TMEM column 0), wait for its completion, then prefetch the
-// next chunks.
-template <int D, bool TASKS>
-__device__ __forceinline__ void issue_gemm(const IssueTable &p, const Ctl ctl, IssueState *sst, int gemm, uint32_t sb,
-                                        uint32_t tmem) {
-  using L = SmemLayout<D, TASKS>;
-  IssueState st = *sst;
-  constexpr int S = L::kStages;
-  const uint32_t bar_full = sb + L::kOffBar, bar_empty = bar_full + 8 * S;
-  const uint32_t bar_op = bar_empty + 8 * S, bar_acc = bar_op + 8;
-  wait_bar_warp(ctl, bar_op, st.oph, false);
-  st.oph ^= 1u;
-  tc_fence_after();
-  const uint32_t a_tile = (gemm == 3) ? (sb + L::kOffU) : (sb + L::kOffAop);
-  const uint32_t a_sbo = (gemm == 3) ? (4u * D / 8u) * 128u : (D / 8u) * 128u;
-  while (st.used < st.total) {
-    const ChunkDesc ch = p.chunks[st.mc];
-    if (ch.gemm != gemm) break;
-    if (st.issued == st.used) copy_next<D, TASKS>(p, ctl, st, sb);
-    wait_bar_warp(ctl, bar_full + 8 * st.ms, st.mround & 1u, false);
+  // whole warp: lane 0 polls (the slow path is bounded and raises the abort flag), then the
+  // warp reconverges
+  __device__ __forceinline__ void wait(uint32_t bar, uint32_t parity) const {
+    if ((threadIdx.x & 31) == 0 && !mbar_try_wait(bar, parity)) wait_bar_slow(ctl, bar, parity, false);
+    __syncwarp();
+  }
+  // start the copy of chunk p of the block whose weights start at `src`
+  __device__ __forceinline__ void copy(int p, const uint8_t *src) const {
+    const ChunkDesc c = W::chunk(p);
+    bulk_g2s_expect_warp(sb + L::kOffW + (p % S) * W::kStageBytes, src + c.off, c.bytes, bar_full(p % S));
+    if ((threadIdx.x & 31) == 0) ++*n_issued;
+  }
+  // chunks 0 .. S-1 of the first block
+  __device__ __forceinline__ void prologue(const uint8_t *w0) const {
+#pragma unroll
+    for (int p = 0; p < S; ++p) copy(p, w0);
+  }
+  // Wait until every warp has published the operand of GEMM G, issue its tcgen05.mma chain
+  // (accumulators at TMEM column 0), wait for its completion, then start the copies of the
+  // chunks that follow the freed stages: chunk p + S of this block, or chunk p + S - CPL of the
+  // next block (`w_next`, when `has_next`).
+  template <int G>
+  __device__ __forceinline__ void gemm(const uint8_t *w_cur, const uint8_t *w_next, bool has_next) const {
+    constexpr int first = W::first(G), count = W::count(G);
+    constexpr uint32_t a_tile = (G == 3) ? L::kOffU : L::kOffAop;
+    constexpr uint32_t a_sbo = (G == 3) ? (4u * D / 8u) * 128u : (D / 8u) * 128u;
+    wait(bar_op(), G & 1);
     tc_fence_after();
-    const uint32_t b_tile = sb + L::kOffW + st.ms * kStageBytes;
-    const uint32_t b_sbo = (ch.kcols / 8u) * 128u;
-    const uint32_t idesc = make_idesc_bf16(128, ch.nrows);
-    for (int ks = 0; ks < ch.kcols / 16; ++ks) {
-      const uint32_t kabs = ch.k0 + 16u * ks;
-      const uint64_t ad = make_sdesc(a_tile + (kabs / 8u) * 128u, 128u, a_sbo);
-      const uint64_t bd = make_sdesc(b_tile + ks * 256u, 128u, b_sbo);
-      mma_bf16_warp(tmem + ch.n0, ad, bd, idesc, kabs > 0 ? 1u : 0u);
+#pragma unroll
+    for (int j = 0; j < count; ++j) {
+      const int p = first + j;
+      const ChunkDesc c = W::chunk(p);
+      if (j >= S) {
+        // this block's GEMM has more chunks than stages (D = 128): reuse the stage of chunk
+        // p - S once its MMAs are done
+        wait(bar_empty((p - S) % S), ((p - S) / S) & 1);
+        copy(p, w_cur);
+      }
+      wait(bar_full(p % S), (p / S) & 1);
+      const uint32_t b_tile = sb + L::kOffW + (p % S) * W::kStageBytes;
+      const uint32_t b_sbo = (c.kcols / 8u) * 128u;
+      const uint32_t idesc = make_idesc_bf16(128, c.nrows);
+#pragma unroll
+      for (int ks = 0; ks < c.kcols / 16; ++ks) {
+        const uint32_t kabs = c.k0 + 16u * ks;
+        mma_bf16_warp(tmem + c.n0, make_sdesc(sb + a_tile + (kabs / 8u) * 128u, 128u, a_sbo),
+                      make_sdesc(b_tile + ks * 256u, 128u, b_sbo), idesc, kabs > 0 ? 1u : 0u);
+      }
+      if (kRefillInGemm) mma_commit_warp(bar_empty(p % S));
     }
-    mma_commit_warp(bar_empty + 8 * st.ms);
-    ++st.used;
-    if (++st.ms == S) st.ms = 0, ++st.mround;
-    if (++st.mc == p.n_chunks) st.mc = 0;
+    mma_commit_warp(bar_acc());
+    // warp 0 alone waits for the accumulators; the other warps of the CTA wait in a named
+    // barrier (no spinning), which warp 0 joins after the wait
+    wait(bar_acc(), G & 1);
+    // every MMA so far is complete, so the stages they read are free
+#pragma unroll
+    for (int q = (count > S ? first + count : first + S); q < first + count + S; ++q) {
+      if (q < CPL) copy(q, w_cur);
+      else if (has_next) copy(q - CPL, w_next);
+    }
   }
-  mma_commit_warp(bar_acc);
-  // warp 0 alone waits for the accumulators; the other warps of the CTA wait in a named barrier
-  // (no spinning), which warp 0 joins after the wait
-  wait_bar_warp(ctl, bar_acc, st.aph, false);
-  st.aph ^= 1u;
-  // every MMA so far is complete, so the stages they read are free: prefetch the next chunks
-  issue_copies_reg<D, TASKS>(p, ctl, st, sb);
-  *sst = st;
-}
-
+  // every copy started has landed (bounded waits that ignore the abort flag)
+  __device__ __forceinline__ void drain() const {
+    const uint32_t n = *n_issued;
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+      const uint32_t cnt = (n + S - 1 - s) / S;  // copies that went to stage s
+      if (cnt > 0) wait_bar_drain(ctl, bar_full(s), (cnt - 1u) & 1u);
+    }
+  }
+};
 // ------------------------------------------------------------------------------------------
 // the kernel
 // ------------------------------------------------------------------------------------------
@@ -611,9 +596,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   volatile int *s_abort = reinterpret_cast<volatile int *>(smem + L::kOffMisc + 4);
   uint64_t *s_kvgen = reinterpret_cast<uint64_t *>(smem + L::kOffMisc + 8);  // [8] generic K/V bases per CTA
   uint64_t *s_zgen = reinterpret_cast<uint64_t *>(smem + L::kOffMisc + 72);   // [8] generic z bases per CTA
-  IssueTable *s_itab = reinterpret_cast<IssueTable *>(smem + L::kOffMisc + 256);
-  IssueState *s_ist = reinterpret_cast<IssueState *>(smem + L::kOffMisc + 256 + sizeof(IssueTable));
-  static_assert(256 + sizeof(IssueTable) + sizeof(IssueState) <= L::kTotal - L::kOffMisc, "misc area too small");
+  uint32_t *s_issued = reinterpret_cast<uint32_t *>(smem + L::kOffMisc + 136);  // weight copies started
 
   if (tid == 0) {
     for (int s = 0; s < S; ++s) {
@@ -628,11 +611,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
     mbar_init(bar_zf, p.C);
     mbar_init(bar_fin, 1);
     *s_abort = 0;
-    for (int c = 0; c < kMaxChunks; ++c) s_itab->chunks[c] = p.chunks[c];
-    s_itab->wstream = p.wstream;
-    s_itab->layer_bytes = p.layer_bytes;
-    s_itab->n_chunks = p.n_chunks;
-    s_itab->n_layers = p.n_layers;
+    *s_issued = 0;
     // generic base of the K/V and z areas of every CTA of the cluster: this CTA's own area through
     // its plain shared-memory window, the others through the distributed shared window
     for (int c = 0; c < p.C; ++c) {
@@ -653,15 +632,8 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   const uint32_t tmem = *s_tmem;
   const Ctl ctl{s_abort, p.err, p.wait_limit};
 
-  if (warp == 0) {
-    if (lane == 0) {
-      IssueState st{};
-      st.total = (p.n_groups - cluster_id + p.n_clusters - 1) / p.n_clusters * p.n_layers * p.n_chunks;
-      *s_ist = st;
-    }
-    __syncwarp();
-    issue_copies<D, TASKS>(*s_itab, ctl, s_ist, sb);
-  }
+  const Issuer<D, TASKS> issuer{sb, tmem, ctl, s_issued};
+  if (warp == 0 && cluster_id < p.n_groups) issuer.prologue(p.wstream);
   {
     // ------------------------------------------------------------ CUDA-core warps
     const int qd = warp & 3, sl = warp >> 2;
@@ -695,14 +667,24 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
       red.sel ^= 1;
       return a;
     };
-    // publish this warp's part of the operand of `gemm`; warp 0 then issues the GEMM
-    auto signal_op = [&](int gemm) {
+    // publish this warp's part of the operand of GEMM `gemm` of block `blk` of group `gi`;
+    // warp 0 then issues the GEMM and prefetches the weights that follow it
+    auto signal_op = [&](int gemm, int blk, int64_t gi) {
       tc_fence_before();  // this thread's TMEM reads are ordered before the MMA the arrive releases
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) mbar_arrive(bar_op);
       __syncwarp();
-      if (warp == 0) issue_gemm<D, TASKS>(*s_itab, ctl, s_ist, gemm, sb, tmem);
+      if (warp == 0) {
+        const bool last_blk = blk + 1 == p.n_layers;
+        const uint8_t *w_cur = p.wstream + static_cast<size_t>(blk) * p.layer_bytes;
+        const uint8_t *w_next = last_blk ? p.wstream : w_cur + p.layer_bytes;
+        const bool has_next = !last_blk || gi + p.n_clusters < p.n_groups;
+        if (gemm == 0) issuer.template gemm<0>(w_cur, w_next, has_next);
+        if (gemm == 1) issuer.template gemm<1>(w_cur, w_next, has_next);
+        if (gemm == 2) issuer.template gemm<2>(w_cur, w_next, has_next);
+        if (gemm == 3) issuer.template gemm<3>(w_cur, w_next, has_next);
+      }
     };
     auto cluster_arrive = [&](uint32_t bar) {
       // all 512 CUDA-core threads of this CTA are past their accesses: tell every CTA
@@ -819,7 +801,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           capture_q(0, 0, qv, sl * XS, XS, alpha_in);
         }
       }
-      signal_op(0);
+      signal_op(0, 0, gi);
 
       for (int l = 0; l < p.n_layers; ++l) {
         const float *lp = p.lparams + (size_t)l * LP::stride(D);
@@ -970,7 +952,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             }
           }
         }
-        signal_op(1);
+        signal_op(1, l, gi);
         if constexpr (!TASKS) cluster_arrive(bar_kvf);  // this CTA no longer reads any K/V of this block
 
         // ---------------- S6: O projection + residual + LayerNorm (Sec. 5, Post-LN)
@@ -992,7 +974,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             capture_q(l, 2, qv, sl * XS, XS, alpha_in);
           }
         }
-        signal_op(2);
+        signal_op(2, l, gi);
 
         // ---------------- S7: FFN1 + ReLU (Sec. 4 item 4), Quant(u) -> FFN2 operand
         wait_acc();
@@ -1046,7 +1028,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             if (cap) capture_q(l, 3, qv, c0, 32, alpha_in);
           }
         }
-        signal_op(3);
+        signal_op(3, l, gi);
 
         // ---------------- S8: FFN2 + residual + LayerNorm
         wait_acc();
@@ -1065,7 +1047,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             codes<XS>(x, rr, qv);
             capture_q(l + 1, 0, qv, sl * XS, XS, alpha_in);
           }
-          signal_op(0);
+          signal_op(0, l + 1, gi);
         }
       }
 
@@ -1131,9 +1113,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
     mma_commit_warp(bar_fin);
     if (lane == 0) {
       wait_bar_drain(ctl, bar_fin, 0);
-      const int64_t issued = s_ist->issued;
-      for (int64_t i = issued - S; i < issued; ++i)
-        if (i >= 0) wait_bar_drain(ctl, bar_full + 8 * static_cast<int>(i % S), static_cast<uint32_t>((i / S) & 1));
+      issuer.drain();
     }
     __syncwarp();
   }
