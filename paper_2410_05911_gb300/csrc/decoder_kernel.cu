@@ -502,16 +502,58 @@ struct Issuer {
     if ((threadIdx.x & 31) == 0 && !mbar_try_wait(bar, parity)) wait_bar_slow(ctl, bar, parity, false);
     __syncwarp();
   }
-  // start the copy of chunk p of the block whose weights start at `src`
-  __device__ __forceinline__ void copy(int p, const uint8_t *src) const {
-    const ChunkDesc c = W::chunk(p);
-    bulk_g2s_expect_warp(sb + L::kOffW + (p % S) * W::kStageBytes, src + c.off, c.bytes, bar_full(p % S));
+  // start the copy of chunk P of the block whose weights start at `src` (P is a template
+  // parameter so that the chunk's geometry is evaluated at compile time)
+  template <int P>
+  __device__ __forceinline__ void copy(const uint8_t *src) const {
+    constexpr ChunkDesc c = W::chunk(P);
+    bulk_g2s_expect_warp(sb + L::kOffW + (P % S) * W::kStageBytes, src + c.off, c.bytes, bar_full(P % S));
     if ((threadIdx.x & 31) == 0) ++*n_issued;
   }
   // chunks 0 .. S-1 of the first block
+  template <int P = 0>
   __device__ __forceinline__ void prologue(const uint8_t *w0) const {
+    if constexpr (P < S) {
+      copy<P>(w0);
+      prologue<P + 1>(w0);
+    }
+  }
+  // chunk J of GEMM G: (reuse a stage if the GEMM has more chunks than stages,) wait for the
+  // weights, issue the MMAs over the chunk's K range, release the stage
+  template <int G, int J>
+  __device__ __forceinline__ void chunk_mmas(const uint8_t *w_cur) const {
+    if constexpr (J < W::count(G)) {
+      constexpr int p = W::first(G) + J;
+      constexpr ChunkDesc c = W::chunk(p);
+      constexpr uint32_t a_tile = (G == 3) ? L::kOffU : L::kOffAop;
+      constexpr uint32_t a_sbo = (G == 3) ? (4u * D / 8u) * 128u : (D / 8u) * 128u;
+      constexpr uint32_t b_sbo = (c.kcols / 8u) * 128u;
+      constexpr uint32_t idesc = make_idesc_bf16(128, c.nrows);
+      if constexpr (J >= S) {
+        // reuse the stage of chunk p - S (same GEMM) once its MMAs are done
+        wait(bar_empty((p - S) % S), ((p - S) / S) & 1);
+        copy<p>(w_cur);
+      }
+      wait(bar_full(p % S), (p / S) & 1);
+      const uint32_t b_tile = sb + L::kOffW + (p % S) * W::kStageBytes;
 #pragma unroll
-    for (int p = 0; p < S; ++p) copy(p, w0);
+      for (int ks = 0; ks < c.kcols / 16; ++ks) {
+        const uint32_t kabs = c.k0 + 16u * ks;
+        mma_bf16_warp(tmem + c.n0, make_sdesc(sb + a_tile + (kabs / 8u) * 128u, 128u, a_sbo),
+                      make_sdesc(b_tile + ks * 256u, 128u, b_sbo), idesc, kabs > 0 ? 1u : 0u);
+      }
+      if constexpr (kRefillInGemm) mma_commit_warp(bar_empty(p % S));
+      chunk_mmas<G, J + 1>(w_cur);
+    }
+  }
+  // copies of chunks Q .. QEND-1 (positions past the block continue in the next block)
+  template <int Q, int QEND>
+  __device__ __forceinline__ void refill(const uint8_t *w_cur, const uint8_t *w_next, bool has_next) const {
+    if constexpr (Q < QEND) {
+      if constexpr (Q < CPL) copy<Q>(w_cur);
+      else if (has_next) copy<Q - CPL>(w_next);
+      refill<Q + 1, QEND>(w_cur, w_next, has_next);
+    }
   }
   // Wait until every warp has published the operand of GEMM G, issue its tcgen05.mma chain
   // (accumulators at TMEM column 0), wait for its completion, then start the copies of the
@@ -520,42 +562,15 @@ struct Issuer {
   template <int G>
   __device__ __forceinline__ void gemm(const uint8_t *w_cur, const uint8_t *w_next, bool has_next) const {
     constexpr int first = W::first(G), count = W::count(G);
-    constexpr uint32_t a_tile = (G == 3) ? L::kOffU : L::kOffAop;
-    constexpr uint32_t a_sbo = (G == 3) ? (4u * D / 8u) * 128u : (D / 8u) * 128u;
     wait(bar_op(), G & 1);
     tc_fence_after();
-#pragma unroll
-    for (int j = 0; j < count; ++j) {
-      const int p = first + j;
-      const ChunkDesc c = W::chunk(p);
-      if (j >= S) {
-        // this block's GEMM has more chunks than stages (D = 128): reuse the stage of chunk
-        // p - S once its MMAs are done
-        wait(bar_empty((p - S) % S), ((p - S) / S) & 1);
-        copy(p, w_cur);
-      }
-      wait(bar_full(p % S), (p / S) & 1);
-      const uint32_t b_tile = sb + L::kOffW + (p % S) * W::kStageBytes;
-      const uint32_t b_sbo = (c.kcols / 8u) * 128u;
-      const uint32_t idesc = make_idesc_bf16(128, c.nrows);
-#pragma unroll
-      for (int ks = 0; ks < c.kcols / 16; ++ks) {
-        const uint32_t kabs = c.k0 + 16u * ks;
-        mma_bf16_warp(tmem + c.n0, make_sdesc(sb + a_tile + (kabs / 8u) * 128u, 128u, a_sbo),
-                      make_sdesc(b_tile + ks * 256u, 128u, b_sbo), idesc, kabs > 0 ? 1u : 0u);
-      }
-      if (kRefillInGemm) mma_commit_warp(bar_empty(p % S));
-    }
+    chunk_mmas<G, 0>(w_cur);
     mma_commit_warp(bar_acc());
     // warp 0 alone waits for the accumulators; the other warps of the CTA wait in a named
     // barrier (no spinning), which warp 0 joins after the wait
     wait(bar_acc(), G & 1);
     // every MMA so far is complete, so the stages they read are free
-#pragma unroll
-    for (int q = (count > S ? first + count : first + S); q < first + count + S; ++q) {
-      if (q < CPL) copy(q, w_cur);
-      else if (has_next) copy(q - CPL, w_next);
-    }
+    refill<(count > S ? first + count : first + S), first + count + S>(w_cur, w_next, has_next);
   }
   // every copy started has landed (bounded waits that ignore the abort flag)
   __device__ __forceinline__ void drain() const {
