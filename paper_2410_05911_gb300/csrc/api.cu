@@ -208,18 +208,19 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
   } else if (d.attention_mode == 0) {
     tasks = task_ok;
   }
-  // choose the number of CTAs that share a group: densest packing of T-token words over C x 128 rows
+  // choose the number of CTAs that share a group: by default the fewest that hold one codeword
+  // (an attention read of a key held by another CTA of the cluster costs far more than the
+  // token rows left idle by a looser packing), with as many words per group as fit; an explicit
+  // cluster_ctas is honoured when it can hold a word
   int best_C = 0, best_G = 0;
-  double best_eff = -1.0;
   const int cmin = (T + kRows - 1) / kRows;
-  for (int C = cmin; C <= kMaxCluster; ++C) {
+  for (int C = cmin; C <= kMaxCluster && !best_C; ++C) {
     if (tasks && C != 1) continue;
     if (d.cluster_ctas && C != d.cluster_ctas) continue;
     const int G = (C * kRows) / T;
     if (G < 1) continue;
     if (((G + C - 1) / C) * n > kOutBitsBytes) continue;
-    const double eff = static_cast<double>(G * T) / (C * kRows);
-    if (eff > best_eff + 1e-9) best_eff = eff, best_C = C, best_G = G;
+    best_C = C, best_G = G;
   }
   if (!best_C) return d.cluster_ctas ? AECCT_ERR_INVALID_ARG : AECCT_ERR_UNSUPPORTED;
 
