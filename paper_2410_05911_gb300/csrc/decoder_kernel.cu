@@ -350,7 +350,8 @@ __device__ __forceinline__ int byte_at(const uint4 &w, int k) {
 // computations, and the folds into l and num stay sequential in key order.
 template <int DH, uint32_t STRIDE>
 __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int cnt, const uint4 *__restrict__ ul,
-                                          const uint8_t *rows, uint32_t kslot, float scale, float *A) {
+                                          const uint8_t *rows, uint32_t kslot, float scale, uint32_t tcache,
+                                          float *A) {
   auto kptr = [&](int off) { return reinterpret_cast<const float4 *>(rows + off * STRIDE + kslot); };
   // dot products of q with two keys: lane x for key a, lane y for key b (FMA chains in feature order)
   auto dot2 = [&](const float4 *ka, const float4 *kb) -> float2 {
@@ -371,12 +372,15 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
     const uint32_t word = jb < 64 ? (jb < 32 ? mask.x : mask.y) : (jb < 96 ? mask.z : mask.w);
     return word >> (jb & 16);
   };
-  // pass 1: maximum score over the lane's keys
+  // pass 1: maximum score over the lane's keys.  The scores sigma = fl(dot * scale) of the first
+  // kTaskCache keys also go to this warp's TMEM columns, so that pass 2 reads them back
+  // instead of reloading K and recomputing the dot products (same values, bit for bit).
   float mx = -INFINITY;
   for (int jb = 0; jb < cnt; jb += 16) {
     const uint4 w = __ldg(ul + (jb >> 4));
     const uint32_t seg = segment(jb);
     const int nk = min(16, cnt - jb);
+    float sgs[16];
     if (nk == 16) {
 #pragma unroll
       for (int k0 = 0; k0 < 16; k0 += U) {
@@ -390,23 +394,32 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
 #pragma unroll
         for (int k = 0; k < U; k += 2) {
           const float2 sg = mul2(dot2(kk[k], kk[k + 1]), sc);
+          sgs[k0 + k] = sg.x, sgs[k0 + k + 1] = sg.y;
           if (((seg >> (k0 + k)) & 1u)) mx = fmaxf(mx, sg.x);
           if (((seg >> (k0 + k + 1)) & 1u)) mx = fmaxf(mx, sg.y);
         }
       }
     } else {
-      for (int k = 0; k < nk; k += 2) {
-        const int k1 = (k + 1 < nk) ? k + 1 : k;
-        float4 ka[DH / 4], kb[DH / 4];
-        const float4 *pa = kptr(byte_at(w, k)), *pb = kptr(byte_at(w, k1));
 #pragma unroll
-        for (int i = 0; i < DH / 4; ++i) ka[i] = pa[i], kb[i] = pb[i];
-        const float2 sg = mul2(dot2(ka, kb), sc);
-        if (((seg >> k) & 1u)) mx = fmaxf(mx, sg.x);
-        if (k1 != k && ((seg >> k1) & 1u)) mx = fmaxf(mx, sg.y);
+      for (int k = 0; k < 16; k += 2) {
+        if (k < nk) {
+          const int k1 = (k + 1 < nk) ? k + 1 : k;
+          float4 ka[DH / 4], kb[DH / 4];
+          const float4 *pa = kptr(byte_at(w, k)), *pb = kptr(byte_at(w, k1));
+#pragma unroll
+          for (int i = 0; i < DH / 4; ++i) ka[i] = pa[i], kb[i] = pb[i];
+          const float2 sg = mul2(dot2(ka, kb), sc);
+          sgs[k] = sg.x, sgs[k + 1] = sg.y;
+          if (((seg >> k) & 1u)) mx = fmaxf(mx, sg.x);
+          if (k1 != k && ((seg >> k1) & 1u)) mx = fmaxf(mx, sg.y);
+        } else {
+          sgs[k] = 0.0f, sgs[k + 1] = 0.0f;
+        }
       }
     }
+    if (jb < kTaskCache) tmem_st<16>(tcache + jb, sgs);
   }
+  tmem_wait_st();
   // pass 2: p = 2^(sigma - m), l += p, num += p v, in key order
   float lsum = 0.0f;
   float num[DH];
@@ -430,7 +443,32 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
     const uint4 w = __ldg(ul + (jb >> 4));
     const uint32_t seg = segment(jb);
     const int nk = min(16, cnt - jb);
-    if (nk == 16) {
+    if (jb < kTaskCache) {
+      float sgs[16];
+      tmem_ld<16>(tcache + jb, sgs);
+      tmem_wait_ld();
+#pragma unroll
+      for (int k0 = 0; k0 < 16; k0 += U) {
+        if (k0 < nk) {
+          float4 vv[U][DH / 4];
+#pragma unroll
+          for (int k = 0; k < U; ++k) {
+            const float4 *kp = kptr(byte_at(w, min(k0 + k, nk - 1)));
+#pragma unroll
+            for (int i = 0; i < DH / 4; ++i) vv[k][i] = kp[DH / 4 + i];
+          }
+          float2 pr[U / 2];
+#pragma unroll
+          for (int k = 0; k < U; k += 2)
+            pr[k / 2] = exp2_series2(make_float2(__fsub_rn(sgs[k0 + k], mx), __fsub_rn(sgs[k0 + k + 1], mx)));
+#pragma unroll
+          for (int k = 0; k < U; k += 2) {
+            if (k0 + k < nk && ((seg >> (k0 + k)) & 1u)) fold(pr[k / 2].x, vv[k]);
+            if (k0 + k + 1 < nk && ((seg >> (k0 + k + 1)) & 1u)) fold(pr[k / 2].y, vv[k + 1]);
+          }
+        }
+      }
+    } else if (nk == 16) {
 #pragma unroll
       for (int k0 = 0; k0 < 16; k0 += U) {
         float4 kk[U][DH / 4], vv[U][DH / 4];
@@ -701,9 +739,12 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         if (gemm == 3) issuer.template gemm<3>(w_cur, w_next, has_next);
       }
     };
+    // A cluster of one CTA needs no cluster-scope signal: the named barrier in cluster_arrive
+    // already orders every access of the CTA, so cluster_wait has nothing left to wait for.
     auto cluster_arrive = [&](uint32_t bar) {
       // all 512 CUDA-core threads of this CTA are past their accesses: tell every CTA
       named_bar_sync(5, kEpiThreads);
+      if (p.C == 1) return;
       if (tid == 0) {
         fence_acq_rel_cluster();
         for (int c = 0; c < p.C; ++c) mbar_arrive_cluster(mapa_cluster(bar, c));
@@ -718,6 +759,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
     };
     // wait for a cluster-wide phase: thread 0 waits on the mbarrier, the others in a named barrier
     auto cluster_wait = [&](uint32_t bar, uint32_t &ph) {
+      if (p.C == 1) return;
       if (tid == 0) wait_bar(ctl, bar, ph, true);
       ph ^= 1u;
       __syncwarp();
@@ -725,6 +767,18 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
     };
 
     for (int64_t gi = cluster_id; gi < p.n_groups; gi += p.n_clusters) {
+      // the group's channel outputs, in one coalesced pass, into the decoded-bits area (free
+      // until S10; G n < C x 128 floats fit); the next group's are prefetched into L2
+      float *ybuf = reinterpret_cast<float *>(obits);
+      {
+        const int64_t y0 = gi * p.G * n;
+        const int64_t ny = min(static_cast<int64_t>(p.G) * n, p.B * n - y0);
+        for (int i = tid; i < ny; i += kEpiThreads) ybuf[i] = __ldg(p.y + y0 + i);
+        const int64_t y1 = y0 + static_cast<int64_t>(p.n_clusters) * p.G * n;
+        const int64_t ny1 = min(static_cast<int64_t>(p.G) * n, p.B * n - y1);
+        for (int64_t i = static_cast<int64_t>(tid) * 32; i < ny1; i += kEpiThreads * 32)
+          asm volatile("prefetch.global.L2 [%0];" ::"l"(p.y + y1 + i));
+      }
       if (named_bar_or(5, kEpiThreads, *s_abort != 0)) break;
       const int rho = static_cast<int>(crank) * kRows + r;
       const int g = rho / T;
@@ -733,7 +787,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
       const bool row_cw = g < p.G;
       const bool valid = row_cw && b < p.B;
       const bool cap = valid && b < p.cap_B;
-      const float *yrow = p.y + (valid ? b : 0) * n;
+      const float *yrow = ybuf + (valid ? g : 0) * n;
 
       float x[XS];
       float alpha_in;
@@ -742,12 +796,12 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         float h = 0.0f;
         if (valid) {
           if (t < n) {
-            h = fabsf(__ldg(yrow + t));
+            h = fabsf(yrow[t]);
           } else {
             const int i = t - n;
             uint32_t par = 0;
             for (uint32_t e = __ldg(p.hrow_off + i); e < __ldg(p.hrow_off + i + 1); ++e)
-              par ^= (__ldg(yrow + __ldg(p.hrow_idx + e)) < 0.0f) ? 1u : 0u;
+              par ^= (yrow[__ldg(p.hrow_idx + e)] < 0.0f) ? 1u : 0u;
             h = __fsub_rn(1.0f, __fmul_rn(2.0f, static_cast<float>(par)));
             if (cap && sl == 0 && p.cap_syn) p.cap_syn[b * m + i] = static_cast<uint8_t>(par);
           }
@@ -867,6 +921,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         if constexpr (TASKS) {
           // ---------------- S5: HPSA (Sec. 4.2), task mode: warp tasks over query groups
           named_bar_sync(5, kEpiThreads);  // every Q, K, V row of this CTA is in shared memory
+          // this warp's score cache: its lane quadrant, kTaskCache columns of [kTaskCacheCol, 512)
+          static_assert(L::kTaskCacheCol >= 4u * D && L::kTaskCacheCol + 4u * kTaskCache <= L::kTmemCols, "TMEM");
+          const uint32_t tcache = tmem + (static_cast<uint32_t>(32 * (warp & 3)) << 16) + L::kTaskCacheCol +
+                                  static_cast<uint32_t>(warp >> 2) * kTaskCache;
           for (int k = 0; k < kMaxTasks; ++k) {
             const uint32_t task = __ldg(p.plan_task + warp * kMaxTasks + k);
             if (task == 0xFFFFu) break;
@@ -885,7 +943,8 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
               q[4 * i] = v.x, q[4 * i + 1] = v.y, q[4 * i + 2] = v.z, q[4 * i + 3] = v.w;
             }
             hpsa_task<DH, L::kKvStride>(q, mk, static_cast<int>(ui & 255u), p.plan_ulist + (ui >> 8),
-                                        smem + L::kOffU + gi.z * L::kKvStride, e * L::kSlot + 4 * DH, p.att_scale, a);
+                                        smem + L::kOffU + gi.z * L::kKvStride, e * L::kSlot + 4 * DH, p.att_scale,
+                                        tcache, a);
             if (act) {
               // A of (row, head e) replaces Q of (row, head e): this task was its only reader
               float4 *ap = reinterpret_cast<float4 *>(smem + L::kOffU + row * L::kKvStride + e * L::kSlot);
@@ -1082,21 +1141,36 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
       // ---------------- S10: decisions x_hat = y * eps, decoded-word syndrome
       {
         const int n_local = (p.G - static_cast<int>(crank) + p.C - 1) / p.C;  // groups g = crank + C*i
+        // z of this CTA's words in token order, gathered once (from peers' rows too) into the
+        // reduction area, which is idle until the next group (n_local T <= 1024 floats)
+        float *ztok = red.buf;
+        for (int it = tid; it < n_local * T; it += kEpiThreads) {
+          const int li = it / T, tt = it - li * T;
+          const int ru = (static_cast<int>(crank) + li * p.C) * T + __ldg(p.pos + tt);
+          ztok[it] = *reinterpret_cast<const float *>(s_zgen[ru >> 7] + static_cast<uint32_t>(ru & 127) * 4u);
+        }
+        named_bar_sync(5, kEpiThreads);
         const int items = n_local * n;
         for (int it = tid; it < items; it += kEpiThreads) {
           const int li = it / n, j = it - li * n;
           const int gg = static_cast<int>(crank) + li * p.C;
           const int64_t bb = gi * p.G + gg;
           if (bb >= p.B) continue;
+          // eps_j = sum over t in token order of W_o[t][j] z_t (one FMA chain), loads ahead
+          const float *zl = ztok + li * T;
+          const float *wo = p.w_out + j;
           float acc = 0.0f;
-          const int rb0 = gg * T;
-          for (int tt = 0; tt < T; ++tt) {
-            const int ru = rb0 + __ldg(p.pos + tt);
-            const float zt = *reinterpret_cast<const float *>(s_zgen[ru >> 7] + static_cast<uint32_t>(ru & 127) * 4u);
-            acc = __fmaf_rn(__ldg(p.w_out + tt * n + j), zt, acc);
+          int tt = 0;
+          for (; tt + 8 <= T; tt += 8) {
+            float wv[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) wv[u] = __ldg(wo + (tt + u) * n);
+#pragma unroll
+            for (int u = 0; u < 8; ++u) acc = __fmaf_rn(wv[u], zl[tt + u], acc);
           }
+          for (; tt < T; ++tt) acc = __fmaf_rn(__ldg(wo + tt * n), zl[tt], acc);
           const float eps = __fadd_rn(acc, __ldg(p.b_out + j));
-          const uint8_t bit = (__fmul_rn(__ldg(p.y + bb * n + j), eps) < 0.0f) ? 1 : 0;
+          const uint8_t bit = (__fmul_rn(__ldg(p.y + bb * n + j), eps) < 0.0f) ? 1 : 0;  // y was staged; re-read from L1/L2
           p.bits[bb * n + j] = bit;
           if (p.logits) p.logits[bb * n + j] = eps;
           obits[li * n + j] = bit;
