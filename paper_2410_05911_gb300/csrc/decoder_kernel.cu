@@ -33,7 +33,10 @@ namespace aecct {
 // fp32(ln(2)^k / k!), k = 0..7: Taylor coefficients of 2^f = e^(f ln 2)
 __device__ __forceinline__ float exp2_series(float x) {
   if (!(x >= -125.0f)) return 0.0f;
-  const float n = rintf(x);
+  // n = rint(x) through the rounding add (x is in [-125, 0] here); the integer n also sits in the
+  // low bits of t, which gives the exponent shift without a conversion
+  const float t = __fadd_rn(x, 12582912.0f);
+  const float n = __fsub_rn(t, 12582912.0f);
   const float f = __fsub_rn(x, n);
   float p = __uint_as_float(0x377fe5feu);      // k = 7
   p = __fmaf_rn(p, f, __uint_as_float(0x39218489u));  // k = 6
@@ -44,7 +47,7 @@ __device__ __forceinline__ float exp2_series(float x) {
   p = __fmaf_rn(p, f, __uint_as_float(0x3f317218u));  // k = 1
   p = __fmaf_rn(p, f, 1.0f);                          // k = 0
   // p is in [0.70, 1.42] and n >= -125, so p * 2^n is normal: scale through the exponent field
-  return __int_as_float(__float_as_int(p) + (__float2int_rn(n) << 23));
+  return __int_as_float(__float_as_int(p) + ((__float_as_int(t) - 0x4B400000) << 23));
 }
 
 // ---- paired fp32 arithmetic (sm_100 f32x2: each lane is one IEEE round-to-nearest operation,
@@ -82,8 +85,9 @@ __device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
 
 // two independent evaluations of exp2_series (same steps on each lane); inputs below -125 give 0
 __device__ __forceinline__ float2 exp2_series2(float2 x) {
-  const float n0 = rintf(x.x), n1 = rintf(x.y);
-  const float2 f = add2(x, make_float2(-n0, -n1));
+  const float2 t = add2(x, make_float2(12582912.0f, 12582912.0f));  // rounding adds, as in exp2_series
+  const float2 nn = add2(t, make_float2(-12582912.0f, -12582912.0f));
+  const float2 f = add2(x, make_float2(-nn.x, -nn.y));
   float2 p = make_float2(__uint_as_float(0x377fe5feu), __uint_as_float(0x377fe5feu));
   p = fma2(p, f, make_float2(__uint_as_float(0x39218489u), __uint_as_float(0x39218489u)));
   p = fma2(p, f, make_float2(__uint_as_float(0x3aaec3ffu), __uint_as_float(0x3aaec3ffu)));
@@ -92,8 +96,8 @@ __device__ __forceinline__ float2 exp2_series2(float2 x) {
   p = fma2(p, f, make_float2(__uint_as_float(0x3e75fdf0u), __uint_as_float(0x3e75fdf0u)));
   p = fma2(p, f, make_float2(__uint_as_float(0x3f317218u), __uint_as_float(0x3f317218u)));
   p = fma2(p, f, make_float2(1.0f, 1.0f));
-  const float r0 = (x.x >= -125.0f) ? __int_as_float(__float_as_int(p.x) + (__float2int_rn(n0) << 23)) : 0.0f;
-  const float r1 = (x.y >= -125.0f) ? __int_as_float(__float_as_int(p.y) + (__float2int_rn(n1) << 23)) : 0.0f;
+  const float r0 = (x.x >= -125.0f) ? __int_as_float(__float_as_int(p.x) + ((__float_as_int(t.x) - 0x4B400000) << 23)) : 0.0f;
+  const float r1 = (x.y >= -125.0f) ? __int_as_float(__float_as_int(p.y) + ((__float_as_int(t.y) - 0x4B400000) << 23)) : 0.0f;
   return make_float2(r0, r1);
 }
 
@@ -163,22 +167,26 @@ __device__ __noinline__ bool wait_bar_drain(const Ctl c, uint32_t bar, uint32_t 
 // ------------------------------------------------------------------------------------------
 // small helpers for the CUDA-core warps
 // ------------------------------------------------------------------------------------------
+// Round to the nearest integer, ties to even, for |x| < 2^22, on the FP32 add pipe: x + 1.5 * 2^23
+// lies in [2^23, 2^24), where the spacing of fp32 values is 1, so the round-to-nearest-even add
+// rounds x exactly as rintf does, and subtracting 1.5 * 2^23 back is exact.  (rintf runs on the
+// quarter-rate conversion pipe.)
+constexpr float kRoundMagic = 12582912.0f;  // 1.5 * 2^23
+__device__ __forceinline__ float round_even(float x) { return __fsub_rn(__fadd_rn(x, kRoundMagic), kRoundMagic); }
+
 // Code of v under r = 127/alpha' (eq. Quant).  |v| <= alpha' gives |v * r| <= 127 (1 + 2^-24)
-// before rounding, so the clip of RoundClip can never act and is left out.
-__device__ __forceinline__ float q_code(float v, float r) { return rintf(__fmul_rn(v, r)); }
+// before rounding, so the clip of RoundClip can never act and is left out.  The product stays a
+// separately rounded scalar multiply (a paired multiply feeding the rounding add would be fused).
+__device__ __forceinline__ float q_code(float v, float r) { return round_even(__fmul_rn(v, r)); }
 template <int N>
 __device__ __forceinline__ void codes(const float *v, float r, float *q) {
 #pragma unroll
-  for (int j = 0; j < N; j += 2) {
-    const float2 t = mul2(make_float2(v[j], v[j + 1]), make_float2(r, r));
-    q[j] = rintf(t.x);
-    q[j + 1] = rintf(t.y);
-  }
+  for (int j = 0; j < N; ++j) q[j] = q_code(v[j], r);
 }
 __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
-  // a, b are integers in [-127, 127]: exact in bf16
-  __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
-  return *reinterpret_cast<uint32_t *>(&v);
+  // a, b are integers in [-127, 127]: their fp32 encodings have 16 zero low bits, so the bf16
+  // encodings are the high halves (one byte permute instead of two conversions)
+  return __byte_perm(__float_as_uint(a), __float_as_uint(b), 0x7632);
 }
 __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
   asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
