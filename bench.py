@@ -15,6 +15,8 @@ the same workload on the host cores, and reports the same metric.
 from __future__ import annotations
 
 import argparse
+import glob
+import hashlib
 import json
 import os
 import subprocess
@@ -41,6 +43,49 @@ def peaks():
         return dict(hbm_gbs=p["hbm_gbs"], bf16_tflops=p["bf16_tflops"],
                     bf16_tflops_sustained=p.get("bf16_tflops_sustained", p["bf16_tflops"]), source="measured")
     return dict(hbm_gbs=6800.0, bf16_tflops=1900.0, bf16_tflops_sustained=1700.0, source="fallback")
+
+
+def kernel_sources_digest() -> str:
+    """SHA-256 over the CUDA sources and build flags of the decoder (paths and contents)."""
+    h = hashlib.sha256()
+    pkg = os.path.join(ROOT, "paper_2410_05911_gb300")
+    files = sorted(glob.glob(os.path.join(pkg, "csrc", "*"))) + [os.path.join(pkg, "build_lib.py")]
+    for f in files:
+        if os.path.isfile(f) and f.endswith((".cu", ".cuh", ".h", ".py")):
+            h.update(os.path.relpath(f, ROOT).encode())
+            with open(f, "rb") as fh:
+                h.update(fh.read())
+    return h.hexdigest()
+
+
+def measured_traffic(workload: str, batch: int):
+    """DRAM bytes per launch from the committed ncu record of this workload, scaled to `batch`
+    words, or None when there is no record or the kernel sources changed since it was taken."""
+    path = os.path.join(ROOT, "profiles", f"aecct_decoder_kernel{I.WORKLOADS[workload]['d']}_{workload}_dram.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        rec = json.load(f)
+    if rec.get("sources_sha256") != kernel_sources_digest() or rec.get("workload") != workload:
+        return None
+    return (rec["dram_bytes_read"] + rec["dram_bytes_write"]) * batch / rec["batch"]
+
+
+def max_over_ranks(x: float, world: int, device=None) -> float:
+    """The maximum of x over the ranks of the process group (x itself when world == 1)."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def rank_seed(rank: int, i: int) -> int:
+    """Seed of the i-th input batch of a rank: every rank decodes its own words (weak scaling)."""
+    return 1000 * rank + 11 + i
 
 
 def work_per_word(w: I.Workload):
@@ -178,7 +223,7 @@ def run_cuda(args, rank, world, local_rank):
     dec = aecct.Decoder(model)
     q = dec.query()
     # inputs: one batch per Eb/N0 point, resident on the device
-    ys_host = [I.channel_batch(w.code, B, e, seed=1000 * rank + 11 + i).y for i, e in enumerate(w.ebn0_db)]
+    ys_host = [I.channel_batch(w.code, B, e, seed=rank_seed(rank, i)).y for i, e in enumerate(w.ebn0_db)]
     ys = [torch.from_numpy(y).to(dev) for y in ys_host]
     bits = torch.empty((B, w.code.n), dtype=torch.uint8, device=dev)
     syn = torch.empty((B, w.code.n - w.code.k), dtype=torch.uint8, device=dev)
@@ -213,11 +258,7 @@ def run_cuda(args, rank, world, local_rank):
     if dec.synchronize() != aecct.AECCT_OK:
         raise RuntimeError("timed decode reported an error")
     ms = [a.elapsed_time(b) for a, b in evs]
-    total_s = sum(ms) / 1e3
-    if world > 1:
-        t = torch.tensor([total_s], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_s = float(t.item())
+    total_s = max_over_ranks(sum(ms) / 1e3, world, dev)
     value = world * B * args.steps / total_s
     kernel_s = total_s / args.steps
 
@@ -229,11 +270,7 @@ def run_cuda(args, rank, world, local_rank):
     t0 = time.perf_counter()
     for i in range(e2e_steps):
         dec.decode_host(y_pin.numpy(), want_logits=False)
-    e2e_s = (time.perf_counter() - t0) / e2e_steps
-    if world > 1:
-        t = torch.tensor([e2e_s], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_s = float(t.item())
+    e2e_s = max_over_ranks((time.perf_counter() - t0) / e2e_steps, world, dev)
     e2e = dict(value=world * B / e2e_s, unit=UNIT, h2d_bytes_per_step=4 * B * w.code.n,
                d2h_bytes_per_step=B * w.code.n + B * (w.code.n - w.code.k))
 
@@ -243,7 +280,8 @@ def run_cuda(args, rank, world, local_rank):
     wk = work_per_word(w)
     achieved_tops = wk["int_ops"] * B / kernel_s / 1e12
     roof = dict(bound="tensor", achieved=achieved_tops, peak=pk["bf16_tflops"], unit="TFLOP/s",
-                frac=achieved_tops / pk["bf16_tflops"], traffic=args.traffic,
+                frac=achieved_tops / pk["bf16_tflops"],
+                traffic=args.traffic if args.traffic is not None else measured_traffic(args.workload, B),
                 kernel=f"aecct_decoder_kernel<{w.d}>", work="2*12*T*d^2*N int ops per word (bf16 tensor cores, "
                 "exact integers); peak = measured bf16 dense burst")
     cpu = None
