@@ -385,6 +385,7 @@ def random_model(
     activation: int = 0,
     ffn_mult: int = 4,
     zero_weights: bool = False,
+    binary: bool = False,
 ) -> ModelTensors:
     """Seeded synthetic AECCT parameters shaped like a trained model.
 
@@ -394,6 +395,10 @@ def random_model(
     in [0.9, 1.1].  Biases and LayerNorm parameters are small random values so that an
     indexing mistake changes the output.  The SPE table is a seeded N(0,1) table standing
     in for the learned one (at inference it is a fixed table).
+
+    binary=True draws the binary-weight variant (App. D): every weight is +1 or -1 and the
+    per-tensor scale is the mean |W| of N(0, 1/d_in) weights, sqrt(2 / (pi d_in)), times the
+    same jitter.
     """
     rng = np.random.Generator(np.random.PCG64(seed))
     T = code.T
@@ -412,13 +417,16 @@ def random_model(
             size = dout * din
             if zero_weights:
                 t = np.zeros(size, dtype=np.int8)
+            elif binary:
+                t = rng.choice(np.array([-1, 1], dtype=np.int8), size=size)
             else:
                 nz = int(round(zero_frac * size))
                 t = rng.choice(np.array([-1, 1], dtype=np.int8), size=size)
                 zpos = rng.permutation(size)[:nz]
                 t[zpos] = 0
             wl.append(t.reshape(dout, din))
-            w_scale[l, g] = ternary_scale_for_zero_fraction(zero_frac, din) * rng.uniform(0.9, 1.1)
+            base = math.sqrt(2.0 / (math.pi * din)) if binary else ternary_scale_for_zero_fraction(zero_frac, din)
+            w_scale[l, g] = base * rng.uniform(0.9, 1.1)
             bl.append((0.1 * rng.standard_normal(dout)).astype(np.float32))
         w_tern.append(wl)
         bias.append(bl)

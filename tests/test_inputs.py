@@ -118,3 +118,14 @@ def test_synthetic_weights_zero_fraction_and_values():
 def test_ternary_scale_constant():
     # half-scale threshold at the median of |N(0, s^2)| gives 50% zeros: scale = 2 * 0.6745 s
     assert I.ternary_scale_for_zero_fraction(0.5, 64) == pytest.approx(2 * 0.67449 / 8, rel=1e-4)
+
+
+def test_binary_weight_variant():
+    code = I.make_code("bch31_16")
+    m = I.random_model(code, 32, 2, seed=3, binary=True)
+    for l in range(2):
+        for g, t in enumerate(m.w_tern[l]):
+            assert set(np.unique(t).tolist()) == {-1, 1}
+            d_in = t.shape[1]
+            base = np.sqrt(2.0 / (np.pi * d_in))
+            assert 0.9 * base - 1e-7 <= m.w_scale[l, g] <= 1.1 * base + 1e-7
