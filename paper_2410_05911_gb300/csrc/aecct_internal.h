@@ -17,6 +17,7 @@ constexpr int kOutBitsBytes = 4096;      // decoded bits of the codewords one CT
 constexpr int kMaxTasks = 16;            // attention tasks per warp (task mode)
 constexpr int kMaxGroups = 32;           // 32-row query groups per CTA (task mode)
 constexpr int kTaskCache = 64;           // attention scores per task kept in TMEM (task mode)
+constexpr int kRowCache = 64;            // attention scores per (row, head) kept in TMEM (row mode)
 
 // One weight chunk of a block: rows [n0, n0 + nrows) and K columns [k0, k0 + kcols) of the
 // block's GEMM `gemm` (0 = QKV, 1 = O, 2 = FFN1, 3 = FFN2), stored as a K-major bf16 tile
@@ -179,10 +180,14 @@ struct SmemLayout {
   static constexpr uint32_t kOffBar = kOffObits + kOutBitsBytes;      // mbarriers
   static constexpr uint32_t kOffMisc = kOffBar + 256;  // tmem base, abort flag, peer bases, copy count
   static constexpr uint32_t kTotal = kOffMisc + 256;
-  // QKV / FFN1 accumulators in [0, 4D); task mode also caches attention scores in
-  // [kTaskCacheCol, 512): 4 warps per lane quadrant x kTaskCache columns
-  static constexpr uint32_t kTmemCols = TASKS ? 512u : 4u * D;
+  // QKV / FFN1 accumulators in [0, 4D) (x parked in [3D, 4D) during attention).  Attention
+  // scores are cached in TMEM between the two softmax passes: task mode in [kTaskCacheCol, 512)
+  // (4 warps per lane quadrant x kTaskCache columns); row mode kRowCache columns per column slice
+  // from kRowCacheCol, each thread in its own row's lane (d = 128: the K and V accumulator
+  // columns [128, 384), dead once K and V are in shared memory; d <= 64: [256, 512)).
+  static constexpr uint32_t kTmemCols = 512u;
   static constexpr uint32_t kTaskCacheCol = 256u;
+  static constexpr uint32_t kRowCacheCol = (D == 128) ? 128u : 256u;
 };
 
 // decoder_kernel.cu

@@ -243,13 +243,18 @@ __device__ __forceinline__ int idx_at(const uint4 &w, int k) {
 // DecodeParams::mask_info).  Two passes in the canonical order:
 // sigma_u = fma-chain(q . k_u) * scale, m = max sigma; p_u = 2^(sigma_u - m);
 // l = sum p_u and num = sum p_u v_u in ascending key order; A = num * (1 / l).
-// Keys come 8 per index load; U keys at a time have their loads issued together and their dot
-// products run as independent chains, while every sum keeps the sequential key order.
+// Every lane has its own list; the warp walks 8-key blocks up to the longest list of its lanes
+// (a lane past its own count computes on a valid dummy row and folds nothing in).  The scores of
+// the first kRowCache keys go to this thread's TMEM columns in pass 1 and come back in pass 2, in
+// place of a second load of K and a second dot product (the same fp32 values).
 template <int DH, int U, uint32_t STRIDE>
-__device__ __forceinline__ void hpsa_head(const float *q, uint32_t info, const uint4 *__restrict__ lists,
-                                          const uint64_t *kvgen, int rowbase, uint32_t hoff, float scale, float *A) {
+__device__ __forceinline__ void hpsa_head(const float *q, uint32_t info, bool active, const uint4 *__restrict__ lists,
+                                          const uint64_t *kvgen, int rowbase, uint32_t hoff, float scale,
+                                          uint32_t tcache, float *A) {
+  static_assert(8 % U == 0, "keys per index block");
   const uint4 *lst = lists + (info >> 11);
-  const int cnt = static_cast<int>(info & 2047u);
+  const int cnt = active ? static_cast<int>(info & 2047u) : 0;
+  const int nmax = __reduce_max_sync(0xffffffffu, cnt);
   auto keyptr = [&](int off) -> const float4 * {
     const int ru = rowbase + off;
     return reinterpret_cast<const float4 *>(kvgen[ru >> 7] + static_cast<uint32_t>(ru & 127) * STRIDE + hoff);
@@ -265,33 +270,29 @@ __device__ __forceinline__ void hpsa_head(const float *q, uint32_t info, const u
     }
     return dot;
   };
-  // pass 1: maximum score
+  // pass 1: scores and their maximum
   float mx = -INFINITY;
-  for (int jb = 0; jb < cnt; jb += 8) {
-    const uint4 w = __ldg(lst + (jb >> 3));
-    if (jb + 8 <= cnt) {
+  for (int jb = 0; jb < nmax; jb += 8) {
+    const uint4 w = (jb < cnt) ? __ldg(lst + (jb >> 3)) : make_uint4(0u, 0u, 0u, 0u);
+    float sg[8];
 #pragma unroll
-      for (int k0 = 0; k0 < 8; k0 += U) {
-        float4 kk[U][DH / 4];
+    for (int k0 = 0; k0 < 8; k0 += U) {
+      float4 kk[U][DH / 4];
 #pragma unroll
-        for (int k = 0; k < U; ++k) {
-          const float4 *kp = keyptr(idx_at(w, k0 + k));
+      for (int k = 0; k < U; ++k) {
+        const float4 *kp = keyptr(idx_at(w, k0 + k));
 #pragma unroll
-          for (int i = 0; i < DH / 4; ++i) kk[k][i] = kp[i];
-        }
-#pragma unroll
-        for (int k = 0; k < U; ++k) mx = fmaxf(mx, __fmul_rn(dotk(kk[k]), scale));
+        for (int i = 0; i < DH / 4; ++i) kk[k][i] = kp[i];
       }
-    } else {
-      for (int k = 0; k < cnt - jb; ++k) {
-        const float4 *kp = keyptr(idx_at(w, k));
-        float4 kk[DH / 4];
 #pragma unroll
-        for (int i = 0; i < DH / 4; ++i) kk[i] = kp[i];
-        mx = fmaxf(mx, __fmul_rn(dotk(kk), scale));
+      for (int k = 0; k < U; ++k) {
+        sg[k0 + k] = __fmul_rn(dotk(kk[k]), scale);
+        if (jb + k0 + k < cnt) mx = fmaxf(mx, sg[k0 + k]);
       }
     }
+    if (jb < kRowCache) tmem_st<8>(tcache + jb, sg);
   }
+  tmem_wait_st();
   // pass 2: probabilities, their sum and the weighted values, in key order
   float lsum = 0.0f;
   float num[DH];
@@ -307,41 +308,40 @@ __device__ __forceinline__ void hpsa_head(const float *q, uint32_t info, const u
       num[4 * i + 3] = __fmaf_rn(pr, vv[i].w, num[4 * i + 3]);
     }
   };
-  for (int jb = 0; jb < cnt; jb += 8) {
-    const uint4 w = __ldg(lst + (jb >> 3));
-    if (jb + 8 <= cnt) {
+  for (int jb = 0; jb < nmax; jb += 8) {
+    const uint4 w = (jb < cnt) ? __ldg(lst + (jb >> 3)) : make_uint4(0u, 0u, 0u, 0u);
+    float sg[8];
+    const bool cached = jb < kRowCache;
+    if (cached) {
+      tmem_ld<8>(tcache + jb, sg);
+      tmem_wait_ld();
+    }
 #pragma unroll
-      for (int k0 = 0; k0 < 8; k0 += U) {
-        float4 kk[U][DH / 4], vv[U][DH / 4];
+    for (int k0 = 0; k0 < 8; k0 += U) {
+      float4 vv[U][DH / 4];
 #pragma unroll
-        for (int k = 0; k < U; ++k) {
-          const float4 *kp = keyptr(idx_at(w, k0 + k));
+      for (int k = 0; k < U; ++k) {
+        const float4 *kp = keyptr(idx_at(w, k0 + k));
+        if (!cached) {
+          float4 kk[DH / 4];
 #pragma unroll
-          for (int i = 0; i < DH / 4; ++i) kk[k][i] = kp[i];
-#pragma unroll
-          for (int i = 0; i < DH / 4; ++i) vv[k][i] = kp[DH / 4 + i];
+          for (int i = 0; i < DH / 4; ++i) kk[i] = kp[i];
+          sg[k0 + k] = __fmul_rn(dotk(kk), scale);
         }
-        float pr[U];
 #pragma unroll
-        for (int k = 0; k < U; ++k) pr[k] = exp2_series(__fsub_rn(__fmul_rn(dotk(kk[k]), scale), mx));
-#pragma unroll
-        for (int k = 0; k < U; ++k) accumulate(pr[k], vv[k]);
+        for (int i = 0; i < DH / 4; ++i) vv[k][i] = kp[DH / 4 + i];
       }
-    } else {
-      for (int k = 0; k < cnt - jb; ++k) {
-        const float4 *kp = keyptr(idx_at(w, k));
-        float4 kk[DH / 4], vv[DH / 4];
+      float pr[U];
 #pragma unroll
-        for (int i = 0; i < DH / 4; ++i) kk[i] = kp[i];
+      for (int k = 0; k < U; ++k) pr[k] = exp2_series(__fsub_rn(sg[k0 + k], mx));
 #pragma unroll
-        for (int i = 0; i < DH / 4; ++i) vv[i] = kp[DH / 4 + i];
-        accumulate(exp2_series(__fsub_rn(__fmul_rn(dotk(kk), scale), mx)), vv);
-      }
+      for (int k = 0; k < U; ++k)
+        if (jb + k0 + k < cnt) accumulate(pr[k], vv[k]);
     }
   }
   const float inv = __fdiv_rn(1.0f, lsum);
 #pragma unroll
-  for (int i = 0; i < DH; ++i) A[i] = __fmul_rn(num[i], inv);
+  for (int i = 0; i < DH; ++i) A[i] = active ? __fmul_rn(num[i], inv) : 0.0f;
 }
 
 // byte k of a 16-entry index block
@@ -523,6 +523,14 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
 // phase per GEMM, four per block, so GEMM g always waits for parity g & 1.  Everything the issue
 // path computes is therefore a compile-time constant or a warp-uniform base address, and the
 // tcgen05 instructions take their operands straight from uniform registers.
+// What the issuer needs to know about the block a GEMM belongs to (used by the d = 128 schedule).
+struct BlockCtx {
+  uint32_t lpar;    // parity of the block's index in this CTA's sequence of blocks
+  uint32_t kvf;     // cluster barrier: every CTA of the cluster has finished reading this CTA's K/V
+  uint32_t kvf_ph;  // its phase parity for this block
+  bool cluster;     // more than one CTA per cluster
+};
+
 template <int D, bool TASKS>
 struct Issuer {
   using L = SmemLayout<D, TASKS>;
@@ -606,7 +614,8 @@ struct Issuer {
   // chunks that follow the freed stages: chunk p + S of this block, or chunk p + S - CPL of the
   // next block (`w_next`, when `has_next`).
   template <int G>
-  __device__ __forceinline__ void gemm(const uint8_t *w_cur, const uint8_t *w_next, bool has_next) const {
+  __device__ __forceinline__ void gemm(const uint8_t *w_cur, const uint8_t *w_next, bool has_next,
+                                       const BlockCtx &) const {
     constexpr int first = W::first(G), count = W::count(G);
     wait(bar_op(), G & 1);
     tc_fence_after();
@@ -628,6 +637,197 @@ struct Issuer {
     }
   }
 };
+// d = 128: the 24 chunks of a block (16 KB each: QKV 0-5, O 6-7, FFN1 8-15, FFN2 16-23) do not
+// fit three 16 KB stages without refilling inside the FFN GEMMs, so the schedule also uses the
+// regions that are idle at that point of the block:
+//   QKV  -> region U (free between the previous FFN2 and this block's K/V), one barrier bar_U;
+//   O    -> stages W0, W1;
+//   FFN1 -> region U again (free once every CTA of the cluster has finished attention);
+//   FFN2 -> W0, W1, W2, then the operand tile (free once FFN1's MMAs are done) as A0, A1, then
+//           W0, W1, W2 again once chunks 16-18 are consumed.
+// A barrier armed u times per block (u odd for W0, W1, A0, A1) completes phase parity
+// (lpar if u is odd) ^ (index of the use within the block), with lpar the block's parity.
+template <bool TASKS>
+struct Issuer<128, TASKS> {
+  static constexpr int D = 128;
+  using L = SmemLayout<D, TASKS>;
+  using W = WeightSchedule<D>;
+  static constexpr uint32_t kChunk = W::kStageBytes;
+  static_assert(W::kCPL == 24 && W::kStages == 3 && kChunk == 16384, "d = 128 schedule");
+  static_assert(L::kRegionU >= 8 * kChunk && L::kAopBytes == 2 * kChunk, "d = 128 regions");
+  uint32_t sb, tmem;
+  Ctl ctl;
+  uint32_t *n_armed;  // [6] phases armed per weight barrier (W0, W1, W2, U, A0, A1), for the drain
+
+  // barrier ids: 0-2 stages W0-W2, 3 region U, 4-5 operand-tile halves A0, A1
+  __device__ __forceinline__ uint32_t bar(int id) const {
+    return sb + L::kOffBar + (id < 3 ? 8 * id : 16 * 3 + 7 * 8 + 8 * (id - 3));
+  }
+  __device__ __forceinline__ uint32_t bar_empty(int s) const { return sb + L::kOffBar + 8 * (3 + s); }
+  __device__ __forceinline__ uint32_t bar_op() const { return sb + L::kOffBar + 48; }
+  __device__ __forceinline__ uint32_t bar_acc() const { return sb + L::kOffBar + 56; }
+
+  // slot of chunk P: shared-memory offset, barrier id, uses of that barrier per block, use index
+  struct Slot {
+    uint32_t off;
+    int id, uses, idx;
+  };
+  __host__ __device__ static constexpr Slot slot(int p) {
+    return p < 6    ? Slot{L::kOffU + kChunk * p, 3, 2, 0}
+           : p < 8  ? Slot{L::kOffW + kChunk * (p - 6), p - 6, 3, 0}
+           : p < 16 ? Slot{L::kOffU + kChunk * (p - 8), 3, 2, 1}
+           : p < 19 ? Slot{L::kOffW + kChunk * (p - 16), p - 16, p - 16 < 2 ? 3 : 2, p - 16 < 2 ? 1 : 0}
+           : p < 21 ? Slot{L::kOffAop + kChunk * (p - 19), 4 + (p - 19), 1, 0}
+                    : Slot{L::kOffW + kChunk * (p - 21), p - 21, p - 21 < 2 ? 3 : 2, p - 21 < 2 ? 2 : 1};
+  }
+  template <int P>
+  __device__ __forceinline__ static uint32_t parity(uint32_t lpar) {
+    constexpr Slot s = slot(P);
+    return ((s.uses & 1) ? lpar : 0u) ^ static_cast<uint32_t>(s.idx & 1);
+  }
+
+  __device__ __forceinline__ void wait(uint32_t b, uint32_t parity, bool cluster_scope = false) const {
+    if ((threadIdx.x & 31) == 0 && !(cluster_scope ? mbar_try_wait_acq_cluster(b, parity) : mbar_try_wait(b, parity)))
+      wait_bar_slow(ctl, b, parity, cluster_scope);
+    __syncwarp();
+  }
+  // arm barrier `id` for `bytes` (one arrive), then the copies of chunks P0 .. P1-1 complete it
+  __device__ __forceinline__ void arm(int id, uint32_t bytes) const {
+    asm volatile(
+        "{\n\t.reg .pred e;\n\t.reg .b32 r;\n\telect.sync r|e, 0xffffffff;\n\t"
+        "@e mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n\t}" ::"r"(bar(id)),
+        "r"(bytes)
+        : "memory");
+    if ((threadIdx.x & 31) == 0) ++n_armed[id];
+  }
+  template <int P0, int P1>
+  __device__ __forceinline__ void copies(const uint8_t *src) const {
+    if constexpr (P0 < P1) {
+      constexpr ChunkDesc c = W::chunk(P0);
+      constexpr Slot s = slot(P0);
+      asm volatile(
+          "{\n\t.reg .pred e;\n\t.reg .b32 r;\n\telect.sync r|e, 0xffffffff;\n\t"
+          "@e cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n\t}" ::"r"(
+              sb + s.off),
+          "l"(src + c.off), "r"(c.bytes), "r"(bar(s.id))
+          : "memory");
+      copies<P0 + 1, P1>(src);
+    }
+  }
+  template <int P>
+  __device__ __forceinline__ void copy1(const uint8_t *src) const {
+    arm(slot(P).id, W::chunk(P).bytes);
+    copies<P, P + 1>(src);
+  }
+  // QKV (region U) and O (W0, W1) of a block
+  __device__ __forceinline__ void stage_qkv_o(const uint8_t *src) const {
+    arm(3, 6 * kChunk);
+    copies<0, 6>(src);
+    copy1<6>(src);
+    copy1<7>(src);
+  }
+  __device__ __forceinline__ void prologue(const uint8_t *w0) const { stage_qkv_o(w0); }
+
+  // the MMAs of chunk P (its weights have landed)
+  template <int G, int P>
+  __device__ __forceinline__ void mmas() const {
+    constexpr ChunkDesc c = W::chunk(P);
+    constexpr uint32_t a_tile = (G == 3) ? L::kOffU : L::kOffAop;
+    constexpr uint32_t a_sbo = (G == 3) ? (4u * D / 8u) * 128u : (D / 8u) * 128u;
+    constexpr uint32_t b_sbo = (c.kcols / 8u) * 128u;
+    constexpr uint32_t idesc = make_idesc_bf16(128, c.nrows);
+    const uint32_t b_tile = sb + slot(P).off;
+#pragma unroll
+    for (int ks = 0; ks < c.kcols / 16; ++ks) {
+      const uint32_t kabs = c.k0 + 16u * ks;
+      mma_bf16_warp(tmem + c.n0, make_sdesc(sb + a_tile + (kabs / 8u) * 128u, 128u, a_sbo),
+                    make_sdesc(b_tile + ks * 256u, 128u, b_sbo), idesc, kabs > 0 ? 1u : 0u);
+    }
+  }
+  template <int G, int P0, int P1>
+  __device__ __forceinline__ void mmas_range() const {
+    if constexpr (P0 < P1) {
+      mmas<G, P0>();
+      mmas_range<G, P0 + 1, P1>();
+    }
+  }
+
+  template <int G>
+  __device__ __forceinline__ void gemm(const uint8_t *w_cur, const uint8_t *w_next, bool has_next,
+                                       const BlockCtx &bc) const {
+    const uint32_t lp = bc.lpar;
+    wait(bar_op(), G & 1);
+    tc_fence_after();
+    if constexpr (G == 0) {
+      wait(bar(3), 0);  // QKV weights in region U
+      mmas_range<0, 0, 6>();
+      mma_commit_warp(bar_acc());
+      wait(bar_acc(), 0);
+    } else if constexpr (G == 1) {
+      wait(bar(0), parity<6>(lp));
+      mmas<1, 6>();
+      wait(bar(1), parity<7>(lp));
+      mmas<1, 7>();
+      mma_commit_warp(bar_acc());
+      // FFN1 weights into region U once no CTA of the cluster reads this CTA's K/V any more;
+      // FFN2 chunk 18 into W2 (its last reader was the previous block's FFN2)
+      if (bc.cluster) wait(bc.kvf, bc.kvf_ph, true);
+      arm(3, 8 * kChunk);
+      copies<8, 16>(w_cur);
+      copy1<18>(w_cur);
+      wait(bar_acc(), 1);
+      copy1<16>(w_cur);  // W0, W1 were O's
+      copy1<17>(w_cur);
+    } else if constexpr (G == 2) {
+      wait(bar(3), 1);  // FFN1 weights in region U
+      mmas_range<2, 8, 16>();
+      mma_commit_warp(bar_acc());
+      wait(bar_acc(), 0);
+      copy1<19>(w_cur);  // the operand tile is free: FFN1's MMAs are done
+      copy1<20>(w_cur);
+    } else {
+      wait(bar(0), parity<16>(lp));
+      mmas<3, 16>();
+      mma_commit_warp(bar_empty(0));
+      wait(bar(1), parity<17>(lp));
+      mmas<3, 17>();
+      mma_commit_warp(bar_empty(1));
+      wait(bar(2), parity<18>(lp));
+      mmas<3, 18>();
+      mma_commit_warp(bar_empty(2));
+      wait(bar(4), parity<19>(lp));
+      mmas<3, 19>();
+      wait(bar(5), parity<20>(lp));
+      mmas<3, 20>();
+      // refill W0-W2 with chunks 21-23 as soon as chunks 16-18 are consumed; the MMAs of 19 and
+      // 20 keep the tensor pipe busy meanwhile
+      wait(bar_empty(0), lp);
+      copy1<21>(w_cur);
+      wait(bar_empty(1), lp);
+      copy1<22>(w_cur);
+      wait(bar_empty(2), lp);
+      copy1<23>(w_cur);
+      wait(bar(0), parity<21>(lp));
+      mmas<3, 21>();
+      wait(bar(1), parity<22>(lp));
+      mmas<3, 22>();
+      wait(bar(2), parity<23>(lp));
+      mmas<3, 23>();
+      mma_commit_warp(bar_acc());
+      wait(bar_acc(), 1);
+      if (has_next) stage_qkv_o(w_next);  // region U and W0, W1 are free again
+    }
+  }
+  // every copy started has landed (bounded waits that ignore the abort flag)
+  __device__ __forceinline__ void drain() const {
+#pragma unroll
+    for (int id = 0; id < 6; ++id) {
+      const uint32_t cnt = n_armed[id];
+      if (cnt > 0) wait_bar_drain(ctl, bar(id), (cnt - 1u) & 1u);
+    }
+  }
+};
+
 // ------------------------------------------------------------------------------------------
 // the kernel
 // ------------------------------------------------------------------------------------------
@@ -657,7 +857,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   volatile int *s_abort = reinterpret_cast<volatile int *>(smem + L::kOffMisc + 4);
   uint64_t *s_kvgen = reinterpret_cast<uint64_t *>(smem + L::kOffMisc + 8);  // [8] generic K/V bases per CTA
   uint64_t *s_zgen = reinterpret_cast<uint64_t *>(smem + L::kOffMisc + 72);   // [8] generic z bases per CTA
-  uint32_t *s_issued = reinterpret_cast<uint32_t *>(smem + L::kOffMisc + 136);  // weight copies started
+  uint32_t *s_issued = reinterpret_cast<uint32_t *>(smem + L::kOffMisc + 136);  // [6] weight copies / phases armed
 
   if (tid == 0) {
     for (int s = 0; s < S; ++s) {
@@ -671,8 +871,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
     mbar_init(bar_zr, p.C);
     mbar_init(bar_zf, p.C);
     mbar_init(bar_fin, 1);
+    if constexpr (D == 128)  // region U and the two operand-tile halves (d = 128 weight schedule)
+      for (int i = 0; i < 3; ++i) mbar_init(bar_fin + 8 + 8 * i, 1);
     *s_abort = 0;
-    *s_issued = 0;
+    for (int i = 0; i < 6; ++i) s_issued[i] = 0;
     // generic base of the K/V and z areas of every CTA of the cluster: this CTA's own area through
     // its plain shared-memory window, the others through the distributed shared window
     for (int c = 0; c < p.C; ++c) {
@@ -730,6 +932,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
     };
     // publish this warp's part of the operand of GEMM `gemm` of block `blk` of group `gi`;
     // warp 0 then issues the GEMM and prefetches the weights that follow it
+    uint32_t blk_base = 0;  // blocks this CTA ran in earlier groups (the block parity of the d = 128 schedule)
     auto signal_op = [&](int gemm, int blk, int64_t gi) {
       tc_fence_before();  // this thread's TMEM reads are ordered before the MMA the arrive releases
       fence_proxy_async_smem();
@@ -741,10 +944,11 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         const uint8_t *w_cur = p.wstream + static_cast<size_t>(blk) * p.layer_bytes;
         const uint8_t *w_next = last_blk ? p.wstream : w_cur + p.layer_bytes;
         const bool has_next = !last_blk || gi + p.n_clusters < p.n_groups;
-        if (gemm == 0) issuer.template gemm<0>(w_cur, w_next, has_next);
-        if (gemm == 1) issuer.template gemm<1>(w_cur, w_next, has_next);
-        if (gemm == 2) issuer.template gemm<2>(w_cur, w_next, has_next);
-        if (gemm == 3) issuer.template gemm<3>(w_cur, w_next, has_next);
+        const BlockCtx bc{(blk_base + static_cast<uint32_t>(blk)) & 1u, bar_kvf, kvf_ph, p.C > 1};
+        if (gemm == 0) issuer.template gemm<0>(w_cur, w_next, has_next, bc);
+        if (gemm == 1) issuer.template gemm<1>(w_cur, w_next, has_next, bc);
+        if (gemm == 2) issuer.template gemm<2>(w_cur, w_next, has_next, bc);
+        if (gemm == 3) issuer.template gemm<3>(w_cur, w_next, has_next, bc);
       }
     };
     // A cluster of one CTA needs no cluster-scope signal: the named barrier in cluster_arrive
@@ -1007,13 +1211,14 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             for (int i = 0; i < DH; ++i) q[i] = __fadd_rn(__fmul_rn(qa[i], fq), bq[i]);
   #pragma unroll
             for (int i = 0; i < DH; ++i) A[hh][i] = 0.0f;
-            if (row_cw) {
+            {
               const int mk = (e < p.h_first) ? 0 : 1;
               constexpr int U = (DH >= 16) ? 2 : 4;
-              hpsa_head<DH, U, L::kKvStride>(q, __ldg(p.mask_info[mk] + t), p.mask_list[mk], s_kvgen, g * T,
-                                             e * (8 * DH), p.att_scale, A[hh]);
+              // this thread's score cache: its own TMEM lane, kRowCache columns per column slice
+              const uint32_t tcache = tl + L::kRowCacheCol + static_cast<uint32_t>(sl) * kRowCache;
+              hpsa_head<DH, U, L::kKvStride>(q, row_cw ? __ldg(p.mask_info[mk] + t) : 0u, row_cw, p.mask_list[mk],
+                                             s_kvgen, g * T, e * (8 * DH), p.att_scale, tcache, A[hh]);
             }
-            __syncwarp();  // lanes leave their key loops at different times; reconverge before tcgen05.ld
   #pragma unroll
             for (int i = 0; i < DH; ++i) amax = fmaxf(amax, fabsf(A[hh][i]));
           }
@@ -1034,8 +1239,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             }
           }
         }
+        // this CTA no longer reads any K/V of this block (arrived before the O GEMM is issued: the
+        // d = 128 schedule stages FFN1's weights over the K/V region once every CTA has arrived)
+        if constexpr (!TASKS) cluster_arrive(bar_kvf);
         signal_op(1, l, gi);
-        if constexpr (!TASKS) cluster_arrive(bar_kvf);  // this CTA no longer reads any K/V of this block
 
         // ---------------- S6: O projection + residual + LayerNorm (Sec. 5, Post-LN)
         wait_acc();
@@ -1199,6 +1406,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         }
         cluster_arrive(bar_zf);  // this CTA no longer reads any z of this group; obits free
       }
+      blk_base += static_cast<uint32_t>(p.n_layers);
     }
   }
 
