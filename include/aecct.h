@@ -63,6 +63,9 @@ typedef struct aecct_handle aecct_handle; /* opaque */
  *   attention_mode 0 = choose automatically; 1 = per-row neighbour lists (any cluster size);
  *                 2 = warp tasks over shared key sets (one CTA per group, d <= 64, at most
  *                 128 tokens).  Every mode computes the same results bit for bit.
+ *   mask_mode     0 = HPSA (Sec. 4.2): heads [0, h_first) first ring, the rest second ring;
+ *                 1 = the ECCT code-aware mask (Sec. 3) for every head: the union of the first
+ *                 and second rings (which contains each node itself).  Other values are rejected.
  *   H             [(n-k)][n] uint8 row-major, entries 0/1, no all-zero row or column.
  *   emb           [T][d-d_spe] fp32: token t's embedding row, scaled by h_t (Sec. 3, ECCT).
  *   spe           [T][d_spe] fp32: spectral positional encoding table (Sec. 4.3);
@@ -86,7 +89,7 @@ typedef struct aecct_handle aecct_handle; /* opaque */
  *                 wait, after which the kernel stops and decode reports AECCT_ERR_TIMEOUT.
  */
 typedef struct {
-  int32_t n, k, d, n_layers, heads, h_first, d_spe, ffn_mult, activation, cluster_ctas, attention_mode;
+  int32_t n, k, d, n_layers, heads, h_first, d_spe, ffn_mult, activation, cluster_ctas, attention_mode, mask_mode;
   const uint8_t *H;
   const float *emb;
   const float *spe;

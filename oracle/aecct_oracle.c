@@ -13,6 +13,8 @@
  *   Sec. 4.1 eq. AAPLinear          int accumulate, dequantise by gamma*delta*alpha/Q_b, add bias
  *   Sec. 4.2 (HPSA)                 first-ring heads on the c<->v mask, second-ring heads on the
  *                                   v<->v / c<->c mask
+ *   Sec. 3 (ECCT, mask_mode 1)      the code-aware mask of the ECCT baseline: every head on the
+ *                                   union of the two rings
  *   Sec. 4.3 eq. SPE                SPE table concatenated to the embedding (table given as input)
  *   Sec. 4 item 4                   ReLU in the feed-forward block
  *   Sec. 5 (Training & Inference)   Post-LN Transformer blocks
@@ -27,6 +29,11 @@
  *     p = 2^(sigma - max sigma), with 2^x evaluated by exp2_series() below (range
  *     reduction x = n + f, |f| <= 1/2, and the degree-7 Taylor series of e^(f ln 2));
  *   - sums over keys and over tokens run in ascending index order.
+ *
+ * Pins (tests/): exp2 against libm and its Taylor coefficients, pairwise sums, quantiser and
+ * LayerNorm closed forms, brute-force integer products, masks against Tanner-graph distances,
+ * codeword-symmetry invariance, the all-zero-weight closed form, and an independent float64
+ * forward pass teacher-forced on the recorded integer core.
  */
 #include <math.h>
 #include <pthread.h>
@@ -43,6 +50,7 @@
 /* ------------------------------------------------------------------------- */
 typedef struct {
   int32_t n, k, d, n_layers, heads, h_first, d_spe, ffn_mult, activation;
+  int32_t mask_mode;       /* 0 = HPSA (Sec. 4.2); 1 = ECCT code-aware mask M1 | M2 for all heads (Sec. 3) */
   const uint8_t *H;        /* [(n-k)][n] 0/1 */
   const float *emb;        /* [T][d-d_spe] */
   const float *spe;        /* [T][d_spe] */
@@ -426,6 +434,12 @@ static int work_alloc(const oracle_model *m, work_t *w) {
       !w->q || !w->acc || !w->b || !w->s || !w->c || !w->M1 || !w->M2)
     return ORACLE_ENOMEM;
   oracle_masks(m->H, m->n - m->k, m->n, w->M1, w->M2);
+  if (m->mask_mode == 1) {
+    /* ECCT's code-aware mask (Sec. 3): a token attends to its Tanner neighbours, to the nodes of
+     * its own type two edges away, and to itself -- the union of the two rings -- in every head */
+    const size_t TT = (size_t)(2 * m->n - m->k) * (size_t)(2 * m->n - m->k);
+    for (size_t i = 0; i < TT; ++i) w->M1[i] = w->M2[i] = (uint8_t)(w->M1[i] | w->M2[i]);
+  }
   return ORACLE_OK;
 }
 
@@ -467,6 +481,7 @@ static int validate(const oracle_model *m) {
   if (m->d & (m->d - 1)) return ORACLE_EINVAL; /* pairwise LN sums take a power-of-two width */
   if (m->d > 1024 || m->d / m->heads > 64 || m->n_layers < 0) return ORACLE_EINVAL;
   if (m->h_first < 0 || m->h_first > m->heads || m->d_spe < 0 || m->d_spe >= m->d) return ORACLE_EINVAL;
+  if (m->mask_mode < 0 || m->mask_mode > 1) return ORACLE_EINVAL;
   if (m->d_spe > 0 && !m->spe) return ORACLE_EINVAL;
   if (m->ffn_mult != 4 || m->activation != 0) return ORACLE_EINVAL; /* FFN width 4d, ReLU */
   return ORACLE_OK;

@@ -112,6 +112,7 @@ int validate(const aecct_model_desc *d) {
   if (d->activation < 0 || d->activation > 1) return AECCT_ERR_INVALID_ARG;
   if (d->cluster_ctas < 0 || d->cluster_ctas > 64) return AECCT_ERR_INVALID_ARG;
   if (d->attention_mode < 0 || d->attention_mode > 2) return AECCT_ERR_INVALID_ARG;
+  if (d->mask_mode < 0 || d->mask_mode > 1) return AECCT_ERR_INVALID_ARG;
   if (!d->H || !d->emb || !d->w_packed || !d->w_scale || !d->bias || !d->ln_gamma || !d->ln_beta || !d->w_d1 ||
       !d->w_out || !d->b_out)
     return AECCT_ERR_INVALID_ARG;
@@ -295,6 +296,16 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
       }
       for (int u = 0; u < T; ++u)
         if (row[u]) nb[1][t].push_back(static_cast<uint16_t>(u));
+    }
+  }
+  if (d.mask_mode == 1) {
+    // ECCT code-aware mask (Sec. 3) for every head: the union of the two rings, ascending
+    for (int t = 0; t < T; ++t) {
+      std::vector<uint16_t> u;
+      std::merge(nb[0][t].begin(), nb[0][t].end(), nb[1][t].begin(), nb[1][t].end(), std::back_inserter(u));
+      u.erase(std::unique(u.begin(), u.end()), u.end());
+      nb[0][t] = u;
+      nb[1][t] = u;
     }
   }
   // Rows of a codeword hold its tokens sorted by attention work (keys over the thread's first-ring

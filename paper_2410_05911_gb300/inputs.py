@@ -343,6 +343,7 @@ class ModelTensors:
     b_out: np.ndarray  # [n]
     ln_eps: float = 1e-5
     alpha_floor: float = 1e-5
+    mask_mode: int = 0  # 0 = HPSA rings (Sec. 4.2); 1 = ECCT code-aware mask for all heads (Sec. 3)
 
     @property
     def T(self) -> int:

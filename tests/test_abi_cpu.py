@@ -65,6 +65,8 @@ def _status(model, **kw):
     (lambda m: m.H.__setitem__((0, slice(None)), 0), A.AECCT_ERR_INVALID_ARG),
     (lambda m: m.H.__setitem__((slice(None), 3), 0), A.AECCT_ERR_INVALID_ARG),
     (lambda m: setattr(m, "activation", 7), A.AECCT_ERR_INVALID_ARG),
+    (lambda m: setattr(m, "mask_mode", 2), A.AECCT_ERR_INVALID_ARG),
+    (lambda m: setattr(m, "mask_mode", -1), A.AECCT_ERR_INVALID_ARG),
     (lambda m: setattr(m, "activation", 1), A.AECCT_ERR_UNSUPPORTED),
     (lambda m: setattr(m, "ffn_mult", 2), A.AECCT_ERR_UNSUPPORTED),
 ])

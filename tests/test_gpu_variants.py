@@ -4,7 +4,9 @@ block, then logits, bits and syndromes):
 
 * the split of heads between the first-ring and second-ring masks (Sec. 4.2 uses half and
   half; App. C discusses other splits): h_first = 2 and 6 of 8 heads;
-* binary weights in {-1, +1} (App. D) in place of ternary ones, through the same 2-bit format.
+* binary weights in {-1, +1} (App. D) in place of ternary ones, through the same 2-bit format;
+* the ECCT code-aware mask (Sec. 3; the CASA baseline the paper compares HPSA with): every head
+  attends over the union of the two rings (mask_mode = 1).
 """
 import numpy as np
 import pytest
@@ -24,6 +26,9 @@ CASES = [
     ("bch31_16", 32, 2, dict(binary=True, h_first=6), (1, 2)),
     ("ldpc128_64", 128, 2, dict(h_first=6), (1,)),
     ("bch63_36", 128, 1, dict(binary=True), (1,)),
+    ("bch31_16", 32, 2, dict(mask_mode=1), (1, 2)),
+    ("polar64_32", 64, 2, dict(mask_mode=1), (1, 2)),
+    ("ldpc128_64", 128, 1, dict(mask_mode=1), (1,)),
 ]
 
 
@@ -41,7 +46,10 @@ def _capture_equal(g, r):
 def test_variant_exact(case):
     key, d, layers, var, modes = case
     code = I.make_code(key)
+    var = dict(var)
+    mask_mode = var.pop("mask_mode", 0)
     model = I.random_model(code, d, layers, seed=77, zero_frac=0.5, **var)
+    model.mask_mode = mask_mode
     if var.get("binary"):
         assert all((np.abs(t) == 1).all() for wl in model.w_tern for t in wl)
     B = 9
