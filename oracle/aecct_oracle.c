@@ -26,6 +26,7 @@
  *     except where fmaf() is written explicitly;
  *   - sums over a feature row use pairwise summation (recursive halving);
  *   - attention scores are taken in base-2 units: sigma = dot(q,k) * fp32(log2(e)/sqrt(d_h)),
+ *     with dot(q,k) = (even-feature FMA chain) + (odd-feature FMA chain), each in feature order,
  *     p = 2^(sigma - max sigma), with 2^x evaluated by exp2_series() below (range
  *     reduction x = n + f, |f| <= 1/2, and the degree-7 Taylor series of e^(f ln 2));
  *   - sums over keys and over tokens run in ascending index order.
@@ -242,6 +243,17 @@ void oracle_layernorm_row(const float *v, int d, const float *g, const float *b,
  * heads e < h_first attend over M1, the rest over M2.  Masked-out keys are skipped.
  * sigma_u = dot(Q_t, K_u) * c, c = fp32(log2(e)/sqrt(dh)); p_u = 2^(sigma_u - max);
  * A_t = (sum_u p_u V_u) * (1 / sum_u p_u).  A row with no key gets zeros. */
+/* q . k over one head (Sec. 4.2): the even-indexed and the odd-indexed feature products each
+ * summed by a chain of fused multiply-adds in feature order, then added (canonical order). */
+static float oracle_dot(const float *q, const float *k, int dh) {
+  float de = 0.0f, dod = 0.0f;
+  for (int i = 0; i < dh; i += 2) {
+    de = fmaf(q[i], k[i], de);
+    dod = fmaf(q[i + 1], k[i + 1], dod);
+  }
+  return de + dod;
+}
+
 void oracle_attention(const float *Q, const float *K, const float *V, int T, int d, int heads,
                       int h_first, const uint8_t *M1, const uint8_t *M2, float *A) {
   int dh = d / heads;
@@ -255,9 +267,7 @@ void oracle_attention(const float *Q, const float *K, const float *V, int T, int
       for (int u = 0; u < T; ++u) {
         if (!M[u]) continue;
         const float *kk = K + (size_t)u * d + e * dh;
-        float dot = 0.0f;
-        for (int i = 0; i < dh; ++i) dot = fmaf(q[i], kk[i], dot);
-        float s = dot * c;
+        float s = oracle_dot(q, kk, dh) * c;
         if (!any || s > mx) mx = s;
         any = 1;
       }
@@ -273,9 +283,7 @@ void oracle_attention(const float *Q, const float *K, const float *V, int T, int
         if (!M[u]) continue;
         const float *kk = K + (size_t)u * d + e * dh;
         const float *vv = V + (size_t)u * d + e * dh;
-        float dot = 0.0f;
-        for (int i = 0; i < dh; ++i) dot = fmaf(q[i], kk[i], dot);
-        float p = oracle_exp2_series(dot * c - mx);
+        float p = oracle_exp2_series(oracle_dot(q, kk, dh) * c - mx);
         l = l + p;
         for (int i = 0; i < dh; ++i) num[i] = fmaf(p, vv[i], num[i]);
       }
@@ -479,7 +487,7 @@ static int validate(const oracle_model *m) {
     return ORACLE_EINVAL;
   if (m->n <= 0 || m->k <= 0 || m->k >= m->n || m->d <= 0 || m->heads <= 0 || m->d % m->heads) return ORACLE_EINVAL;
   if (m->d & (m->d - 1)) return ORACLE_EINVAL; /* pairwise LN sums take a power-of-two width */
-  if (m->d > 1024 || m->d / m->heads > 64 || m->n_layers < 0) return ORACLE_EINVAL;
+  if (m->d > 1024 || m->d / m->heads > 64 || (m->d / m->heads) % 2 || m->n_layers < 0) return ORACLE_EINVAL;
   if (m->h_first < 0 || m->h_first > m->heads || m->d_spe < 0 || m->d_spe >= m->d) return ORACLE_EINVAL;
   if (m->mask_mode < 0 || m->mask_mode > 1) return ORACLE_EINVAL;
   if (m->d_spe > 0 && !m->spe) return ORACLE_EINVAL;

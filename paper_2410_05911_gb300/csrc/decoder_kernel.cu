@@ -259,16 +259,16 @@ __device__ __forceinline__ void hpsa_head(const float *q, uint32_t info, bool ac
     const int ru = rowbase + off;
     return reinterpret_cast<const float4 *>(kvgen[ru >> 7] + static_cast<uint32_t>(ru & 127) * STRIDE + hoff);
   };
+  // q . k in the canonical order: even-feature and odd-feature FMA chains (the two lanes of
+  // paired FMAs over adjacent features), then their sum
   auto dotk = [&](const float4 *kk) -> float {
-    float dot = 0.0f;
+    float2 d = make_float2(0.0f, 0.0f);
 #pragma unroll
     for (int i = 0; i < DH / 4; ++i) {
-      dot = __fmaf_rn(q[4 * i], kk[i].x, dot);
-      dot = __fmaf_rn(q[4 * i + 1], kk[i].y, dot);
-      dot = __fmaf_rn(q[4 * i + 2], kk[i].z, dot);
-      dot = __fmaf_rn(q[4 * i + 3], kk[i].w, dot);
+      d = fma2(make_float2(q[4 * i], q[4 * i + 1]), make_float2(kk[i].x, kk[i].y), d);
+      d = fma2(make_float2(q[4 * i + 2], q[4 * i + 3]), make_float2(kk[i].z, kk[i].w), d);
     }
-    return dot;
+    return __fadd_rn(d.x, d.y);
   };
   // pass 1: scores and their maximum
   float mx = -INFINITY;
@@ -361,18 +361,18 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
                                           const uint8_t *rows, uint32_t kslot, float scale, uint32_t tcache,
                                           float *A) {
   auto kptr = [&](int off) { return reinterpret_cast<const float4 *>(rows + off * STRIDE + kslot); };
-  // dot products of q with two keys: lane x for key a, lane y for key b (FMA chains in feature order)
-  auto dot2 = [&](const float4 *ka, const float4 *kb) -> float2 {
+  // q . k (canonical order: even-feature and odd-feature FMA chains, then their sum); the two
+  // chains are the two lanes of paired FMAs over adjacent features
+  auto dot = [&](const float4 *k) -> float {
     float2 d = make_float2(0.0f, 0.0f);
 #pragma unroll
     for (int i = 0; i < DH / 4; ++i) {
-      d = fma2(make_float2(q[4 * i], q[4 * i]), make_float2(ka[i].x, kb[i].x), d);
-      d = fma2(make_float2(q[4 * i + 1], q[4 * i + 1]), make_float2(ka[i].y, kb[i].y), d);
-      d = fma2(make_float2(q[4 * i + 2], q[4 * i + 2]), make_float2(ka[i].z, kb[i].z), d);
-      d = fma2(make_float2(q[4 * i + 3], q[4 * i + 3]), make_float2(ka[i].w, kb[i].w), d);
+      d = fma2(make_float2(q[4 * i], q[4 * i + 1]), make_float2(k[i].x, k[i].y), d);
+      d = fma2(make_float2(q[4 * i + 2], q[4 * i + 3]), make_float2(k[i].z, k[i].w), d);
     }
-    return d;
+    return __fadd_rn(d.x, d.y);
   };
+  auto dot2 = [&](const float4 *ka, const float4 *kb) -> float2 { return make_float2(dot(ka), dot(kb)); };
   const float2 sc = make_float2(scale, scale);
   constexpr int U = 4;
   // membership bits of a 16-key block (jb is a multiple of 16)
