@@ -121,8 +121,8 @@ struct DecodeParams {
   float b_d1;
   const float *w_out;    // [T][n]
   const float *b_out;    // [n]
-  const uint32_t *hrow_off;  // [m + 1] check i -> variables
-  const uint16_t *hrow_idx;
+  const uint32_t *hbits;  // [m][hwords] row i of H as a bitmask over the variables (bit j%32 of word j/32)
+  int hwords;             // ceil(n / 32)
   const uint16_t *perm;         // [T] row offset within a codeword -> token
   const uint16_t *pos;          // [T] token -> row offset within its codeword
   // HPSA neighbour lists, 0 = first ring, 1 = second ring.  mask_info[mk][t] = (start << 11) | count:
@@ -177,7 +177,8 @@ struct SmemLayout {
   static constexpr uint32_t kOffRed = kOffW + kStages * kStageBytes;  // 2 x 4 x 128 floats
   static constexpr uint32_t kOffZ = kOffRed + 4096;                   // 128 floats
   static constexpr uint32_t kOffObits = kOffZ + 512;                  // decoded bits
-  static constexpr uint32_t kOffBar = kOffObits + kOutBitsBytes;      // mbarriers
+  static constexpr uint32_t kOffBitWords = kOffObits + kOutBitsBytes;  // 128 words: bitmasks of a group's words
+  static constexpr uint32_t kOffBar = kOffBitWords + 512;              // mbarriers
   static constexpr uint32_t kOffMisc = kOffBar + 256;  // tmem base, abort flag, peer bases, copy count
   static constexpr uint32_t kTotal = kOffMisc + 256;
   // QKV / FFN1 accumulators in [0, 4D) (x parked in [3D, 4D) during attention).  Attention

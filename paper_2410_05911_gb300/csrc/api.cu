@@ -42,8 +42,9 @@ struct aecct_handle {
   int n_chunks = 0;
   ChunkDesc chunks[32] = {};  // WeightSchedule<d> order
   float *lparams = nullptr, *emb = nullptr, *spe = nullptr, *w_d1 = nullptr, *w_out = nullptr, *b_out = nullptr;
-  uint32_t *hrow_off = nullptr, *mask_info[2] = {nullptr, nullptr};
-  uint16_t *hrow_idx = nullptr, *mask_list[2] = {nullptr, nullptr};
+  uint32_t *hbits = nullptr, *mask_info[2] = {nullptr, nullptr};
+  int hwords = 0;
+  uint16_t *mask_list[2] = {nullptr, nullptr};
   uint16_t *perm = nullptr, *pos = nullptr;
   uint16_t *plan_task = nullptr;
   uint32_t *plan_grp = nullptr, *plan_uinfo = nullptr, *plan_mask = nullptr;
@@ -224,6 +225,7 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
     best_C = C, best_G = G;
   }
   if (!best_C) return d.cluster_ctas ? AECCT_ERR_INVALID_ARG : AECCT_ERR_UNSUPPORTED;
+  if (best_G * ((n + 31) / 32) > 128) return AECCT_ERR_UNSUPPORTED;  // hard-decision bitmasks of a group
 
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -254,14 +256,12 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
   h->att_scale = static_cast<float>(1.4426950408889634074 / std::sqrt(static_cast<double>(D / kHeads)));
   h->wait_limit = d.wait_limit_cycles ? d.wait_limit_cycles : (1LL << 32);
 
-  // ---- H rows (check -> variables) for the syndromes
-  std::vector<uint32_t> hoff(m + 1, 0);
-  std::vector<uint16_t> hidx;
-  for (int i = 0; i < m; ++i) {
+  // ---- H rows as bitmasks over the variables, for the syndromes (parity of popcounts)
+  h->hwords = (n + 31) / 32;
+  std::vector<uint32_t> hbits((size_t)m * h->hwords, 0u);
+  for (int i = 0; i < m; ++i)
     for (int j = 0; j < n; ++j)
-      if (d.H[(size_t)i * n + j]) hidx.push_back(static_cast<uint16_t>(j));
-    hoff[i + 1] = static_cast<uint32_t>(hidx.size());
-  }
+      if (d.H[(size_t)i * n + j]) hbits[(size_t)i * h->hwords + j / 32] |= 1u << (j % 32);
   // ---- HPSA neighbour lists (Sec. 4.2): token t < n is variable t, token n + i is check i.
   // First ring: Tanner-graph neighbours.  Second ring: same-type nodes at distance two, and the
   // node itself.  Lists are in ascending token order (the order the softmax sums run in).
@@ -470,8 +470,7 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
       (rc = dev_upload(h, &h->w_d1, d.w_d1, (size_t)D)) ||
       (rc = dev_upload(h, &h->w_out, d.w_out, (size_t)T * n)) ||
       (rc = dev_upload(h, &h->b_out, d.b_out, (size_t)n)) ||
-      (rc = dev_upload(h, &h->hrow_off, hoff.data(), hoff.size())) ||
-      (rc = dev_upload(h, &h->hrow_idx, hidx.data(), hidx.size())) ||
+      (rc = dev_upload(h, &h->hbits, hbits.data(), hbits.size())) ||
       (rc = dev_upload(h, &h->perm, perm.data(), perm.size())) ||
       (rc = dev_upload(h, &h->pos, pos.data(), pos.size())) ||
       (rc = dev_upload(h, &h->mask_info[0], minfo[0].data(), minfo[0].size())) ||
@@ -534,7 +533,7 @@ int aecct_decode(aecct_handle *h, const float *y_dev, int64_t B, uint8_t *bits_d
   p.y = y_dev, p.bits = bits_dev, p.syn = syndrome_dev, p.logits = logits_dev;
   p.wstream = h->wstream, p.layer_bytes = h->layer_bytes;
   p.lparams = h->lparams, p.emb = h->emb, p.spe = h->spe, p.w_d1 = h->w_d1, p.b_d1 = h->b_d1;
-  p.w_out = h->w_out, p.b_out = h->b_out, p.hrow_off = h->hrow_off, p.hrow_idx = h->hrow_idx;
+  p.w_out = h->w_out, p.b_out = h->b_out, p.hbits = h->hbits, p.hwords = h->hwords;
   p.perm = h->perm, p.pos = h->pos;
   p.plan_task = h->plan_task;
   p.plan_grp = reinterpret_cast<const uint4 *>(h->plan_grp);

@@ -908,6 +908,8 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
     RowRed red{reinterpret_cast<float *>(smem + L::kOffRed), 0};
     float *zbuf = reinterpret_cast<float *>(smem + L::kOffZ);
     uint8_t *obits = smem + L::kOffObits;
+    uint32_t *bitw = reinterpret_cast<uint32_t *>(smem + L::kOffBitWords);  // [G][hwords] bitmasks
+    const int W = p.hwords;
     const uint32_t qbar = 1 + qd;  // named barrier of the 4 warps sharing a lane quadrant
     const int T = p.T, n = p.n, m = p.m, de = D - p.d_spe;
     const int W4 = 4 * D;
@@ -992,6 +994,14 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           asm volatile("prefetch.global.L2 [%0];" ::"l"(p.y + y1 + i));
       }
       if (named_bar_or(5, kEpiThreads, *s_abort != 0)) break;
+      // hard decisions of the group's words as bitmasks (one warp ballot per 32 variables)
+      for (int wi = warp; wi < p.G * W; wi += kEpiWarps) {
+        const int gw = wi / W, j = 32 * (wi - gw * W) + lane;
+        const bool neg = j < n && gi * p.G + gw < p.B && ybuf[gw * n + j] < 0.0f;
+        const uint32_t word = __ballot_sync(0xffffffffu, neg);
+        if (lane == 0) bitw[wi] = word;
+      }
+      named_bar_sync(5, kEpiThreads);
       const int rho = static_cast<int>(crank) * kRows + r;
       const int g = rho / T;
       const int t = __ldg(p.perm + (rho - g * T));  // token held by this row (rows are ordered by attention work)
@@ -1011,9 +1021,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             h = fabsf(yrow[t]);
           } else {
             const int i = t - n;
+            // s_i = parity of H_i AND b(y) (Sec. 3), over the bitmask words
             uint32_t par = 0;
-            for (uint32_t e = __ldg(p.hrow_off + i); e < __ldg(p.hrow_off + i + 1); ++e)
-              par ^= (yrow[__ldg(p.hrow_idx + e)] < 0.0f) ? 1u : 0u;
+            for (int w = 0; w < W; ++w) par += __popc(__ldg(p.hbits + i * W + w) & bitw[g * W + w]);
+            par &= 1u;
             h = __fsub_rn(1.0f, __fmul_rn(2.0f, static_cast<float>(par)));
             if (cap && sl == 0 && p.cap_syn) p.cap_syn[b * m + i] = static_cast<uint8_t>(par);
           }
@@ -1365,30 +1376,35 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           ztok[it] = *reinterpret_cast<const float *>(s_zgen[ru >> 7] + static_cast<uint32_t>(ru & 127) * 4u);
         }
         named_bar_sync(5, kEpiThreads);
-        const int items = n_local * n;
-        for (int it = tid; it < items; it += kEpiThreads) {
-          const int li = it / n, j = it - li * n;
+        // one warp per 32 variables of a word, so that the decoded bits come out as bitmask words
+        const int witems = n_local * W * 32;
+        for (int it = tid; it < (witems + 31) / 32 * 32; it += kEpiThreads) {
+          const int li = it / (W * 32), j = it - li * (W * 32);
           const int gg = static_cast<int>(crank) + li * p.C;
           const int64_t bb = gi * p.G + gg;
-          if (bb >= p.B) continue;
-          // eps_j = sum over t in token order of W_o[t][j] z_t (one FMA chain), loads ahead
-          const float *zl = ztok + li * T;
-          const float *wo = p.w_out + j;
-          float acc = 0.0f;
-          int tt = 0;
-          for (; tt + 8 <= T; tt += 8) {
-            float wv[8];
+          const bool valid = it < witems && j < n && bb < p.B;
+          bool bit = false;
+          if (valid) {
+            // eps_j = sum over t in token order of W_o[t][j] z_t (one FMA chain), loads ahead
+            const float *zl = ztok + li * T;
+            const float *wo = p.w_out + j;
+            float acc = 0.0f;
+            int tt = 0;
+            for (; tt + 8 <= T; tt += 8) {
+              float wv[8];
 #pragma unroll
-            for (int u = 0; u < 8; ++u) wv[u] = __ldg(wo + (tt + u) * n);
+              for (int u = 0; u < 8; ++u) wv[u] = __ldg(wo + (tt + u) * n);
 #pragma unroll
-            for (int u = 0; u < 8; ++u) acc = __fmaf_rn(wv[u], zl[tt + u], acc);
+              for (int u = 0; u < 8; ++u) acc = __fmaf_rn(wv[u], zl[tt + u], acc);
+            }
+            for (; tt < T; ++tt) acc = __fmaf_rn(__ldg(wo + tt * n), zl[tt], acc);
+            const float eps = __fadd_rn(acc, __ldg(p.b_out + j));
+            bit = __fmul_rn(__ldg(p.y + bb * n + j), eps) < 0.0f;  // y was staged; re-read from L1/L2
+            p.bits[bb * n + j] = bit ? 1 : 0;
+            if (p.logits) p.logits[bb * n + j] = eps;
           }
-          for (; tt < T; ++tt) acc = __fmaf_rn(__ldg(wo + tt * n), zl[tt], acc);
-          const float eps = __fadd_rn(acc, __ldg(p.b_out + j));
-          const uint8_t bit = (__fmul_rn(__ldg(p.y + bb * n + j), eps) < 0.0f) ? 1 : 0;  // y was staged; re-read from L1/L2
-          p.bits[bb * n + j] = bit;
-          if (p.logits) p.logits[bb * n + j] = eps;
-          obits[li * n + j] = bit;
+          const uint32_t word = __ballot_sync(0xffffffffu, bit);
+          if (lane == 0 && it < witems) bitw[it / 32] = word;
         }
         named_bar_sync(5, kEpiThreads);
         if (p.syn) {
@@ -1399,9 +1415,8 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             const int64_t bb = gi * p.G + gg;
             if (bb >= p.B) continue;
             uint32_t par = 0;
-            for (uint32_t e = __ldg(p.hrow_off + i); e < __ldg(p.hrow_off + i + 1); ++e)
-              par ^= obits[li * n + __ldg(p.hrow_idx + e)];
-            p.syn[bb * m + i] = static_cast<uint8_t>(par);
+            for (int w = 0; w < W; ++w) par += __popc(__ldg(p.hbits + i * W + w) & bitw[li * W + w]);
+            p.syn[bb * m + i] = static_cast<uint8_t>(par & 1u);
           }
         }
         cluster_arrive(bar_zf);  // this CTA no longer reads any z of this group; obits free
