@@ -25,6 +25,8 @@
 // the results are bit-identical to any implementation that follows the same order.
 #include <cuda_runtime.h>
 
+#include <type_traits>
+
 #include "aecct_internal.h"
 #include "sm103_ptx.cuh"
 
@@ -389,7 +391,9 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
     const uint32_t seg = segment(jb);
     const int nk = min(16, cnt - jb);
     float sgs[16];
-    if (nk == 16) {
+    // the 16 keys of a full segment; DENSE: every lane holds all of them (no membership tests)
+    auto full_segment = [&](auto dense_tag) {
+      constexpr bool DENSE = decltype(dense_tag)::value;
 #pragma unroll
       for (int k0 = 0; k0 < 16; k0 += U) {
         float4 kk[U][DH / 4];
@@ -403,10 +407,14 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
         for (int k = 0; k < U; k += 2) {
           const float2 sg = mul2(dot2(kk[k], kk[k + 1]), sc);
           sgs[k0 + k] = sg.x, sgs[k0 + k + 1] = sg.y;
-          if (((seg >> (k0 + k)) & 1u)) mx = fmaxf(mx, sg.x);
-          if (((seg >> (k0 + k + 1)) & 1u)) mx = fmaxf(mx, sg.y);
+          if (DENSE || ((seg >> (k0 + k)) & 1u)) mx = fmaxf(mx, sg.x);
+          if (DENSE || ((seg >> (k0 + k + 1)) & 1u)) mx = fmaxf(mx, sg.y);
         }
       }
+    };
+    if (nk == 16) {
+      if (__all_sync(0xffffffffu, (seg & 0xFFFFu) == 0xFFFFu)) full_segment(std::true_type{});
+      else full_segment(std::false_type{});
     } else {
 #pragma unroll
       for (int k = 0; k < 16; k += 2) {
@@ -455,27 +463,33 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
       float sgs[16];
       tmem_ld<16>(tcache + jb, sgs);
       tmem_wait_ld();
+      // DENSE: a full segment held by every lane (no membership or range tests)
+      auto cached_segment = [&](auto dense_tag) {
+        constexpr bool DENSE = decltype(dense_tag)::value;
 #pragma unroll
-      for (int k0 = 0; k0 < 16; k0 += U) {
-        if (k0 < nk) {
-          float4 vv[U][DH / 4];
+        for (int k0 = 0; k0 < 16; k0 += U) {
+          if (DENSE || k0 < nk) {
+            float4 vv[U][DH / 4];
 #pragma unroll
-          for (int k = 0; k < U; ++k) {
-            const float4 *kp = kptr(byte_at(w, min(k0 + k, nk - 1)));
+            for (int k = 0; k < U; ++k) {
+              const float4 *kp = kptr(byte_at(w, DENSE ? k0 + k : min(k0 + k, nk - 1)));
 #pragma unroll
-            for (int i = 0; i < DH / 4; ++i) vv[k][i] = kp[DH / 4 + i];
-          }
-          float2 pr[U / 2];
+              for (int i = 0; i < DH / 4; ++i) vv[k][i] = kp[DH / 4 + i];
+            }
+            float2 pr[U / 2];
 #pragma unroll
-          for (int k = 0; k < U; k += 2)
-            pr[k / 2] = exp2_series2(make_float2(__fsub_rn(sgs[k0 + k], mx), __fsub_rn(sgs[k0 + k + 1], mx)));
+            for (int k = 0; k < U; k += 2)
+              pr[k / 2] = exp2_series2(make_float2(__fsub_rn(sgs[k0 + k], mx), __fsub_rn(sgs[k0 + k + 1], mx)));
 #pragma unroll
-          for (int k = 0; k < U; k += 2) {
-            if (k0 + k < nk && ((seg >> (k0 + k)) & 1u)) fold(pr[k / 2].x, vv[k]);
-            if (k0 + k + 1 < nk && ((seg >> (k0 + k + 1)) & 1u)) fold(pr[k / 2].y, vv[k + 1]);
+            for (int k = 0; k < U; k += 2) {
+              if (DENSE || (k0 + k < nk && ((seg >> (k0 + k)) & 1u))) fold(pr[k / 2].x, vv[k]);
+              if (DENSE || (k0 + k + 1 < nk && ((seg >> (k0 + k + 1)) & 1u))) fold(pr[k / 2].y, vv[k + 1]);
+            }
           }
         }
-      }
+      };
+      if (nk == 16 && __all_sync(0xffffffffu, (seg & 0xFFFFu) == 0xFFFFu)) cached_segment(std::true_type{});
+      else cached_segment(std::false_type{});
     } else if (nk == 16) {
 #pragma unroll
       for (int k0 = 0; k0 < 16; k0 += U) {
@@ -1156,7 +1170,9 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             const uint4 gi = __ldg(p.plan_grp + grp);
             const bool act = lane < static_cast<int>(gi.y);
             const int row = static_cast<int>(gi.x) + (act ? lane : 0);
-            const uint4 mk = act ? __ldg(p.plan_mask + (grp * 2 + ring) * 32 + lane) : make_uint4(0u, 0u, 0u, 0u);
+            // a lane past the group's rows computes on row 0 and its result is dropped; an all-ones
+            // mask keeps it from breaking the dense fast path
+            const uint4 mk = act ? __ldg(p.plan_mask + (grp * 2 + ring) * 32 + lane) : make_uint4(~0u, ~0u, ~0u, ~0u);
             const uint32_t ui = __ldg(p.plan_uinfo + grp * 2 + ring);
             float q[DH], a[DH];
             const float4 *qp = reinterpret_cast<const float4 *>(smem + L::kOffU + row * L::kKvStride + e * L::kSlot);
