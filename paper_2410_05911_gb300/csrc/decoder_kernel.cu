@@ -783,16 +783,24 @@ struct Issuer<128, TASKS> {
       wait(bar(1), parity<7>(lp));
       mmas<1, 7>();
       mma_commit_warp(bar_acc());
-      // FFN1 weights into region U once no CTA of the cluster reads this CTA's K/V any more;
-      // FFN2 chunk 18 into W2 (its last reader was the previous block's FFN2)
-      if (bc.cluster) wait(bc.kvf, bc.kvf_ph, true);
-      arm(3, 8 * kChunk);
-      copies<8, 16>(w_cur);
+      // FFN1 weights into region U: a one-CTA cluster has finished reading its K/V (every warp
+      // published the O operand); a larger cluster stages them at FFN1 instead, so that the O
+      // epilogue overlaps the peers' attention.  FFN2 chunk 18 into W2 (last read by the
+      // previous block's FFN2).
+      if (!bc.cluster) {
+        arm(3, 8 * kChunk);
+        copies<8, 16>(w_cur);
+      }
       copy1<18>(w_cur);
       wait(bar_acc(), 1);
       copy1<16>(w_cur);  // W0, W1 were O's
       copy1<17>(w_cur);
     } else if constexpr (G == 2) {
+      if (bc.cluster) {  // every CTA of the cluster is done with this CTA's K/V
+        wait(bc.kvf, bc.kvf_ph, true);
+        arm(3, 8 * kChunk);
+        copies<8, 16>(w_cur);
+      }
       wait(bar(3), 1);  // FFN1 weights in region U
       mmas_range<2, 8, 16>();
       mma_commit_warp(bar_acc());
