@@ -66,6 +66,10 @@ typedef struct aecct_handle aecct_handle; /* opaque */
  *   mask_mode     0 = HPSA (Sec. 4.2): heads [0, h_first) first ring, the rest second ring;
  *                 1 = the ECCT code-aware mask (Sec. 3) for every head: the union of the first
  *                 and second rings (which contains each node itself).  Other values are rejected.
+ *   alpha_mode    absmax granularity of eq. Quant (Sec. 4.1): 0 = one alpha per token row;
+ *                 1 = one alpha per quantised matrix of a codeword (the max over its T rows).
+ *                 1 needs one CTA per codeword (T <= 128 and cluster_ctas 0 or 1), else
+ *                 AECCT_ERR_UNSUPPORTED.
  *   H             [(n-k)][n] uint8 row-major, entries 0/1, no all-zero row or column.
  *   emb           [T][d-d_spe] fp32: token t's embedding row, scaled by h_t (Sec. 3, ECCT).
  *   spe           [T][d_spe] fp32: spectral positional encoding table (Sec. 4.3);
@@ -90,6 +94,7 @@ typedef struct aecct_handle aecct_handle; /* opaque */
  */
 typedef struct {
   int32_t n, k, d, n_layers, heads, h_first, d_spe, ffn_mult, activation, cluster_ctas, attention_mode, mask_mode;
+  int32_t alpha_mode;
   const uint8_t *H;
   const float *emb;
   const float *spe;

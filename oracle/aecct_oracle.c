@@ -52,6 +52,7 @@
 typedef struct {
   int32_t n, k, d, n_layers, heads, h_first, d_spe, ffn_mult, activation;
   int32_t mask_mode;       /* 0 = HPSA (Sec. 4.2); 1 = ECCT code-aware mask M1 | M2 for all heads (Sec. 3) */
+  int32_t alpha_mode;      /* 0 = one alpha per token (C-1); 1 = one alpha per quantised matrix of a word */
   const uint8_t *H;        /* [(n-k)][n] 0/1 */
   const float *emb;        /* [T][d-d_spe] */
   const float *spe;        /* [T][d_spe] */
@@ -163,13 +164,16 @@ void oracle_masks(const uint8_t *H, int m, int n, uint8_t *M1, uint8_t *M2) {
 /* Sec. 4.1 eq. Quant, one token row: alpha = ||x||_inf, Q_b = 127,
  * q = RoundClip(x * (Q_b / alpha), -Q_b, Q_b), round half to even.
  * alpha is floored at alpha_floor so an all-zero row quantises to zeros. */
-void oracle_quant_row(const float *x, int len, float alpha_floor, int8_t *q, float *alpha_out) {
+static float absmax(const float *x, int len) {
   float a = 0.0f;
   for (int i = 0; i < len; ++i) {
     float ax = fabsf(x[i]);
     if (ax > a) a = ax;
   }
-  if (!(a > alpha_floor)) a = alpha_floor;
+  return a;
+}
+/* q = RoundClip(x * (Q_b / a), -Q_b, Q_b) for a given (floored) alpha a */
+static void quant_with_alpha(const float *x, int len, float a, int8_t *q) {
   float r = 127.0f / a;
   for (int i = 0; i < len; ++i) {
     float v = rintf(x[i] * r);
@@ -177,7 +181,23 @@ void oracle_quant_row(const float *x, int len, float alpha_floor, int8_t *q, flo
     if (v < -127.0f) v = -127.0f;
     q[i] = (int8_t)v;
   }
+}
+void oracle_quant_row(const float *x, int len, float alpha_floor, int8_t *q, float *alpha_out) {
+  float a = absmax(x, len);
+  if (!(a > alpha_floor)) a = alpha_floor;
+  quant_with_alpha(x, len, a, q);
   *alpha_out = a;
+}
+/* The alternative granularity (Sec. 4.1 writes alpha as a scalar of the whole input x in
+ * R^{m x n}): alpha = ||x||_inf over all rows of a word's matrix, floored. */
+static float matrix_alpha(const float *x, int rows, int len, size_t stride, float alpha_floor) {
+  float a = 0.0f;
+  for (int t = 0; t < rows; ++t) {
+    float r = absmax(x + (size_t)t * stride, len);
+    if (r > a) a = r;
+  }
+  if (!(a > alpha_floor)) a = alpha_floor;
+  return a;
 }
 
 /* Sec. 4.1 eq. AAPLinear for one row: acc_o = sum_i q_i t_oi (exact integer), then
@@ -339,11 +359,14 @@ static void decode_one(const oracle_model *m, const float *y, uint8_t *bits, uin
     const float *bq = m->bias + blayer * l, *bk = bq + d, *bv = bk + d, *bo = bv + d, *b1 = bo + d, *b2 = b1 + F;
     const float *g1 = m->ln_gamma + (size_t)2 * d * l, *g2 = g1 + d;
     const float *be1 = m->ln_beta + (size_t)2 * d * l, *be2 = be1 + d;
+    const int per_word = m->alpha_mode == 1;
     /* S3/S4: Quant(x) and the Q, K, V AAP-linear layers (Sec. 4.1) */
+    const float aw0 = per_word ? matrix_alpha(w->x, T, d, (size_t)d, m->alpha_floor) : 0.0f;
     for (int t = 0; t < T; ++t) {
       int8_t *qr = w->q + (size_t)t * F;
       float al;
-      oracle_quant_row(w->x + (size_t)t * d, d, m->alpha_floor, qr, &al);
+      if (per_word) quant_with_alpha(w->x + (size_t)t * d, d, al = aw0, qr);
+      else oracle_quant_row(w->x + (size_t)t * d, d, m->alpha_floor, qr, &al);
       int32_t *ar = w->acc + (size_t)t * 3 * d;
       oracle_aap_linear_row(qr, al, d, Wq, d, sw[0], bq, ar, w->qf + (size_t)t * d);
       oracle_aap_linear_row(qr, al, d, Wk, d, sw[1], bk, ar + d, w->kf + (size_t)t * d);
@@ -358,11 +381,13 @@ static void decode_one(const oracle_model *m, const float *y, uint8_t *bits, uin
     /* S5: HPSA (Sec. 4.2) */
     oracle_attention(w->qf, w->kf, w->vf, T, d, m->heads, m->h_first, w->M1, w->M2, w->a);
     /* S6: O projection, residual, LayerNorm (Post-LN, Sec. 5) */
+    const float aw1 = per_word ? matrix_alpha(w->a, T, d, (size_t)d, m->alpha_floor) : 0.0f;
     for (int t = 0; t < T; ++t) {
       int8_t *qr = w->q + (size_t)t * F;
       float al;
       int32_t *ar = w->acc + (size_t)t * 4 * d;
-      oracle_quant_row(w->a + (size_t)t * d, d, m->alpha_floor, qr, &al);
+      if (per_word) quant_with_alpha(w->a + (size_t)t * d, d, al = aw1, qr);
+      else oracle_quant_row(w->a + (size_t)t * d, d, m->alpha_floor, qr, &al);
       oracle_aap_linear_row(qr, al, d, Wo, d, sw[3], bo, ar, w->o + (size_t)t * d);
       for (int c = 0; c < d; ++c) w->v[c] = w->x[(size_t)t * d + c] + w->o[(size_t)t * d + c];
       oracle_layernorm_row(w->v, d, g1, be1, m->ln_eps, w->x + (size_t)t * d);
@@ -374,20 +399,31 @@ static void decode_one(const oracle_model *m, const float *y, uint8_t *bits, uin
       }
     }
     /* S7/S8: FFN with ReLU (Sec. 4 item 4), residual, LayerNorm */
+    const float aw2 = per_word ? matrix_alpha(w->x, T, d, (size_t)d, m->alpha_floor) : 0.0f;
     for (int t = 0; t < T; ++t) {
       int8_t *qr = w->q + (size_t)t * F;
       float al;
       int32_t *ar = w->acc + (size_t)t * 4 * d;
-      oracle_quant_row(w->x + (size_t)t * d, d, m->alpha_floor, qr, &al);
-      oracle_aap_linear_row(qr, al, d, W1, F, sw[4], b1, ar, w->u);
+      float *ur = w->u + (size_t)t * F;
+      if (per_word) quant_with_alpha(w->x + (size_t)t * d, d, al = aw2, qr);
+      else oracle_quant_row(w->x + (size_t)t * d, d, m->alpha_floor, qr, &al);
+      oracle_aap_linear_row(qr, al, d, W1, F, sw[4], b1, ar, ur);
       if (capture) {
         int64_t off = cap_row_off(m, bi, l, 2, t);
         if (cap->q) memcpy(cap->q + off, qr, (size_t)d);
         if (cap->acc) memcpy(cap->acc + off, ar, sizeof(int32_t) * F);
         if (cap->alpha) cap->alpha[off / (4 * d)] = al;
       }
-      for (int c = 0; c < F; ++c) w->u[c] = w->u[c] > 0.0f ? w->u[c] : 0.0f;
-      oracle_quant_row(w->u, F, m->alpha_floor, qr, &al);
+      for (int c = 0; c < F; ++c) ur[c] = ur[c] > 0.0f ? ur[c] : 0.0f;
+    }
+    const float aw3 = per_word ? matrix_alpha(w->u, T, F, (size_t)F, m->alpha_floor) : 0.0f;
+    for (int t = 0; t < T; ++t) {
+      int8_t *qr = w->q + (size_t)t * F;
+      float al;
+      int32_t *ar = w->acc + (size_t)t * 4 * d;
+      const float *ur = w->u + (size_t)t * F;
+      if (per_word) quant_with_alpha(ur, F, al = aw3, qr);
+      else oracle_quant_row(ur, F, m->alpha_floor, qr, &al);
       oracle_aap_linear_row(qr, al, F, W2, d, sw[5], b2, ar, w->o);
       for (int c = 0; c < d; ++c) w->v[c] = w->x[(size_t)t * d + c] + w->o[c];
       oracle_layernorm_row(w->v, d, g2, be2, m->ln_eps, w->x + (size_t)t * d);
@@ -427,7 +463,7 @@ static int work_alloc(const oracle_model *m, work_t *w) {
   w->vf = (float *)calloc((size_t)T * d, sizeof(float));
   w->a = (float *)calloc((size_t)T * d, sizeof(float));
   w->o = (float *)calloc((size_t)T * d, sizeof(float));
-  w->u = (float *)calloc((size_t)F, sizeof(float));
+  w->u = (float *)calloc((size_t)T * F, sizeof(float));
   w->v = (float *)calloc((size_t)(d > T ? d : T), sizeof(float));
   w->z = (float *)calloc((size_t)T, sizeof(float));
   w->eps = (float *)calloc((size_t)m->n, sizeof(float));
@@ -489,7 +525,7 @@ static int validate(const oracle_model *m) {
   if (m->d & (m->d - 1)) return ORACLE_EINVAL; /* pairwise LN sums take a power-of-two width */
   if (m->d > 1024 || m->d / m->heads > 64 || (m->d / m->heads) % 2 || m->n_layers < 0) return ORACLE_EINVAL;
   if (m->h_first < 0 || m->h_first > m->heads || m->d_spe < 0 || m->d_spe >= m->d) return ORACLE_EINVAL;
-  if (m->mask_mode < 0 || m->mask_mode > 1) return ORACLE_EINVAL;
+  if (m->mask_mode < 0 || m->mask_mode > 1 || m->alpha_mode < 0 || m->alpha_mode > 1) return ORACLE_EINVAL;
   if (m->d_spe > 0 && !m->spe) return ORACLE_EINVAL;
   if (m->ffn_mult != 4 || m->activation != 0) return ORACLE_EINVAL; /* FFN width 4d, ReLU */
   return ORACLE_OK;

@@ -40,6 +40,7 @@ class OracleModel(ctypes.Structure):
         ("n", ctypes.c_int32), ("k", ctypes.c_int32), ("d", ctypes.c_int32), ("n_layers", ctypes.c_int32),
         ("heads", ctypes.c_int32), ("h_first", ctypes.c_int32), ("d_spe", ctypes.c_int32),
         ("ffn_mult", ctypes.c_int32), ("activation", ctypes.c_int32), ("mask_mode", ctypes.c_int32),
+        ("alpha_mode", ctypes.c_int32),
         ("H", ctypes.c_void_p), ("emb", ctypes.c_void_p), ("spe", ctypes.c_void_p), ("w", ctypes.c_void_p),
         ("w_scale", ctypes.c_void_p), ("bias", ctypes.c_void_p), ("ln_gamma", ctypes.c_void_p),
         ("ln_beta", ctypes.c_void_p), ("w_d1", ctypes.c_void_p), ("b_d1", ctypes.c_float),
@@ -211,7 +212,7 @@ class _Packed:
             self.ln_beta = np.zeros(1, np.float32)
         self.st = OracleModel(
             model.n, model.k, model.d, model.n_layers, model.heads, model.h_first, model.d_spe, model.ffn_mult,
-            model.activation, int(getattr(model, "mask_mode", 0)), _p(self.H), _p(self.emb), _p(self.spe) if self.spe.size else None, _p(self.w),
+            model.activation, int(getattr(model, "mask_mode", 0)), int(getattr(model, "alpha_mode", 0)), _p(self.H), _p(self.emb), _p(self.spe) if self.spe.size else None, _p(self.w),
             _p(self.w_scale), _p(self.bias), _p(self.ln_gamma), _p(self.ln_beta), _p(self.w_d1),
             float(model.b_d1), _p(self.w_out), _p(self.b_out), float(model.ln_eps), float(model.alpha_floor))
 

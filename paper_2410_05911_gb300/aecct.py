@@ -41,6 +41,7 @@ class ModelDesc(ctypes.Structure):
         ("heads", ctypes.c_int32), ("h_first", ctypes.c_int32), ("d_spe", ctypes.c_int32),
         ("ffn_mult", ctypes.c_int32), ("activation", ctypes.c_int32), ("cluster_ctas", ctypes.c_int32),
         ("attention_mode", ctypes.c_int32), ("mask_mode", ctypes.c_int32),
+        ("alpha_mode", ctypes.c_int32),
         ("H", ctypes.c_void_p), ("emb", ctypes.c_void_p), ("spe", ctypes.c_void_p), ("w_packed", ctypes.c_void_p),
         ("w_scale", ctypes.c_void_p), ("bias", ctypes.c_void_p), ("ln_gamma", ctypes.c_void_p),
         ("ln_beta", ctypes.c_void_p), ("w_d1", ctypes.c_void_p), ("b_d1", ctypes.c_float),
@@ -140,7 +141,8 @@ class _HostModel:
         ptr = lambda a: a.ctypes.data if a.size else None  # noqa: E731
         self.desc = ModelDesc(
             model.n, model.k, model.d, model.n_layers, model.heads, model.h_first, model.d_spe, model.ffn_mult,
-            model.activation, int(cluster_ctas), int(attention_mode), int(getattr(model, "mask_mode", 0)), ptr(self.H), ptr(self.emb), ptr(self.spe), ptr(self.w_packed),
+            model.activation, int(cluster_ctas), int(attention_mode), int(getattr(model, "mask_mode", 0)),
+            int(getattr(model, "alpha_mode", 0)), ptr(self.H), ptr(self.emb), ptr(self.spe), ptr(self.w_packed),
             ptr(self.w_scale), ptr(self.bias), ptr(self.ln_gamma), ptr(self.ln_beta), ptr(self.w_d1),
             float(model.b_d1), ptr(self.w_out), ptr(self.b_out), float(model.ln_eps), float(model.alpha_floor),
             int(wait_limit_cycles))

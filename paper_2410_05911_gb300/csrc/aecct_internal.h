@@ -139,6 +139,7 @@ struct DecodeParams {
   const uint4 *plan_ulist;     // union lists: 16 row offsets (one byte each) per entry
   const uint4 *plan_mask;      // [groups][2][32 lanes]: 128 membership bits over the union list
   float ln_eps, alpha_floor, att_scale;
+  int alpha_mode;  // 0 = absmax alpha per token row, 1 = per quantised matrix of a word (C == 1)
   // integer-core capture (device, optional)
   int64_t cap_B;
   int8_t *cap_q;

@@ -33,6 +33,7 @@ struct aecct_handle {
   int n = 0, k = 0, T = 0, m = 0, d = 0, n_layers = 0, h_first = 0, d_spe = 0;
   int C = 1, G = 1, max_clusters = 0;
   bool tasks = false;  // warp-task attention (one CTA per group, d <= 64)
+  int alpha_mode = 0;  // 1 = one alpha per quantised matrix of a word
   float ln_eps = 0, alpha_floor = 0, att_scale = 0, b_d1 = 0;
   long long wait_limit = 0;
   int device = 0;
@@ -114,6 +115,7 @@ int validate(const aecct_model_desc *d) {
   if (d->cluster_ctas < 0 || d->cluster_ctas > 64) return AECCT_ERR_INVALID_ARG;
   if (d->attention_mode < 0 || d->attention_mode > 2) return AECCT_ERR_INVALID_ARG;
   if (d->mask_mode < 0 || d->mask_mode > 1) return AECCT_ERR_INVALID_ARG;
+  if (d->alpha_mode < 0 || d->alpha_mode > 1) return AECCT_ERR_INVALID_ARG;
   if (!d->H || !d->emb || !d->w_packed || !d->w_scale || !d->bias || !d->ln_gamma || !d->ln_beta || !d->w_d1 ||
       !d->w_out || !d->b_out)
     return AECCT_ERR_INVALID_ARG;
@@ -226,6 +228,7 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
   }
   if (!best_C) return d.cluster_ctas ? AECCT_ERR_INVALID_ARG : AECCT_ERR_UNSUPPORTED;
   if (best_G * ((n + 31) / 32) > 128) return AECCT_ERR_UNSUPPORTED;  // hard-decision bitmasks of a group
+  if (d.alpha_mode == 1 && best_C != 1) return AECCT_ERR_UNSUPPORTED;  // per-word alpha: one CTA per word
 
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -253,6 +256,7 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
   h->n = n, h->k = k, h->T = T, h->m = m, h->d = D, h->n_layers = d.n_layers, h->h_first = d.h_first;
   h->d_spe = d.d_spe, h->C = best_C, h->G = best_G, h->max_clusters = max_clusters, h->tasks = tasks;
   h->ln_eps = d.ln_eps, h->alpha_floor = d.alpha_floor, h->b_d1 = d.b_d1, h->device = dev;
+  h->alpha_mode = d.alpha_mode;
   h->att_scale = static_cast<float>(1.4426950408889634074 / std::sqrt(static_cast<double>(D / kHeads)));
   h->wait_limit = d.wait_limit_cycles ? d.wait_limit_cycles : (1LL << 32);
 
@@ -543,7 +547,7 @@ int aecct_decode(aecct_handle *h, const float *y_dev, int64_t B, uint8_t *bits_d
   p.mask_info[0] = h->mask_info[0], p.mask_info[1] = h->mask_info[1];
   p.mask_list[0] = reinterpret_cast<const uint4 *>(h->mask_list[0]);
   p.mask_list[1] = reinterpret_cast<const uint4 *>(h->mask_list[1]);
-  p.ln_eps = h->ln_eps, p.alpha_floor = h->alpha_floor, p.att_scale = h->att_scale;
+  p.ln_eps = h->ln_eps, p.alpha_floor = h->alpha_floor, p.att_scale = h->att_scale, p.alpha_mode = h->alpha_mode;
   p.cap_B = h->cap_B, p.cap_q = h->cap_q, p.cap_acc = h->cap_acc, p.cap_alpha = h->cap_alpha, p.cap_syn = h->cap_syn;
   p.err = h->d_err, p.wait_limit = h->wait_limit;
   cudaError_t e;

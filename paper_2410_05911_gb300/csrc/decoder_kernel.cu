@@ -947,6 +947,26 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
       red.sel ^= 1;
       return a;
     };
+    // Per-word alpha (alpha_mode 1, one CTA per word): the max of the row absmaxes over the rows
+    // of this row's codeword, through the z area (free until S9) and the bitmask area (free
+    // between the group start and S10).  Word g's rows are [g T, g T + T).
+    float *rowmax_s = reinterpret_cast<float *>(smem + L::kOffZ);
+    float *wordmax_s = reinterpret_cast<float *>(smem + L::kOffBitWords);
+    auto word_alpha = [&](float a_row) -> float {
+      if (p.alpha_mode == 0) return a_row;
+      if (sl == 0) rowmax_s[r] = a_row;
+      named_bar_sync(5, kEpiThreads);
+      if (warp < p.G) {
+        float a = 0.0f;
+        for (int i = lane; i < p.T; i += 32) a = fmaxf(a, rowmax_s[warp * p.T + i]);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, o));
+        if (lane == 0) wordmax_s[warp] = a;
+      }
+      named_bar_sync(5, kEpiThreads);
+      const int gw = (static_cast<int>(crank) * kRows + r) / p.T;
+      return gw < p.G ? wordmax_s[gw] : a_row;
+    };
     auto row_sum = [&](float v) -> float {
       *red.slot(sl, r) = v;
       named_bar_sync(qbar, 128);
@@ -1064,7 +1084,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         float a = 0.0f;
 #pragma unroll
         for (int j = 0; j < XS; ++j) a = fmaxf(a, fabsf(x[j]));
-        a = row_max(a);
+        a = word_alpha(row_max(a));
         a = (a > p.alpha_floor) ? a : p.alpha_floor;
         alpha_in = a;
         const float rr = __fdiv_rn(127.0f, a);
@@ -1218,7 +1238,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           float amax = 0.0f;
 #pragma unroll
           for (int j = 0; j < XS; ++j) amax = fmaxf(amax, fabsf(av[j]));
-          float a = row_max(amax);
+          float a = word_alpha(row_max(amax));
           a = (a > p.alpha_floor) ? a : p.alpha_floor;
           alpha_in = a;
           const float rr = __fdiv_rn(127.0f, a);
@@ -1259,7 +1279,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           }
           // Quant(A) -> O operand
           {
-            float a = row_max(amax);
+            float a = word_alpha(row_max(amax));
             a = (a > p.alpha_floor) ? a : p.alpha_floor;
             alpha_in = a;
             const float rr = __fdiv_rn(127.0f, a);
@@ -1324,7 +1344,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
               if constexpr (KEEP) uk[32 * ch + j] = u[j];
             }
           }
-          float a = row_max(umax);
+          float a = word_alpha(row_max(umax));
           a = (a > p.alpha_floor) ? a : p.alpha_floor;
           alpha_in = a;
           const float rr = __fdiv_rn(127.0f, a);

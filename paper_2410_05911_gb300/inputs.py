@@ -344,6 +344,7 @@ class ModelTensors:
     ln_eps: float = 1e-5
     alpha_floor: float = 1e-5
     mask_mode: int = 0  # 0 = HPSA rings (Sec. 4.2); 1 = ECCT code-aware mask for all heads (Sec. 3)
+    alpha_mode: int = 0  # 0 = one absmax alpha per token (C-1); 1 = one per quantised matrix of a word
 
     @property
     def T(self) -> int:

@@ -67,6 +67,7 @@ def _status(model, **kw):
     (lambda m: setattr(m, "activation", 7), A.AECCT_ERR_INVALID_ARG),
     (lambda m: setattr(m, "mask_mode", 2), A.AECCT_ERR_INVALID_ARG),
     (lambda m: setattr(m, "mask_mode", -1), A.AECCT_ERR_INVALID_ARG),
+    (lambda m: setattr(m, "alpha_mode", 2), A.AECCT_ERR_INVALID_ARG),
     (lambda m: setattr(m, "activation", 1), A.AECCT_ERR_UNSUPPORTED),
     (lambda m: setattr(m, "ffn_mult", 2), A.AECCT_ERR_UNSUPPORTED),
 ])
@@ -94,6 +95,10 @@ def test_create_rejects_invalid_packed_code_and_shapes():
     assert _status(I.workload_model("bch31_16"), attention_mode=3) == A.AECCT_ERR_INVALID_ARG
     assert _status(I.workload_model("ldpc128_64"), attention_mode=2) == A.AECCT_ERR_UNSUPPORTED
     assert _status(I.workload_model("bch63_36"), attention_mode=2) == A.AECCT_ERR_UNSUPPORTED
+    # one alpha per word needs one CTA per word
+    m2 = copy.deepcopy(I.workload_model("ldpc128_64"))
+    m2.alpha_mode = 1
+    assert _status(m2) == A.AECCT_ERR_UNSUPPORTED
     # NULL description / output pointer
     assert A.load().aecct_create(None, ctypes.byref(h)) == A.AECCT_ERR_INVALID_ARG
     assert A.load().aecct_create(ctypes.byref(hm.desc), None) == A.AECCT_ERR_INVALID_ARG

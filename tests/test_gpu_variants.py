@@ -6,7 +6,9 @@ block, then logits, bits and syndromes):
   half; App. C discusses other splits): h_first = 2 and 6 of 8 heads;
 * binary weights in {-1, +1} (App. D) in place of ternary ones, through the same 2-bit format;
 * the ECCT code-aware mask (Sec. 3; the CASA baseline the paper compares HPSA with): every head
-  attends over the union of the two rings (mask_mode = 1).
+  attends over the union of the two rings (mask_mode = 1);
+* one absmax alpha per quantised matrix of a word instead of per token (alpha_mode = 1, the
+  other reading of Sec. 4.1's scalar alpha of x).
 """
 import numpy as np
 import pytest
@@ -29,6 +31,9 @@ CASES = [
     ("bch31_16", 32, 2, dict(mask_mode=1), (1, 2)),
     ("polar64_32", 64, 2, dict(mask_mode=1), (1, 2)),
     ("ldpc128_64", 128, 1, dict(mask_mode=1), (1,)),
+    ("bch31_16", 32, 2, dict(alpha_mode=1), (1, 2)),
+    ("polar64_32", 64, 2, dict(alpha_mode=1), (1, 2)),
+    ("bch63_36", 128, 1, dict(alpha_mode=1, mask_mode=1), (1,)),
 ]
 
 
@@ -48,8 +53,10 @@ def test_variant_exact(case):
     code = I.make_code(key)
     var = dict(var)
     mask_mode = var.pop("mask_mode", 0)
+    alpha_mode = var.pop("alpha_mode", 0)
     model = I.random_model(code, d, layers, seed=77, zero_frac=0.5, **var)
     model.mask_mode = mask_mode
+    model.alpha_mode = alpha_mode
     if var.get("binary"):
         assert all((np.abs(t) == 1).all() for wl in model.w_tern for t in wl)
     B = 9

@@ -38,9 +38,11 @@ def ln64(v, g, b, eps):
     return (v - mu) / np.sqrt(var + eps) * g + b
 
 
-def check_quant(x, q, alpha, floor, label):
-    # per token (C-1): alpha_t = max(max_i |x_ti|, floor)
+def check_quant(x, q, alpha, floor, label, per_word=False):
+    # per token (C-1): alpha_t = max(max_i |x_ti|, floor); per word: one max over the matrix
     a = np.maximum(np.abs(x).max(1), floor)
+    if per_word:
+        a = np.full_like(a, a.max())
     assert (np.abs(alpha - a) <= 1e-5 * a).all(), f"{label}: alpha {alpha} vs {a}"
     v = x * (127.0 / a)[:, None]
     ref = np.rint(v)
@@ -59,6 +61,7 @@ def forward64(model, y, cap):
     F = model.ffn_mult * d
     M1, M2 = masks64(H, model.mask_mode)
     q, acc, alpha = cap["q"], cap["acc"], cap["alpha"]
+    pw = getattr(model, "alpha_mode", 0) == 1
     boundary = 0
     logits = np.zeros((y.shape[0], n))
     for b in range(q.shape[0]):
@@ -70,7 +73,7 @@ def forward64(model, y, cap):
             sw = model.w_scale[l].astype(np.float64)
             bias = [bb.astype(np.float64) for bb in model.bias[l]]
             # QKV
-            boundary += check_quant(x, q[b, l, 0, :, :d], alpha[b, l, 0], model.alpha_floor, f"b{b} l{l} qkv")
+            boundary += check_quant(x, q[b, l, 0, :, :d], alpha[b, l, 0], model.alpha_floor, f"b{b} l{l} qkv", pw)
             f = alpha[b, l, 0][:, None] / 127.0
             A0 = acc[b, l, 0, :, :3 * d].astype(np.float64)
             Q = A0[:, :d] * (sw[0] * f) + bias[0]
@@ -87,14 +90,14 @@ def forward64(model, y, cap):
                 P /= P.sum(1, keepdims=True)
                 A[:, sl] = P @ V[:, sl]
             # O projection, residual, LayerNorm
-            boundary += check_quant(A, q[b, l, 1, :, :d], alpha[b, l, 1], model.alpha_floor, f"b{b} l{l} o")
+            boundary += check_quant(A, q[b, l, 1, :, :d], alpha[b, l, 1], model.alpha_floor, f"b{b} l{l} o", pw)
             o = acc[b, l, 1, :, :d].astype(np.float64) * (sw[3] * alpha[b, l, 1][:, None] / 127.0) + bias[3]
             x = ln64(x + o, model.ln_gamma[l, 0], model.ln_beta[l, 0], model.ln_eps)
             # FFN
-            boundary += check_quant(x, q[b, l, 2, :, :d], alpha[b, l, 2], model.alpha_floor, f"b{b} l{l} ffn1")
+            boundary += check_quant(x, q[b, l, 2, :, :d], alpha[b, l, 2], model.alpha_floor, f"b{b} l{l} ffn1", pw)
             u = acc[b, l, 2, :, :F].astype(np.float64) * (sw[4] * alpha[b, l, 2][:, None] / 127.0) + bias[4]
             u = np.maximum(u, 0.0)
-            boundary += check_quant(u, q[b, l, 3, :, :F], alpha[b, l, 3], model.alpha_floor, f"b{b} l{l} ffn2")
+            boundary += check_quant(u, q[b, l, 3, :, :F], alpha[b, l, 3], model.alpha_floor, f"b{b} l{l} ffn2", pw)
             o2 = acc[b, l, 3, :, :d].astype(np.float64) * (sw[5] * alpha[b, l, 3][:, None] / 127.0) + bias[5]
             x = ln64(x + o2, model.ln_gamma[l, 1], model.ln_beta[l, 1], model.ln_eps)
         z = x @ model.w_d1.astype(np.float64) + model.b_d1
@@ -108,12 +111,17 @@ def forward64(model, y, cap):
     ("bch31_16", 32, 2, dict(h_first=2)),
     ("bch31_16", 32, 2, dict(mask_mode=1)),
     ("polar64_32", 64, 1, dict(mask_mode=1, binary=True)),
+    ("bch31_16", 32, 2, dict(alpha_mode=1)),
+    ("polar64_32", 64, 1, dict(alpha_mode=1, h_first=6)),
 ])
 def test_oracle_matches_float64_forward(key, d, layers, var):
     code = I.make_code(key)
+    var = dict(var)
     mask_mode = var.pop("mask_mode", 0)
+    alpha_mode = var.pop("alpha_mode", 0)
     model = I.random_model(code, d, layers, seed=41, **var)
     model.mask_mode = mask_mode
+    model.alpha_mode = alpha_mode
     B = 3
     y = I.channel_batch(code, B, 2.0, seed=43).y
     r = O.decode(model, y, nthreads=2, cap_B=B)
