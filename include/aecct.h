@@ -139,6 +139,30 @@ int aecct_decode(aecct_handle *h, const float *y_dev, int64_t B, uint8_t *bits_d
 int aecct_decode_host(aecct_handle *h, const float *y_host, int64_t B, uint8_t *bits_host, uint8_t *syndrome_host,
                       float *logits_host, void *cuda_stream);
 
+/* The paper has no counterpart of this call (it is an implementation convenience).
+ * The same decode as aecct_decode_host, with HOST buffers, that allocates nothing: the device
+ * staging of y, bits, syndromes and logits and the kernel's status word live in one file-scope
+ * static device array of AECCT_NOALLOC_SCRATCH_BYTES (4 MiB).  It serves callers that must not
+ * allocate device memory while they decode: a process whose device memory is a fixed budget
+ * taken up front, or a latency-bound loop in which a cudaMalloc/cudaFree (which may synchronise
+ * the device) would stall other work.  aecct_decode_host instead grows its staging with
+ * cudaMalloc.
+ *   Limit: B words need B*(4n + n) bytes, + B*(n-k) with a syndrome, + B*4n with logits, each
+ *   part rounded up to 256 bytes, plus 256 bytes for the status word, at most 4 MiB (Polar(64,32)
+ *   with all outputs: 6,897 words).  A larger B returns AECCT_ERR_INVALID_ARG and
+ *   aecct_last_error says so.
+ *   Set-up: the first call on a device (that device current) resolves the array's address with
+ *   cudaGetSymbolAddress; make that first call before any stream capture.
+ *   Zeroing: the status word is cleared (cudaMemsetAsync on `cuda_stream`) before each launch;
+ *   the staging needs no clearing (y is copied in, every output element is written).
+ *   Concurrency: every call uses the same array, so calls that overlap in time (two host threads,
+ *   or two streams whose work interleaves on the device) race; serialise them.
+ * The call waits for its stream and returns the decode status (AECCT_ERR_TIMEOUT as
+ * aecct_synchronize reports it). */
+#define AECCT_NOALLOC_SCRATCH_BYTES (4u << 20)
+int aecct_decode_host_noalloc(aecct_handle *h, const float *y_host, int64_t B, uint8_t *bits_host,
+                              uint8_t *syndrome_host, float *logits_host, void *cuda_stream);
+
 /* Wait for the handle's last decode and report whether its kernel stopped on a
  * device-side timeout (AECCT_ERR_TIMEOUT) or a CUDA error occurred. */
 int aecct_synchronize(aecct_handle *h);

@@ -25,7 +25,7 @@ AECCT_ERR_NO_DEVICE = -6
 EXPORTED_SYMBOLS = (
     "aecct_create", "aecct_decode", "aecct_decode_host", "aecct_synchronize", "aecct_set_capture",
     "aecct_query", "aecct_destroy", "aecct_status_string", "aecct_last_error", "aecct_selftest_mma",
-    "aecct_selftest_timeout",
+    "aecct_selftest_timeout", "aecct_decode_host_noalloc",
 )
 
 
@@ -72,6 +72,7 @@ def load(build_if_missing: bool = True):
     L.aecct_create.argtypes = [ctypes.POINTER(ModelDesc), ctypes.POINTER(P)]
     L.aecct_decode.argtypes = [P, P, I64, P, P, P, P]
     L.aecct_decode_host.argtypes = [P, P, I64, P, P, P, P]
+    L.aecct_decode_host_noalloc.argtypes = [P, P, I64, P, P, P, P]
     L.aecct_synchronize.argtypes = [P]
     L.aecct_set_capture.argtypes = [P, I64, P, P, P, P]
     L.aecct_query.argtypes = [P] + [ctypes.POINTER(I32)] * 6
@@ -228,6 +229,19 @@ class Decoder:
                                        logits.ctypes.data if logits is not None else None, None)
         _check(st, "aecct_decode_host")
         return bits, syn, logits
+
+    def decode_host_noalloc(self, y: np.ndarray, want_syndrome: bool = True, want_logits: bool = True):
+        """aecct_decode_host_noalloc: host arrays, device staging from the library's static scratch
+        (no allocation).  Returns (status, bits, syndrome, logits); calls must not overlap."""
+        y = np.ascontiguousarray(y, dtype=np.float32)
+        B = y.shape[0]
+        bits = np.empty((B, self.n), np.uint8)
+        syn = np.empty((B, self.m), np.uint8) if want_syndrome else None
+        logits = np.empty((B, self.n), np.float32) if want_logits else None
+        st = self._L.aecct_decode_host_noalloc(self._h, y.ctypes.data, B, bits.ctypes.data,
+                                               syn.ctypes.data if syn is not None else None,
+                                               logits.ctypes.data if logits is not None else None, None)
+        return st, bits, syn, logits
 
     def synchronize(self) -> int:
         return self._L.aecct_synchronize(self._h)

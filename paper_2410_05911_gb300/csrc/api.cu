@@ -602,6 +602,102 @@ int aecct_decode_host(aecct_handle *h, const float *y_host, int64_t B, uint8_t *
   return collect_status(h, true);
 }
 
+// ---- host-buffer decode with no allocation (the paper has no counterpart).  Callers that must
+// not allocate device memory while they decode -- a fixed device-memory budget taken up front,
+// or a latency-bound loop where cudaMalloc/cudaFree may synchronise the device -- get their
+// staging and the kernel's status word from this static array instead of cudaMalloc.
+namespace {
+__device__ __align__(256) unsigned char g_noalloc_scratch[AECCT_NOALLOC_SCRATCH_BYTES];
+constexpr int kNoAllocMaxDevices = 64;
+void *g_noalloc_base[kNoAllocMaxDevices] = {};  // per device, resolved by its first call
+size_t round256(size_t v) { return (v + 255u) & ~static_cast<size_t>(255u); }
+}  // namespace
+
+int aecct_decode_host_noalloc(aecct_handle *h, const float *y_host, int64_t B, uint8_t *bits_host,
+                              uint8_t *syndrome_host, float *logits_host, void *cuda_stream) {
+  if (!h || B < 0) return AECCT_ERR_INVALID_ARG;
+  if (B == 0) return AECCT_OK;
+  if (!y_host || !bits_host) return AECCT_ERR_INVALID_ARG;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= kNoAllocMaxDevices) {
+    g_last_error = "aecct_decode_host_noalloc: device index beyond the per-device table";
+    return AECCT_ERR_UNSUPPORTED;
+  }
+  if (!g_noalloc_base[dev]) {  // set-up, once per device, with that device current
+    void *base = nullptr;
+    if ((e = cudaGetSymbolAddress(&base, g_noalloc_scratch)) != cudaSuccess)
+      return cuda_fail(e, "cudaGetSymbolAddress (aecct_decode_host_noalloc scratch)");
+    g_noalloc_base[dev] = base;
+  }
+  // layout: status word | y | bits | syndromes | logits, each part on a 256-byte boundary
+  const size_t n = static_cast<size_t>(h->n), m = static_cast<size_t>(h->m), b = static_cast<size_t>(B);
+  const size_t off_y = 256, off_bits = off_y + round256(sizeof(float) * b * n), off_syn = off_bits + round256(b * n);
+  const size_t off_log = off_syn + (syndrome_host ? round256(b * m) : 0);
+  const size_t end = off_log + (logits_host ? round256(sizeof(float) * b * n) : 0);
+  if (end > AECCT_NOALLOC_SCRATCH_BYTES) {
+    g_last_error = "aecct_decode_host_noalloc: B = " + std::to_string(B) + " needs " + std::to_string(end) +
+                   " bytes of staging, more than the " + std::to_string(AECCT_NOALLOC_SCRATCH_BYTES) +
+                   "-byte static scratch holds";
+    return AECCT_ERR_INVALID_ARG;
+  }
+  uint8_t *base = static_cast<uint8_t *>(g_noalloc_base[dev]);
+  int *err = reinterpret_cast<int *>(base);
+  float *y_dev = reinterpret_cast<float *>(base + off_y);
+  uint8_t *bits_dev = base + off_bits;
+  uint8_t *syn_dev = syndrome_host ? base + off_syn : nullptr;
+  float *logits_dev = logits_host ? reinterpret_cast<float *>(base + off_log) : nullptr;
+  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+  // the status word must start at zero (the kernel only ORs into it)
+  if ((e = cudaMemsetAsync(err, 0, sizeof(int), stream)) != cudaSuccess) return cuda_fail(e, "clear status");
+  if ((e = cudaMemcpyAsync(y_dev, y_host, sizeof(float) * b * n, cudaMemcpyHostToDevice, stream)) != cudaSuccess)
+    return cuda_fail(e, "copy y");
+  DecodeParams p = {};
+  p.n = h->n, p.k = h->k, p.T = h->T, p.m = h->m, p.n_layers = h->n_layers, p.h_first = h->h_first;
+  p.d_spe = h->d_spe, p.C = h->C, p.G = h->G;
+  p.B = B;
+  p.n_groups = (B + h->G - 1) / h->G;
+  p.n_clusters = static_cast<int>(p.n_groups < h->max_clusters ? p.n_groups : h->max_clusters);
+  p.y = y_dev, p.bits = bits_dev, p.syn = syn_dev, p.logits = logits_dev;
+  p.wstream = h->wstream, p.layer_bytes = h->layer_bytes;
+  p.lparams = h->lparams, p.emb = h->emb, p.spe = h->spe, p.w_d1 = h->w_d1, p.b_d1 = h->b_d1;
+  p.w_out = h->w_out, p.b_out = h->b_out, p.hbits = h->hbits, p.hwords = h->hwords;
+  p.perm = h->perm, p.pos = h->pos;
+  p.plan_task = h->plan_task;
+  p.plan_grp = reinterpret_cast<const uint4 *>(h->plan_grp);
+  p.plan_uinfo = h->plan_uinfo;
+  p.plan_ulist = reinterpret_cast<const uint4 *>(h->plan_ulist);
+  p.plan_mask = reinterpret_cast<const uint4 *>(h->plan_mask);
+  p.mask_info[0] = h->mask_info[0], p.mask_info[1] = h->mask_info[1];
+  p.mask_list[0] = reinterpret_cast<const uint4 *>(h->mask_list[0]);
+  p.mask_list[1] = reinterpret_cast<const uint4 *>(h->mask_list[1]);
+  p.ln_eps = h->ln_eps, p.alpha_floor = h->alpha_floor, p.att_scale = h->att_scale, p.alpha_mode = h->alpha_mode;
+  p.cap_B = h->cap_B, p.cap_q = h->cap_q, p.cap_acc = h->cap_acc, p.cap_alpha = h->cap_alpha, p.cap_syn = h->cap_syn;
+  p.err = err, p.wait_limit = h->wait_limit;
+  if (h->tasks) e = h->d == 32 ? launch_decode<32, true>(p, stream) : launch_decode<64, true>(p, stream);
+  else if (h->d == 32) e = launch_decode<32, false>(p, stream);
+  else if (h->d == 64) e = launch_decode<64, false>(p, stream);
+  else e = launch_decode<128, false>(p, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "decode launch");
+  if ((e = cudaMemcpyAsync(bits_host, bits_dev, b * n, cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
+    return cuda_fail(e, "copy bits");
+  if (syndrome_host && (e = cudaMemcpyAsync(syndrome_host, syn_dev, b * m, cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
+    return cuda_fail(e, "copy syndrome");
+  if (logits_host &&
+      (e = cudaMemcpyAsync(logits_host, logits_dev, sizeof(float) * b * n, cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
+    return cuda_fail(e, "copy logits");
+  int status_word = 0;
+  if ((e = cudaMemcpyAsync(&status_word, err, sizeof(int), cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
+    return cuda_fail(e, "copy status");
+  if ((e = cudaStreamSynchronize(stream)) != cudaSuccess) return cuda_fail(e, "stream sync");
+  if (status_word) {
+    g_last_error = "a device-side wait exceeded its limit";
+    return AECCT_ERR_TIMEOUT;
+  }
+  return AECCT_OK;
+}
+
 int aecct_set_capture(aecct_handle *h, int64_t cap_B, int8_t *q_dev, int32_t *acc_dev, float *alpha_dev,
                       uint8_t *syn_dev) {
   if (!h || cap_B < 0) return AECCT_ERR_INVALID_ARG;
