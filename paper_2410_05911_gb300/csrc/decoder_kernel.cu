@@ -249,17 +249,37 @@ __device__ __forceinline__ int idx_at(const uint4 &w, int k) {
 // (a lane past its own count computes on a valid dummy row and folds nothing in).  The scores of
 // the first kRowCache keys go to this thread's TMEM columns in pass 1 and come back in pass 2, in
 // place of a second load of K and a second dot product (the same fp32 values).
-template <int DH, int U, uint32_t STRIDE>
+// K (then V) row of one head, as float4s: in this CTA's shared memory (one-CTA cluster; plain
+// loads the compiler schedules) or in the CTA of the cluster that holds the row (32-bit
+// shared::cluster address)
+template <bool CLUSTER>
+struct KeyRow;
+template <>
+struct KeyRow<false> {
+  const float4 *p;
+  __device__ __forceinline__ float4 operator[](int i) const { return p[i]; }
+};
+template <>
+struct KeyRow<true> {
+  uint32_t a;
+  __device__ __forceinline__ float4 operator[](int i) const { return ld_cluster_f32x4(a + 16u * i); }
+};
+
+template <int DH, int U, uint32_t STRIDE, bool CLUSTER>
 __device__ __forceinline__ void hpsa_head(const float *q, uint32_t info, bool active, const uint4 *__restrict__ lists,
-                                          const uint64_t *kvgen, int rowbase, uint32_t hoff, float scale,
-                                          uint32_t tcache, float *A) {
+                                          const uint8_t *kvlocal, const uint32_t *kvbase, int rowbase,
+                                          uint32_t hoff, float scale, uint32_t tcache, float *A) {
   static_assert(8 % U == 0, "keys per index block");
   const uint4 *lst = lists + (info >> 11);
   const int cnt = active ? static_cast<int>(info & 2047u) : 0;
   const int nmax = __reduce_max_sync(0xffffffffu, cnt);
-  auto keyptr = [&](int off) -> const float4 * {
+  // K (then V) of key row `off` of this head, from the CTA that holds it
+  auto keyptr = [&](int off) -> KeyRow<CLUSTER> {
     const int ru = rowbase + off;
-    return reinterpret_cast<const float4 *>(kvgen[ru >> 7] + static_cast<uint32_t>(ru & 127) * STRIDE + hoff);
+    if constexpr (CLUSTER)
+      return KeyRow<true>{kvbase[ru >> 7] + static_cast<uint32_t>(ru & 127) * STRIDE + hoff};
+    else
+      return KeyRow<false>{reinterpret_cast<const float4 *>(kvlocal + static_cast<uint32_t>(ru) * STRIDE + hoff)};
   };
   // q . k in the canonical order: even-feature and odd-feature FMA chains (the two lanes of
   // paired FMAs over adjacent features), then their sum
@@ -282,7 +302,7 @@ __device__ __forceinline__ void hpsa_head(const float *q, uint32_t info, bool ac
       float4 kk[U][DH / 4];
 #pragma unroll
       for (int k = 0; k < U; ++k) {
-        const float4 *kp = keyptr(idx_at(w, k0 + k));
+        const KeyRow<CLUSTER> kp = keyptr(idx_at(w, k0 + k));
 #pragma unroll
         for (int i = 0; i < DH / 4; ++i) kk[k][i] = kp[i];
       }
@@ -323,7 +343,7 @@ __device__ __forceinline__ void hpsa_head(const float *q, uint32_t info, bool ac
       float4 vv[U][DH / 4];
 #pragma unroll
       for (int k = 0; k < U; ++k) {
-        const float4 *kp = keyptr(idx_at(w, k0 + k));
+        const KeyRow<CLUSTER> kp = keyptr(idx_at(w, k0 + k));
         if (!cached) {
           float4 kk[DH / 4];
 #pragma unroll
@@ -350,6 +370,11 @@ __device__ __forceinline__ void hpsa_head(const float *q, uint32_t info, bool ac
 __device__ __forceinline__ int byte_at(const uint4 &w, int k) {
   const uint32_t v = k < 8 ? (k < 4 ? w.x : w.y) : (k < 12 ? w.z : w.w);
   return static_cast<int>((v >> (8 * (k & 3))) & 0xFFu);
+}
+// a 16-entry index block of consecutive rows r0, r0 + 1, ..., r0 + 15 (rows < 240, no byte carry)
+__device__ __forceinline__ bool contiguous(const uint4 &w) {
+  const uint32_t pat = (w.x & 0xFFu) * 0x01010101u + 0x03020100u;
+  return w.x == pat && w.y == pat + 0x04040404u && w.z == pat + 0x08080808u && w.w == pat + 0x0C0C0C0Cu;
 }
 
 // One HPSA head for a query group (task mode).  Every lane walks the group's union key list in
@@ -391,15 +416,17 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
     const uint32_t seg = segment(jb);
     const int nk = min(16, cnt - jb);
     float sgs[16];
-    // the 16 keys of a full segment; DENSE: every lane holds all of them (no membership tests)
-    auto full_segment = [&](auto dense_tag) {
-      constexpr bool DENSE = decltype(dense_tag)::value;
+    // the 16 keys of a full segment; DENSE: every lane holds all of them (no membership tests);
+    // CONTIG: the keys are 16 consecutive rows (addresses at fixed offsets from the first)
+    const bool contig = nk == 16 && contiguous(w);
+    auto full_segment = [&](auto dense_tag, auto contig_tag) {
+      constexpr bool DENSE = decltype(dense_tag)::value, CONTIG = decltype(contig_tag)::value;
 #pragma unroll
       for (int k0 = 0; k0 < 16; k0 += U) {
         float4 kk[U][DH / 4];
 #pragma unroll
         for (int k = 0; k < U; ++k) {
-          const float4 *kp = kptr(byte_at(w, k0 + k));
+          const float4 *kp = CONTIG ? kptr(static_cast<int>(w.x & 0xFFu) + k0 + k) : kptr(byte_at(w, k0 + k));
 #pragma unroll
           for (int i = 0; i < DH / 4; ++i) kk[k][i] = kp[i];
         }
@@ -413,8 +440,14 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
       }
     };
     if (nk == 16) {
-      if (__all_sync(0xffffffffu, (seg & 0xFFFFu) == 0xFFFFu)) full_segment(std::true_type{});
-      else full_segment(std::false_type{});
+      const bool dense = __all_sync(0xffffffffu, (seg & 0xFFFFu) == 0xFFFFu);
+      if (contig) {
+        if (dense) full_segment(std::true_type{}, std::true_type{});
+        else full_segment(std::false_type{}, std::true_type{});
+      } else {
+        if (dense) full_segment(std::true_type{}, std::false_type{});
+        else full_segment(std::false_type{}, std::false_type{});
+      }
     } else {
 #pragma unroll
       for (int k = 0; k < 16; k += 2) {
@@ -463,16 +496,18 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
       float sgs[16];
       tmem_ld<16>(tcache + jb, sgs);
       tmem_wait_ld();
-      // DENSE: a full segment held by every lane (no membership or range tests)
-      auto cached_segment = [&](auto dense_tag) {
-        constexpr bool DENSE = decltype(dense_tag)::value;
+      // DENSE: a full segment held by every lane (no membership or range tests); CONTIG: a full
+      // segment of 16 consecutive rows
+      auto cached_segment = [&](auto dense_tag, auto contig_tag) {
+        constexpr bool DENSE = decltype(dense_tag)::value, CONTIG = decltype(contig_tag)::value;
 #pragma unroll
         for (int k0 = 0; k0 < 16; k0 += U) {
-          if (DENSE || k0 < nk) {
+          if (DENSE || CONTIG || k0 < nk) {
             float4 vv[U][DH / 4];
 #pragma unroll
             for (int k = 0; k < U; ++k) {
-              const float4 *kp = kptr(byte_at(w, DENSE ? k0 + k : min(k0 + k, nk - 1)));
+              const float4 *kp = CONTIG ? kptr(static_cast<int>(w.x & 0xFFu) + k0 + k)
+                                        : kptr(byte_at(w, DENSE ? k0 + k : min(k0 + k, nk - 1)));
 #pragma unroll
               for (int i = 0; i < DH / 4; ++i) vv[k][i] = kp[DH / 4 + i];
             }
@@ -482,14 +517,21 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
               pr[k / 2] = exp2_series2(make_float2(__fsub_rn(sgs[k0 + k], mx), __fsub_rn(sgs[k0 + k + 1], mx)));
 #pragma unroll
             for (int k = 0; k < U; k += 2) {
-              if (DENSE || (k0 + k < nk && ((seg >> (k0 + k)) & 1u))) fold(pr[k / 2].x, vv[k]);
-              if (DENSE || (k0 + k + 1 < nk && ((seg >> (k0 + k + 1)) & 1u))) fold(pr[k / 2].y, vv[k + 1]);
+              if (DENSE || ((CONTIG || k0 + k < nk) && ((seg >> (k0 + k)) & 1u))) fold(pr[k / 2].x, vv[k]);
+              if (DENSE || ((CONTIG || k0 + k + 1 < nk) && ((seg >> (k0 + k + 1)) & 1u)))
+                fold(pr[k / 2].y, vv[k + 1]);
             }
           }
         }
       };
-      if (nk == 16 && __all_sync(0xffffffffu, (seg & 0xFFFFu) == 0xFFFFu)) cached_segment(std::true_type{});
-      else cached_segment(std::false_type{});
+      const bool dense = nk == 16 && __all_sync(0xffffffffu, (seg & 0xFFFFu) == 0xFFFFu);
+      if (nk == 16 && contiguous(w)) {
+        if (dense) cached_segment(std::true_type{}, std::true_type{});
+        else cached_segment(std::false_type{}, std::true_type{});
+      } else {
+        if (dense) cached_segment(std::true_type{}, std::false_type{});
+        else cached_segment(std::false_type{}, std::false_type{});
+      }
     } else if (nk == 16) {
 #pragma unroll
       for (int k0 = 0; k0 < 16; k0 += U) {
@@ -877,7 +919,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   const uint32_t bar_fin = bar_zf + 8;
   uint32_t *s_tmem = reinterpret_cast<uint32_t *>(smem + L::kOffMisc);
   volatile int *s_abort = reinterpret_cast<volatile int *>(smem + L::kOffMisc + 4);
-  uint64_t *s_kvgen = reinterpret_cast<uint64_t *>(smem + L::kOffMisc + 8);  // [8] generic K/V bases per CTA
+  uint32_t *s_kvcl = reinterpret_cast<uint32_t *>(smem + L::kOffMisc + 8);   // [8] shared::cluster K/V bases per CTA
   uint64_t *s_zgen = reinterpret_cast<uint64_t *>(smem + L::kOffMisc + 72);   // [8] generic z bases per CTA
   uint32_t *s_issued = reinterpret_cast<uint32_t *>(smem + L::kOffMisc + 136);  // [6] weight copies / phases armed
 
@@ -897,11 +939,12 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
       for (int i = 0; i < 3; ++i) mbar_init(bar_fin + 8 + 8 * i, 1);
     *s_abort = 0;
     for (int i = 0; i < 6; ++i) s_issued[i] = 0;
-    // generic base of the K/V and z areas of every CTA of the cluster: this CTA's own area through
-    // its plain shared-memory window, the others through the distributed shared window
+    // base of the K/V area of every CTA of the cluster as a shared::cluster address, and generic
+    // base of its z area: this CTA's own through its plain shared-memory window, the others
+    // through the distributed shared window
     for (int c = 0; c < p.C; ++c) {
       const bool own = c == static_cast<int>(crank);
-      s_kvgen[c] = own ? reinterpret_cast<uint64_t>(smem + L::kOffU) : mapa_generic(smem + L::kOffU, c);
+      s_kvcl[c] = mapa_cluster(smem_u32(smem + L::kOffU), c);
       s_zgen[c] = own ? reinterpret_cast<uint64_t>(smem + L::kOffZ) : mapa_generic(smem + L::kOffZ, c);
     }
     fence_mbar_init_cluster();
@@ -1271,8 +1314,13 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
               constexpr int U = (DH >= 16) ? 2 : 4;
               // this thread's score cache: its own TMEM lane, kRowCache columns per column slice
               const uint32_t tcache = tl + L::kRowCacheCol + static_cast<uint32_t>(sl) * kRowCache;
-              hpsa_head<DH, U, L::kKvStride>(q, row_cw ? __ldg(p.mask_info[mk] + t) : 0u, row_cw, p.mask_list[mk],
-                                             s_kvgen, g * T, e * (8 * DH), p.att_scale, tcache, A[hh]);
+              const uint32_t info = row_cw ? __ldg(p.mask_info[mk] + t) : 0u;
+              if (p.C == 1)
+                hpsa_head<DH, U, L::kKvStride, false>(q, info, row_cw, p.mask_list[mk], smem + L::kOffU, s_kvcl,
+                                                      g * T, e * (8 * DH), p.att_scale, tcache, A[hh]);
+              else
+                hpsa_head<DH, U, L::kKvStride, true>(q, info, row_cw, p.mask_list[mk], smem + L::kOffU, s_kvcl,
+                                                     g * T, e * (8 * DH), p.att_scale, tcache, A[hh]);
             }
   #pragma unroll
             for (int i = 0; i < DH; ++i) amax = fmaxf(amax, fabsf(A[hh][i]));
