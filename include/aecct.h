@@ -57,7 +57,9 @@ typedef struct aecct_handle aecct_handle; /* opaque */
  *   d_spe         width of the SPE table (0 <= d_spe < d); the per-position embedding
  *                 fills the first d - d_spe features (Sec. 4.3; Sec. 5 ablation text).
  *   ffn_mult      feed-forward width multiplier; must be 4.
- *   activation    0 = ReLU (Sec. 4 item 4).  Other values are rejected.
+ *   activation    0 = ReLU (Sec. 4 item 4); 1 = GELU, x Phi(x) = 0.5 x (1 + erf(x / sqrt 2)),
+ *                 with erf by the rational approximation 7.1.26 of Abramowitz & Stegun
+ *                 (|error| <= 1.5e-7) in a fixed fp32 order.  Other values are rejected.
  *   cluster_ctas  0 = choose automatically; otherwise the number of CTAs (1..8) that
  *                 share one group of codewords (tuning knob).
  *   attention_mode 0 = choose automatically; 1 = per-row neighbour lists (any cluster size);

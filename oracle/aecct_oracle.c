@@ -16,7 +16,8 @@
  *   Sec. 3 (ECCT, mask_mode 1)      the code-aware mask of the ECCT baseline: every head on the
  *                                   union of the two rings
  *   Sec. 4.3 eq. SPE                SPE table concatenated to the embedding (table given as input)
- *   Sec. 4 item 4                   ReLU in the feed-forward block
+ *   Sec. 4 item 4                   ReLU in the feed-forward block (activation 0); GELU as the
+ *                                   option activation 1 (x Phi(x), erf by Abramowitz & Stegun 7.1.26)
  *   Sec. 5 (Training & Inference)   Post-LN Transformer blocks
  *
  * Arithmetic is IEEE fp32 (the paper's FP32 model) with one canonical order of
@@ -31,7 +32,8 @@
  *     reduction x = n + f, |f| <= 1/2, and the degree-7 Taylor series of e^(f ln 2));
  *   - sums over keys and over tokens run in ascending index order.
  *
- * Pins (tests/): exp2 against libm and its Taylor coefficients, pairwise sums, quantiser and
+ * Pins (tests/): exp2 against libm and its Taylor coefficients, GELU against the erf of libm and
+ * its odd-part identity, pairwise sums, quantiser and
  * LayerNorm closed forms, brute-force integer products, masks against Tanner-graph distances,
  * codeword-symmetry invariance, the all-zero-weight closed form, and an independent float64
  * forward pass teacher-forced on the recorded integer core.
@@ -108,6 +110,28 @@ float oracle_exp2_series(float x) {
   float p = g_exp2_coef[7];
   for (int k = 6; k >= 0; --k) p = fmaf(p, f, g_exp2_coef[k]);
   return ldexpf(p, (int)n);
+}
+
+/* GELU(x) = x Phi(x) = 0.5 x (1 + erf(x / sqrt 2)) (activation 1).  erf by the rational
+ * approximation 7.1.26 of Abramowitz & Stegun, Handbook of Mathematical Functions
+ * (|error| <= 1.5e-7 for x >= 0, odd symmetry below 0), in fixed fp32 steps:
+ *   z = x * fp32(1/sqrt 2), t = 1 / (1 + p |z|) (one fused multiply-add, then an IEEE divide),
+ *   poly = t * (a1 + t (a2 + t (a3 + t (a4 + t a5)))) (Horner with fused multiply-adds, then a multiply),
+ *   e = 2^((|z| * |z|) * fp32(-log2 e)) by exp2_series, erf|z| = 1 - poly * e,
+ *   GELU = (0.5 x) * (1 + sign(z) erf|z|). */
+float oracle_gelu(float x) {
+  float z = x * 0.70710678118654752f;
+  float az = fabsf(z);
+  float t = 1.0f / fmaf(0.3275911f, az, 1.0f);
+  float q = 1.061405429f;
+  q = fmaf(q, t, -1.453152027f);
+  q = fmaf(q, t, 1.421413741f);
+  q = fmaf(q, t, -0.284496736f);
+  q = fmaf(q, t, 0.254829592f);
+  q = q * t;
+  float e = oracle_exp2_series((az * az) * -1.44269504088896341f);
+  float er = 1.0f - q * e;
+  return (0.5f * x) * (1.0f + (z < 0.0f ? -er : er));
 }
 
 /* pairwise sum of v[0..len) (len a power of two): sum(lo half) + sum(hi half) */
@@ -398,7 +422,7 @@ static void decode_one(const oracle_model *m, const float *y, uint8_t *bits, uin
         if (cap->alpha) cap->alpha[off / (4 * d)] = al;
       }
     }
-    /* S7/S8: FFN with ReLU (Sec. 4 item 4), residual, LayerNorm */
+    /* S7/S8: FFN with ReLU (Sec. 4 item 4) or GELU, residual, LayerNorm */
     const float aw2 = per_word ? matrix_alpha(w->x, T, d, (size_t)d, m->alpha_floor) : 0.0f;
     for (int t = 0; t < T; ++t) {
       int8_t *qr = w->q + (size_t)t * F;
@@ -414,7 +438,10 @@ static void decode_one(const oracle_model *m, const float *y, uint8_t *bits, uin
         if (cap->acc) memcpy(cap->acc + off, ar, sizeof(int32_t) * F);
         if (cap->alpha) cap->alpha[off / (4 * d)] = al;
       }
-      for (int c = 0; c < F; ++c) ur[c] = ur[c] > 0.0f ? ur[c] : 0.0f;
+      if (m->activation == 0)
+        for (int c = 0; c < F; ++c) ur[c] = ur[c] > 0.0f ? ur[c] : 0.0f;
+      else
+        for (int c = 0; c < F; ++c) ur[c] = oracle_gelu(ur[c]);
     }
     const float aw3 = per_word ? matrix_alpha(w->u, T, F, (size_t)F, m->alpha_floor) : 0.0f;
     for (int t = 0; t < T; ++t) {
@@ -527,7 +554,7 @@ static int validate(const oracle_model *m) {
   if (m->h_first < 0 || m->h_first > m->heads || m->d_spe < 0 || m->d_spe >= m->d) return ORACLE_EINVAL;
   if (m->mask_mode < 0 || m->mask_mode > 1 || m->alpha_mode < 0 || m->alpha_mode > 1) return ORACLE_EINVAL;
   if (m->d_spe > 0 && !m->spe) return ORACLE_EINVAL;
-  if (m->ffn_mult != 4 || m->activation != 0) return ORACLE_EINVAL; /* FFN width 4d, ReLU */
+  if (m->ffn_mult != 4 || m->activation < 0 || m->activation > 1) return ORACLE_EINVAL; /* FFN width 4d, ReLU/GELU */
   return ORACLE_OK;
 }
 

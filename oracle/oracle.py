@@ -66,6 +66,8 @@ def lib():
             L.oracle_decode.restype = ctypes.c_int
             L.oracle_exp2_series.argtypes = [ctypes.c_float]
             L.oracle_exp2_series.restype = ctypes.c_float
+            L.oracle_gelu.argtypes = [ctypes.c_float]
+            L.oracle_gelu.restype = ctypes.c_float
             L.oracle_psum.argtypes = [P, ctypes.c_int]
             L.oracle_psum.restype = ctypes.c_float
             L.oracle_hard_decision.argtypes = [P, ctypes.c_int, P]
@@ -96,6 +98,12 @@ def exp2_series(x) -> np.ndarray:
     L = lib()
     xs = np.asarray(x, dtype=np.float32).ravel()
     return np.array([L.oracle_exp2_series(float(v)) for v in xs], dtype=np.float32)
+
+
+def gelu(x) -> np.ndarray:
+    L = lib()
+    xs = np.asarray(x, dtype=np.float32).ravel()
+    return np.array([L.oracle_gelu(float(v)) for v in xs], dtype=np.float32)
 
 
 def exp2_coefficients() -> np.ndarray:

@@ -1,5 +1,5 @@
 // aecct_internal.h -- parameters shared by the host side (api.cu) and the decoder kernel
-// (decoder_kernel.cu) of libaecct.  Not part of the public ABI.
+// (decoder_kernel.cuh) of libaecct.  Not part of the public ABI.
 #pragma once
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -192,10 +192,11 @@ struct SmemLayout {
   static constexpr uint32_t kRowCacheCol = (D == 128) ? 128u : 256u;
 };
 
-// decoder_kernel.cu
-template <int D, bool TASKS>
+// decoder_kernel.cuh (ACT: 0 = ReLU, instantiated in decoder_kernel.cu; 1 = GELU, in
+// decoder_kernel_gelu.cu)
+template <int D, bool TASKS, int ACT>
 cudaError_t launch_decode(const DecodeParams &p, cudaStream_t stream);
-template <int D, bool TASKS>
+template <int D, bool TASKS, int ACT>
 cudaError_t prepare_decode_kernel(int cluster_ctas, int *max_active_clusters);
 
 // api.cu diagnostics kernels live in selftest.cu

@@ -3,7 +3,7 @@
 // aecct_create validates the model description, builds the HPSA neighbour lists from H
 // (Sec. 4.2), unpacks the 2-bit ternary weights into bf16 tensor-core tiles, picks how many
 // CTAs share a group of codewords, and copies everything to the device once.  aecct_decode
-// launches the fused decoder kernel (decoder_kernel.cu) on the caller's stream.
+// launches the fused decoder kernel (decoder_kernel.cuh) on the caller's stream.
 #include <cuda_runtime.h>
 
 #include <cmath>
@@ -34,6 +34,7 @@ struct aecct_handle {
   int C = 1, G = 1, max_clusters = 0;
   bool tasks = false;  // warp-task attention (one CTA per group, d <= 64)
   int alpha_mode = 0;  // 1 = one alpha per quantised matrix of a word
+  int activation = 0;  // 0 = ReLU, 1 = GELU
   float ln_eps = 0, alpha_floor = 0, att_scale = 0, b_d1 = 0;
   long long wait_limit = 0;
   int device = 0;
@@ -141,7 +142,7 @@ int validate(const aecct_model_desc *d) {
   // shape limits of this build
   if (d->heads != kHeads) return AECCT_ERR_UNSUPPORTED;
   if (d->d != 32 && d->d != 64 && d->d != 128) return AECCT_ERR_UNSUPPORTED;
-  if (d->ffn_mult != 4 || d->activation != 0) return AECCT_ERR_UNSUPPORTED;
+  if (d->ffn_mult != 4) return AECCT_ERR_UNSUPPORTED;
   const int T = 2 * n - d->k;
   if (T > kMaxCluster * kRows || T > 65535) return AECCT_ERR_UNSUPPORTED;
   // packed weights: no code 10
@@ -171,6 +172,23 @@ int schedule_chunks_t(ChunkDesc *out) {
 }
 int schedule_chunks(int D, ChunkDesc *out) {
   return D == 32 ? schedule_chunks_t<32>(out) : D == 64 ? schedule_chunks_t<64>(out) : schedule_chunks_t<128>(out);
+}
+
+// the compiled kernel for (d, attention mode, activation): task mode exists for d = 32 and 64
+template <int ACT>
+cudaError_t prepare_any(int D, bool tasks, int C, int *max_clusters) {
+  if (tasks) return D == 32 ? prepare_decode_kernel<32, true, ACT>(C, max_clusters)
+                            : prepare_decode_kernel<64, true, ACT>(C, max_clusters);
+  if (D == 32) return prepare_decode_kernel<32, false, ACT>(C, max_clusters);
+  if (D == 64) return prepare_decode_kernel<64, false, ACT>(C, max_clusters);
+  return prepare_decode_kernel<128, false, ACT>(C, max_clusters);
+}
+template <int ACT>
+cudaError_t launch_any(int D, bool tasks, const DecodeParams &p, cudaStream_t stream) {
+  if (tasks) return D == 32 ? launch_decode<32, true, ACT>(p, stream) : launch_decode<64, true, ACT>(p, stream);
+  if (D == 32) return launch_decode<32, false, ACT>(p, stream);
+  if (D == 64) return launch_decode<64, false, ACT>(p, stream);
+  return launch_decode<128, false, ACT>(p, stream);
 }
 
 }  // namespace
@@ -241,11 +259,8 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
     return AECCT_ERR_NO_DEVICE;
   }
   int max_clusters = 0;
-  if (tasks) e = D == 32 ? prepare_decode_kernel<32, true>(best_C, &max_clusters)
-                         : prepare_decode_kernel<64, true>(best_C, &max_clusters);
-  else if (D == 32) e = prepare_decode_kernel<32, false>(best_C, &max_clusters);
-  else if (D == 64) e = prepare_decode_kernel<64, false>(best_C, &max_clusters);
-  else e = prepare_decode_kernel<128, false>(best_C, &max_clusters);
+  e = d.activation == 0 ? prepare_any<0>(D, tasks, best_C, &max_clusters)
+                        : prepare_any<1>(D, tasks, best_C, &max_clusters);
   if (e != cudaSuccess) return cuda_fail(e, "kernel occupancy");
   if (max_clusters < 1) {
     g_last_error = "no cluster of this size fits on the device";
@@ -257,6 +272,7 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
   h->d_spe = d.d_spe, h->C = best_C, h->G = best_G, h->max_clusters = max_clusters, h->tasks = tasks;
   h->ln_eps = d.ln_eps, h->alpha_floor = d.alpha_floor, h->b_d1 = d.b_d1, h->device = dev;
   h->alpha_mode = d.alpha_mode;
+  h->activation = d.activation;
   h->att_scale = static_cast<float>(1.4426950408889634074 / std::sqrt(static_cast<double>(D / kHeads)));
   h->wait_limit = d.wait_limit_cycles ? d.wait_limit_cycles : (1LL << 32);
 
@@ -551,10 +567,7 @@ int aecct_decode(aecct_handle *h, const float *y_dev, int64_t B, uint8_t *bits_d
   p.cap_B = h->cap_B, p.cap_q = h->cap_q, p.cap_acc = h->cap_acc, p.cap_alpha = h->cap_alpha, p.cap_syn = h->cap_syn;
   p.err = h->d_err, p.wait_limit = h->wait_limit;
   cudaError_t e;
-  if (h->tasks) e = h->d == 32 ? launch_decode<32, true>(p, stream) : launch_decode<64, true>(p, stream);
-  else if (h->d == 32) e = launch_decode<32, false>(p, stream);
-  else if (h->d == 64) e = launch_decode<64, false>(p, stream);
-  else e = launch_decode<128, false>(p, stream);
+  e = h->activation == 0 ? launch_any<0>(h->d, h->tasks, p, stream) : launch_any<1>(h->d, h->tasks, p, stream);
   if (e != cudaSuccess) return cuda_fail(e, "decode launch");
   if ((e = cudaMemcpyAsync(h->h_err, h->d_err, sizeof(int), cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
     return cuda_fail(e, "status copy");
@@ -675,10 +688,7 @@ int aecct_decode_host_noalloc(aecct_handle *h, const float *y_host, int64_t B, u
   p.ln_eps = h->ln_eps, p.alpha_floor = h->alpha_floor, p.att_scale = h->att_scale, p.alpha_mode = h->alpha_mode;
   p.cap_B = h->cap_B, p.cap_q = h->cap_q, p.cap_acc = h->cap_acc, p.cap_alpha = h->cap_alpha, p.cap_syn = h->cap_syn;
   p.err = err, p.wait_limit = h->wait_limit;
-  if (h->tasks) e = h->d == 32 ? launch_decode<32, true>(p, stream) : launch_decode<64, true>(p, stream);
-  else if (h->d == 32) e = launch_decode<32, false>(p, stream);
-  else if (h->d == 64) e = launch_decode<64, false>(p, stream);
-  else e = launch_decode<128, false>(p, stream);
+  e = h->activation == 0 ? launch_any<0>(h->d, h->tasks, p, stream) : launch_any<1>(h->d, h->tasks, p, stream);
   if (e != cudaSuccess) return cuda_fail(e, "decode launch");
   if ((e = cudaMemcpyAsync(bits_host, bits_dev, b * n, cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
     return cuda_fail(e, "copy bits");

@@ -68,7 +68,6 @@ def _status(model, **kw):
     (lambda m: setattr(m, "mask_mode", 2), A.AECCT_ERR_INVALID_ARG),
     (lambda m: setattr(m, "mask_mode", -1), A.AECCT_ERR_INVALID_ARG),
     (lambda m: setattr(m, "alpha_mode", 2), A.AECCT_ERR_INVALID_ARG),
-    (lambda m: setattr(m, "activation", 1), A.AECCT_ERR_UNSUPPORTED),
     (lambda m: setattr(m, "ffn_mult", 2), A.AECCT_ERR_UNSUPPORTED),
 ])
 def test_create_rejects_invalid_descriptions(mutate, expected):

@@ -8,7 +8,8 @@ block, then logits, bits and syndromes):
 * the ECCT code-aware mask (Sec. 3; the CASA baseline the paper compares HPSA with): every head
   attends over the union of the two rings (mask_mode = 1);
 * one absmax alpha per quantised matrix of a word instead of per token (alpha_mode = 1, the
-  other reading of Sec. 4.1's scalar alpha of x).
+  other reading of Sec. 4.1's scalar alpha of x);
+* GELU in place of ReLU in the feed-forward block (activation = 1), whose output can be negative.
 """
 import numpy as np
 import pytest
@@ -34,6 +35,10 @@ CASES = [
     ("bch31_16", 32, 2, dict(alpha_mode=1), (1, 2)),
     ("polar64_32", 64, 2, dict(alpha_mode=1), (1, 2)),
     ("bch63_36", 128, 1, dict(alpha_mode=1, mask_mode=1), (1,)),
+    ("bch31_16", 32, 2, dict(activation=1), (1, 2)),
+    ("polar64_32", 64, 2, dict(activation=1), (1, 2)),
+    ("ldpc128_64", 128, 1, dict(activation=1), (1,)),
+    ("bch63_36", 128, 2, dict(activation=1, alpha_mode=1), (1,)),
 ]
 
 

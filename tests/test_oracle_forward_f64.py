@@ -5,11 +5,13 @@ The integer core is teacher-forced: the oracle's recorded int32 accumulators of 
 pass, which recomputes everything in between on its own -- embedding with the syndrome tokens
 (Sec. 3), dequantisation (eq. AAPLinear), masked multi-head softmax attention with masks built
 here from H (Sec. 4.2, or the ECCT code-aware mask of Sec. 3 when mask_mode = 1), residual +
-LayerNorm (Post-LN, Sec. 5), ReLU FFN, the output head -- and checks at every quantised GEMM
+LayerNorm (Post-LN, Sec. 5), ReLU (or GELU) FFN, the output head -- and checks at every quantised GEMM
 input that the oracle's alpha is max|x| and its int8 codes are rint(x * 127 / alpha) of this
 float64 x, and finally that the logits agree.  A dropped term, a wrong index, a transposed
 operand or a mask mistake in the oracle changes codes or logits far beyond fp32 rounding.
 """
+import math
+
 import numpy as np
 import pytest
 
@@ -96,7 +98,10 @@ def forward64(model, y, cap):
             # FFN
             boundary += check_quant(x, q[b, l, 2, :, :d], alpha[b, l, 2], model.alpha_floor, f"b{b} l{l} ffn1", pw)
             u = acc[b, l, 2, :, :F].astype(np.float64) * (sw[4] * alpha[b, l, 2][:, None] / 127.0) + bias[4]
-            u = np.maximum(u, 0.0)
+            if model.activation == 0:
+                u = np.maximum(u, 0.0)
+            else:  # GELU(u) = u Phi(u) with the exact erf
+                u = 0.5 * u * (1.0 + np.vectorize(math.erf)(u / math.sqrt(2.0)))
             boundary += check_quant(u, q[b, l, 3, :, :F], alpha[b, l, 3], model.alpha_floor, f"b{b} l{l} ffn2", pw)
             o2 = acc[b, l, 3, :, :d].astype(np.float64) * (sw[5] * alpha[b, l, 3][:, None] / 127.0) + bias[5]
             x = ln64(x + o2, model.ln_gamma[l, 1], model.ln_beta[l, 1], model.ln_eps)
@@ -113,6 +118,8 @@ def forward64(model, y, cap):
     ("polar64_32", 64, 1, dict(mask_mode=1, binary=True)),
     ("bch31_16", 32, 2, dict(alpha_mode=1)),
     ("polar64_32", 64, 1, dict(alpha_mode=1, h_first=6)),
+    ("bch31_16", 32, 2, dict(activation=1)),
+    ("polar64_32", 64, 1, dict(activation=1, mask_mode=1)),
 ])
 def test_oracle_matches_float64_forward(key, d, layers, var):
     code = I.make_code(key)

@@ -37,6 +37,26 @@ def test_exp2_series_accuracy_vs_libm():
     assert (np.abs(got - ref) <= 2.0 * ulp).all()
 
 
+def test_gelu_against_libm_erf():
+    # GELU(x) = 0.5 x (1 + erf(x / sqrt 2)); the oracle's erf (Abramowitz & Stegun 7.1.26) is within
+    # 1.5e-7 of erf, so GELU is within 0.5 |x| 1.5e-7 plus a few fp32 roundings of |x| and |GELU|
+    rng = np.random.default_rng(3)
+    xs = np.concatenate([np.linspace(-12, 12, 4001), rng.normal(0, 3, 4000)]).astype(np.float32)
+    got = O.gelu(xs).astype(np.float64)
+    x = xs.astype(np.float64)
+    ref = np.array([0.5 * v * (1.0 + math.erf(v / math.sqrt(2.0))) for v in x])
+    assert (np.abs(got - ref) <= 2.5e-7 * (np.abs(x) + np.abs(ref)) + 1e-45).all()
+
+
+def test_gelu_special_values_and_odd_part():
+    g = O.gelu([0.0, 30.0, -30.0, 100.0])
+    assert g[0] == 0.0 and g[1] == 30.0 and g[2] == 0.0 and g[3] == 100.0
+    # x Phi(x) - (-x) Phi(-x) = x Phi(x) + x (1 - Phi(x)) = x
+    x = np.linspace(0.0, 10.0, 2001).astype(np.float32)
+    d = O.gelu(x).astype(np.float64) - O.gelu(-x).astype(np.float64)
+    assert (np.abs(d - x) <= 2e-7 * x + 1e-45).all()
+
+
 def test_exp2_series_coefficients_are_taylor_terms():
     c = O.exp2_coefficients()
     for kk in range(8):
