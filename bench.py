@@ -1,6 +1,7 @@
 """Throughput benchmark of the AECCT batched decoder on GB300.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl {cuda,reference}] [--workload KEY]
+                  [--variant {aecct,ecct,fp-hpsa}]
 
 A step decodes one batch of the workload (default: Polar(64,32), d = 64, N = 6, 8 heads,
 B = 65,536 received words, BPSK/AWGN at Eb/N0 cycling over 4, 5, 6 dB) through the C ABI
@@ -8,6 +9,10 @@ B = 65,536 received words, BPSK/AWGN at Eb/N0 cycling over 4, 5, 6 dB) through t
 steps by writing a 256 MB buffer outside the timed events.  One JSON line is printed by
 rank 0.  Under torchrun each rank decodes its own batch (weak scaling, no collective on the
 data path); the time is the maximum over ranks.
+
+--variant selects the model: aecct (default, the paper's method), ecct (the ECCT baseline of
+Sec. 3: full-precision linears on bf16 tensor cores, the code-aware mask on every head, GELU) or
+fp-hpsa (full-precision linears with HPSA and ReLU).
 
 --impl reference times the CPU oracle (the plain C forward pass) on a bounded sample of
 the same workload on the host cores, and reports the same metric.
@@ -168,9 +173,25 @@ def cpu_oracle_rate(model, y, budget_s: float = 12.0, chunk: int = 64, max_words
     return done / dt, done, dt, cores
 
 
+VARIANTS = {
+    # name: (model overrides, mask_mode, description)
+    "aecct": (dict(), 0, "AECCT: AAP ternary linears, HPSA, ReLU"),
+    "ecct": (dict(full_precision=True, activation=1), 1,
+             "ECCT baseline: full-precision (bf16) linears, code-aware mask on every head, GELU"),
+    "fp-hpsa": (dict(full_precision=True), 0, "full-precision (bf16) linears with HPSA and ReLU"),
+}
+
+
+def variant_model(key: str, variant: str):
+    overrides, mask_mode, _ = VARIANTS[variant]
+    model = I.workload_model(key, **overrides)
+    model.mask_mode = mask_mode
+    return model
+
+
 def run_reference(args, rank, world):
     w = I.workload(args.workload)
-    model = I.workload_model(args.workload)
+    model = variant_model(args.workload, args.variant)
     if rank != 0:
         return
     chunk = max(16, w.code.T and 64)
@@ -196,8 +217,8 @@ def run_reference(args, rank, world):
     value = words / secs
     line = dict(metric=METRIC, value=value, unit=UNIT, n_gpus=world, steps=args.steps, warmup=args.warmup,
                 ms_per_step=1e3 * secs / args.steps, higher_is_better=True, scaling="weak", vs_baseline=None,
-                dtype="i8/f32", data="synthetic", impl="reference",
-                config=dict(workload=workload_label(w), batch=w.batch),
+                dtype="i8/f32" if args.variant == "aecct" else "bf16/f32", data="synthetic", impl="reference",
+                config=dict(workload=workload_label(w), batch=w.batch, variant=args.variant),
                 cpu_baseline=dict(value=value, unit=UNIT, cores=cores, kind="oracle",
                                   sample=f"{words} words over {args.steps} steps, each a time-bounded prefix of a "
                                          f"1024-word batch of the workload"),
@@ -218,7 +239,7 @@ def run_cuda(args, rank, world, local_rank):
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
     w = I.workload(args.workload)
-    model = I.workload_model(args.workload)
+    model = variant_model(args.workload, args.variant)
     B = args.batch or w.batch
     dec = aecct.Decoder(model)
     q = dec.query()
@@ -281,9 +302,10 @@ def run_cuda(args, rank, world, local_rank):
     achieved_tops = wk["int_ops"] * B / kernel_s / 1e12
     roof = dict(bound="tensor", achieved=achieved_tops, peak=pk["bf16_tflops"], unit="TFLOP/s",
                 frac=achieved_tops / pk["bf16_tflops"],
-                traffic=args.traffic if args.traffic is not None else measured_traffic(args.workload, B),
-                kernel=f"aecct_decoder_kernel<{w.d}>", work="2*12*T*d^2*N int ops per word (bf16 tensor cores, "
-                "exact integers); peak = measured bf16 dense burst")
+                traffic=args.traffic if args.traffic is not None else
+                (measured_traffic(args.workload, B) if args.variant == "aecct" else None),
+                kernel=f"aecct_decoder_kernel<{w.d}>", work="2*12*T*d^2*N ops per word on the bf16 tensor cores "
+                "(AAP: exact integers; full-precision linears: bf16 products); peak = measured bf16 dense burst")
     cpu = None
     if not args.no_cpu_baseline:
         rate, words, secs, cores = cpu_oracle_rate(model, ys_host[0], budget_s=args.cpu_budget)
@@ -291,9 +313,10 @@ def run_cuda(args, rank, world, local_rank):
                    sample=f"first {words} words of the {w.ebn0_db[0]} dB batch ({secs:.1f} s)")
     line = dict(
         metric=METRIC, value=value, unit=UNIT, n_gpus=world, steps=args.steps, warmup=args.warmup,
-        ms_per_step=1e3 * kernel_s, higher_is_better=True, scaling="weak", vs_baseline=None, dtype="i8/f32",
-        data="synthetic",
-        config=dict(workload=workload_label(w), batch=B, tokens=w.code.T, cluster_ctas=q["cluster_ctas"],
+        ms_per_step=1e3 * kernel_s, higher_is_better=True, scaling="weak", vs_baseline=None,
+        dtype="i8/f32" if args.variant == "aecct" else "bf16/f32", data="synthetic",
+        config=dict(workload=workload_label(w), variant=args.variant, batch=B, tokens=w.code.T,
+                    cluster_ctas=q["cluster_ctas"],
                     words_per_group=q["words_per_group"], l2="flushed between steps (256 MB write)",
                     info_gbit_s=value * w.code.k / 1e9, hbm_io_gbs=value * wk["io_bytes"] / 1e9),
         e2e=e2e, roofline=roof, cpu_baseline=cpu, gpu_launches=args.steps, clocks=clk.summary())
@@ -308,6 +331,8 @@ def main():
     ap.add_argument("--impl", default="cuda", choices=["cuda", "reference"])
     ap.add_argument("--workload", default="polar64_32", choices=sorted(I.WORKLOADS))
     ap.add_argument("--batch", type=int, default=0, help="override the batch size (0 = the workload's)")
+    ap.add_argument("--variant", default="aecct", choices=sorted(VARIANTS),
+                    help="; ".join(f"{k}: {v[2]}" for k, v in VARIANTS.items()))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--traffic", type=float, default=None, help="ncu DRAM bytes per launch, if measured")

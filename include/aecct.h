@@ -72,6 +72,13 @@ typedef struct aecct_handle aecct_handle; /* opaque */
  *                 1 = one alpha per quantised matrix of a codeword (the max over its T rows).
  *                 1 needs one CTA per codeword (T <= 128 and cluster_ctas 0 or 1), else
  *                 AECCT_ERR_UNSUPPORTED.
+ *   linear_mode   0 = AAP linear layers (Sec. 4.1): ternary w_packed, scales w_scale, int8
+ *                 activations (eq. Quant, eq. AAPLinear).
+ *                 1 = full-precision linear layers, as in the ECCT baseline (Sec. 3): weights
+ *                 w_full (fp32, rounded once to bf16, round to nearest even), each GEMM input
+ *                 row rounded to bf16 (round to nearest even), products accumulated in fp32 on
+ *                 the tensor cores (order of the accumulation not specified), out = acc + b.
+ *                 w_packed and w_scale are not read (may be NULL); alpha_mode must be 0.
  *   H             [(n-k)][n] uint8 row-major, entries 0/1, no all-zero row or column.
  *   emb           [T][d-d_spe] fp32: token t's embedding row, scaled by h_t (Sec. 3, ECCT).
  *   spe           [T][d_spe] fp32: spectral positional encoding table (Sec. 4.3);
@@ -93,10 +100,14 @@ typedef struct aecct_handle aecct_handle; /* opaque */
  *                 zero codes instead of dividing by zero).
  *   wait_limit_cycles  0 = default (about 2^32 SM cycles); bound on every device-side
  *                 wait, after which the kernel stops and decode reports AECCT_ERR_TIMEOUT.
+ *   w_full        linear_mode 1 only: fp32 weights of all blocks, per block W_q [d][d],
+ *                 W_k [d][d], W_v [d][d], W_o [d][d], W_1 [F][d], W_2 [d][F] (row = output
+ *                 unit), n_layers * 12 * d * d floats.  NULL when linear_mode is 0.
  */
 typedef struct {
   int32_t n, k, d, n_layers, heads, h_first, d_spe, ffn_mult, activation, cluster_ctas, attention_mode, mask_mode;
   int32_t alpha_mode;
+  int32_t linear_mode;
   const uint8_t *H;
   const float *emb;
   const float *spe;
@@ -112,6 +123,7 @@ typedef struct {
   float ln_eps;
   float alpha_floor;
   int64_t wait_limit_cycles;
+  const float *w_full;
 } aecct_model_desc;
 
 /* Validate the description, build the HPSA masks from H (Sec. 4.2: first ring = Tanner

@@ -11,6 +11,7 @@
  *   Sec. 4.1 eq. Ternary            AAP weight ternarisation (used by tests, not by decode)
  *   Sec. 4.1 eq. Quant              per-token absmax int8 activation quantisation
  *   Sec. 4.1 eq. AAPLinear          int accumulate, dequantise by gamma*delta*alpha/Q_b, add bias
+ *   Sec. 3 (ECCT, linear_mode 1)    full-precision linear layers, on bf16 inputs and weights
  *   Sec. 4.2 (HPSA)                 first-ring heads on the c<->v mask, second-ring heads on the
  *                                   v<->v / c<->c mask
  *   Sec. 3 (ECCT, mask_mode 1)      the code-aware mask of the ECCT baseline: every head on the
@@ -55,6 +56,7 @@ typedef struct {
   int32_t n, k, d, n_layers, heads, h_first, d_spe, ffn_mult, activation;
   int32_t mask_mode;       /* 0 = HPSA (Sec. 4.2); 1 = ECCT code-aware mask M1 | M2 for all heads (Sec. 3) */
   int32_t alpha_mode;      /* 0 = one alpha per token (C-1); 1 = one alpha per quantised matrix of a word */
+  int32_t linear_mode;     /* 0 = AAP linears (Sec. 4.1); 1 = full-precision linears (ECCT, Sec. 3) on bf16 */
   const uint8_t *H;        /* [(n-k)][n] 0/1 */
   const float *emb;        /* [T][d-d_spe] */
   const float *spe;        /* [T][d_spe] */
@@ -69,12 +71,15 @@ typedef struct {
   const float *b_out;      /* [n] */
   float ln_eps;
   float alpha_floor;
+  const float *w_full;     /* linear_mode 1: fp32 weights, same order and shapes as w */
 } oracle_model;
 
 /* Optional record of the integer core for the first cap_B codewords.
  * gemm index g: 0 = QKV (K=d, N=3d), 1 = O (K=d, N=d), 2 = FFN1 (K=d, N=4d), 3 = FFN2 (K=4d, N=d).
  * q     int8  [cap_B][n_layers][4][T][4d]  quantised GEMM input (first K entries of a row used)
- * acc   int32 [cap_B][n_layers][4][T][4d]  integer accumulators (first N entries used)
+ * acc   int32 [cap_B][n_layers][4][T][4d]  integer accumulators (first N entries used); with
+ *                                          linear_mode 1 the bit patterns of the fp32 sums, and
+ *                                          q and alpha are left untouched
  * alpha fp32  [cap_B][n_layers][4][T]      max(absmax, floor) of the GEMM input row
  * syn   uint8 [cap_B][n-k]                 syndrome of the channel output */
 typedef struct {
@@ -238,6 +243,38 @@ void oracle_aap_linear_row(const int8_t *q, float alpha, int K, const int8_t *W,
   }
 }
 
+/* bf16 value of a finite fp32 x, rounded to nearest even: keep the sign, the exponent and the top
+ * 7 fraction bits; the 16 dropped bits round up when above half an ulp, or at exactly half when
+ * the kept part is odd. */
+float oracle_bf16_round(float x) {
+  uint32_t u;
+  memcpy(&u, &x, 4);
+  uint32_t low = u & 0xFFFFu, keep = u & 0xFFFF0000u;
+  if (low > 0x8000u || (low == 0x8000u && (keep & 0x10000u))) keep += 0x10000u;
+  float r;
+  memcpy(&r, &keep, 4);
+  return r;
+}
+
+/* The full-precision linear layer of the ECCT baseline (Sec. 3) in the number format of the
+ * tensor cores: out_o = fp32(sum_i bf16(x_i) bf16(W_oi)) + b_o.  Each product of two bf16 values
+ * is exact in double and the sum runs in double (ascending i); it stays exact while the products
+ * span fewer than 53 bits (always for the activations and weights here), so the sum is rounded
+ * to fp32 once.  sum_out receives that fp32 sum (before the bias). */
+void oracle_full_linear_row(const float *x, int K, const float *W, int N, const float *b, float *sum_out,
+                            float *out) {
+  double xb[4096];
+  for (int i = 0; i < K; ++i) xb[i] = (double)oracle_bf16_round(x[i]);
+  for (int o = 0; o < N; ++o) {
+    const float *wr = W + (size_t)o * K;
+    double acc = 0.0;
+    for (int i = 0; i < K; ++i) acc += xb[i] * (double)oracle_bf16_round(wr[i]);
+    float s = (float)acc;
+    if (sum_out) sum_out[o] = s;
+    out[o] = s + b[o];
+  }
+}
+
 /* Sec. 4.1 eq. Ternary: gamma = Percentile(|W|, 0.5) (linear interpolation between order
  * statistics), t = RoundClip(W / (gamma*delta + eps), -1, 1); returns scale gamma*delta. */
 static int cmp_float(const void *a, const void *b) {
@@ -372,34 +409,50 @@ static void decode_one(const oracle_model *m, const float *y, uint8_t *bits, uin
   }
   size_t wlayer = (size_t)4 * d * d + (size_t)2 * F * d;
   size_t blayer = (size_t)5 * d + F;
+  const int full = m->linear_mode == 1;
   for (int l = 0; l < m->n_layers; ++l) {
-    const int8_t *Wq = m->w + wlayer * l;
-    const int8_t *Wk = Wq + (size_t)d * d;
-    const int8_t *Wv = Wk + (size_t)d * d;
-    const int8_t *Wo = Wv + (size_t)d * d;
-    const int8_t *W1 = Wo + (size_t)d * d;
-    const int8_t *W2 = W1 + (size_t)F * d;
-    const float *sw = m->w_scale + (size_t)6 * l;
+    const int8_t *Wq = full ? NULL : m->w + wlayer * l;
+    const int8_t *Wk = full ? NULL : Wq + (size_t)d * d;
+    const int8_t *Wv = full ? NULL : Wk + (size_t)d * d;
+    const int8_t *Wo = full ? NULL : Wv + (size_t)d * d;
+    const int8_t *W1 = full ? NULL : Wo + (size_t)d * d;
+    const int8_t *W2 = full ? NULL : W1 + (size_t)F * d;
+    /* full-precision weights, same order */
+    const float *Fq = full ? m->w_full + wlayer * l : NULL;
+    const float *Fk = full ? Fq + (size_t)d * d : NULL;
+    const float *Fv = full ? Fk + (size_t)d * d : NULL;
+    const float *Fo = full ? Fv + (size_t)d * d : NULL;
+    const float *F1 = full ? Fo + (size_t)d * d : NULL;
+    const float *F2 = full ? F1 + (size_t)F * d : NULL;
+    const float *sw = full ? NULL : m->w_scale + (size_t)6 * l;
     const float *bq = m->bias + blayer * l, *bk = bq + d, *bv = bk + d, *bo = bv + d, *b1 = bo + d, *b2 = b1 + F;
     const float *g1 = m->ln_gamma + (size_t)2 * d * l, *g2 = g1 + d;
     const float *be1 = m->ln_beta + (size_t)2 * d * l, *be2 = be1 + d;
     const int per_word = m->alpha_mode == 1;
-    /* S3/S4: Quant(x) and the Q, K, V AAP-linear layers (Sec. 4.1) */
+    /* S3/S4: Quant(x) and the Q, K, V AAP-linear layers (Sec. 4.1), or the full-precision ones */
     const float aw0 = per_word ? matrix_alpha(w->x, T, d, (size_t)d, m->alpha_floor) : 0.0f;
     for (int t = 0; t < T; ++t) {
       int8_t *qr = w->q + (size_t)t * F;
-      float al;
-      if (per_word) quant_with_alpha(w->x + (size_t)t * d, d, al = aw0, qr);
-      else oracle_quant_row(w->x + (size_t)t * d, d, m->alpha_floor, qr, &al);
+      float al = 0.0f;
       int32_t *ar = w->acc + (size_t)t * 3 * d;
-      oracle_aap_linear_row(qr, al, d, Wq, d, sw[0], bq, ar, w->qf + (size_t)t * d);
-      oracle_aap_linear_row(qr, al, d, Wk, d, sw[1], bk, ar + d, w->kf + (size_t)t * d);
-      oracle_aap_linear_row(qr, al, d, Wv, d, sw[2], bv, ar + 2 * d, w->vf + (size_t)t * d);
+      const float *xr = w->x + (size_t)t * d;
+      if (full) {
+        float *sr = (float *)ar;
+        oracle_full_linear_row(xr, d, Fq, d, bq, sr, w->qf + (size_t)t * d);
+        oracle_full_linear_row(xr, d, Fk, d, bk, sr + d, w->kf + (size_t)t * d);
+        oracle_full_linear_row(xr, d, Fv, d, bv, sr + 2 * d, w->vf + (size_t)t * d);
+      } else {
+        if (per_word) quant_with_alpha(xr, d, al = aw0, qr);
+        else oracle_quant_row(xr, d, m->alpha_floor, qr, &al);
+        oracle_aap_linear_row(qr, al, d, Wq, d, sw[0], bq, ar, w->qf + (size_t)t * d);
+        oracle_aap_linear_row(qr, al, d, Wk, d, sw[1], bk, ar + d, w->kf + (size_t)t * d);
+        oracle_aap_linear_row(qr, al, d, Wv, d, sw[2], bv, ar + 2 * d, w->vf + (size_t)t * d);
+      }
       if (capture) {
         int64_t off = cap_row_off(m, bi, l, 0, t);
-        if (cap->q) memcpy(cap->q + off, qr, (size_t)d);
+        if (cap->q && !full) memcpy(cap->q + off, qr, (size_t)d);
         if (cap->acc) memcpy(cap->acc + off, ar, sizeof(int32_t) * 3 * d);
-        if (cap->alpha) cap->alpha[off / (4 * d)] = al;
+        if (cap->alpha && !full) cap->alpha[off / (4 * d)] = al;
       }
     }
     /* S5: HPSA (Sec. 4.2) */
@@ -408,35 +461,45 @@ static void decode_one(const oracle_model *m, const float *y, uint8_t *bits, uin
     const float aw1 = per_word ? matrix_alpha(w->a, T, d, (size_t)d, m->alpha_floor) : 0.0f;
     for (int t = 0; t < T; ++t) {
       int8_t *qr = w->q + (size_t)t * F;
-      float al;
+      float al = 0.0f;
       int32_t *ar = w->acc + (size_t)t * 4 * d;
-      if (per_word) quant_with_alpha(w->a + (size_t)t * d, d, al = aw1, qr);
-      else oracle_quant_row(w->a + (size_t)t * d, d, m->alpha_floor, qr, &al);
-      oracle_aap_linear_row(qr, al, d, Wo, d, sw[3], bo, ar, w->o + (size_t)t * d);
+      const float *arow = w->a + (size_t)t * d;
+      if (full) {
+        oracle_full_linear_row(arow, d, Fo, d, bo, (float *)ar, w->o + (size_t)t * d);
+      } else {
+        if (per_word) quant_with_alpha(arow, d, al = aw1, qr);
+        else oracle_quant_row(arow, d, m->alpha_floor, qr, &al);
+        oracle_aap_linear_row(qr, al, d, Wo, d, sw[3], bo, ar, w->o + (size_t)t * d);
+      }
       for (int c = 0; c < d; ++c) w->v[c] = w->x[(size_t)t * d + c] + w->o[(size_t)t * d + c];
       oracle_layernorm_row(w->v, d, g1, be1, m->ln_eps, w->x + (size_t)t * d);
       if (capture) {
         int64_t off = cap_row_off(m, bi, l, 1, t);
-        if (cap->q) memcpy(cap->q + off, qr, (size_t)d);
+        if (cap->q && !full) memcpy(cap->q + off, qr, (size_t)d);
         if (cap->acc) memcpy(cap->acc + off, ar, sizeof(int32_t) * d);
-        if (cap->alpha) cap->alpha[off / (4 * d)] = al;
+        if (cap->alpha && !full) cap->alpha[off / (4 * d)] = al;
       }
     }
     /* S7/S8: FFN with ReLU (Sec. 4 item 4) or GELU, residual, LayerNorm */
     const float aw2 = per_word ? matrix_alpha(w->x, T, d, (size_t)d, m->alpha_floor) : 0.0f;
     for (int t = 0; t < T; ++t) {
       int8_t *qr = w->q + (size_t)t * F;
-      float al;
+      float al = 0.0f;
       int32_t *ar = w->acc + (size_t)t * 4 * d;
       float *ur = w->u + (size_t)t * F;
-      if (per_word) quant_with_alpha(w->x + (size_t)t * d, d, al = aw2, qr);
-      else oracle_quant_row(w->x + (size_t)t * d, d, m->alpha_floor, qr, &al);
-      oracle_aap_linear_row(qr, al, d, W1, F, sw[4], b1, ar, ur);
+      const float *xr = w->x + (size_t)t * d;
+      if (full) {
+        oracle_full_linear_row(xr, d, F1, F, b1, (float *)ar, ur);
+      } else {
+        if (per_word) quant_with_alpha(xr, d, al = aw2, qr);
+        else oracle_quant_row(xr, d, m->alpha_floor, qr, &al);
+        oracle_aap_linear_row(qr, al, d, W1, F, sw[4], b1, ar, ur);
+      }
       if (capture) {
         int64_t off = cap_row_off(m, bi, l, 2, t);
-        if (cap->q) memcpy(cap->q + off, qr, (size_t)d);
+        if (cap->q && !full) memcpy(cap->q + off, qr, (size_t)d);
         if (cap->acc) memcpy(cap->acc + off, ar, sizeof(int32_t) * F);
-        if (cap->alpha) cap->alpha[off / (4 * d)] = al;
+        if (cap->alpha && !full) cap->alpha[off / (4 * d)] = al;
       }
       if (m->activation == 0)
         for (int c = 0; c < F; ++c) ur[c] = ur[c] > 0.0f ? ur[c] : 0.0f;
@@ -446,19 +509,23 @@ static void decode_one(const oracle_model *m, const float *y, uint8_t *bits, uin
     const float aw3 = per_word ? matrix_alpha(w->u, T, F, (size_t)F, m->alpha_floor) : 0.0f;
     for (int t = 0; t < T; ++t) {
       int8_t *qr = w->q + (size_t)t * F;
-      float al;
+      float al = 0.0f;
       int32_t *ar = w->acc + (size_t)t * 4 * d;
       const float *ur = w->u + (size_t)t * F;
-      if (per_word) quant_with_alpha(ur, F, al = aw3, qr);
-      else oracle_quant_row(ur, F, m->alpha_floor, qr, &al);
-      oracle_aap_linear_row(qr, al, F, W2, d, sw[5], b2, ar, w->o);
+      if (full) {
+        oracle_full_linear_row(ur, F, F2, d, b2, (float *)ar, w->o);
+      } else {
+        if (per_word) quant_with_alpha(ur, F, al = aw3, qr);
+        else oracle_quant_row(ur, F, m->alpha_floor, qr, &al);
+        oracle_aap_linear_row(qr, al, F, W2, d, sw[5], b2, ar, w->o);
+      }
       for (int c = 0; c < d; ++c) w->v[c] = w->x[(size_t)t * d + c] + w->o[c];
       oracle_layernorm_row(w->v, d, g2, be2, m->ln_eps, w->x + (size_t)t * d);
       if (capture) {
         int64_t off = cap_row_off(m, bi, l, 3, t);
-        if (cap->q) memcpy(cap->q + off, qr, (size_t)F);
+        if (cap->q && !full) memcpy(cap->q + off, qr, (size_t)F);
         if (cap->acc) memcpy(cap->acc + off, ar, sizeof(int32_t) * d);
-        if (cap->alpha) cap->alpha[off / (4 * d)] = al;
+        if (cap->alpha && !full) cap->alpha[off / (4 * d)] = al;
       }
     }
   }
@@ -553,6 +620,8 @@ static int validate(const oracle_model *m) {
   if (m->d > 1024 || m->d / m->heads > 64 || (m->d / m->heads) % 2 || m->n_layers < 0) return ORACLE_EINVAL;
   if (m->h_first < 0 || m->h_first > m->heads || m->d_spe < 0 || m->d_spe >= m->d) return ORACLE_EINVAL;
   if (m->mask_mode < 0 || m->mask_mode > 1 || m->alpha_mode < 0 || m->alpha_mode > 1) return ORACLE_EINVAL;
+  if (m->linear_mode < 0 || m->linear_mode > 1) return ORACLE_EINVAL;
+  if (m->linear_mode == 1 && (!m->w_full || m->alpha_mode != 0)) return ORACLE_EINVAL;
   if (m->d_spe > 0 && !m->spe) return ORACLE_EINVAL;
   if (m->ffn_mult != 4 || m->activation < 0 || m->activation > 1) return ORACLE_EINVAL; /* FFN width 4d, ReLU/GELU */
   return ORACLE_OK;

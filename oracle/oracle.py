@@ -40,12 +40,12 @@ class OracleModel(ctypes.Structure):
         ("n", ctypes.c_int32), ("k", ctypes.c_int32), ("d", ctypes.c_int32), ("n_layers", ctypes.c_int32),
         ("heads", ctypes.c_int32), ("h_first", ctypes.c_int32), ("d_spe", ctypes.c_int32),
         ("ffn_mult", ctypes.c_int32), ("activation", ctypes.c_int32), ("mask_mode", ctypes.c_int32),
-        ("alpha_mode", ctypes.c_int32),
+        ("alpha_mode", ctypes.c_int32), ("linear_mode", ctypes.c_int32),
         ("H", ctypes.c_void_p), ("emb", ctypes.c_void_p), ("spe", ctypes.c_void_p), ("w", ctypes.c_void_p),
         ("w_scale", ctypes.c_void_p), ("bias", ctypes.c_void_p), ("ln_gamma", ctypes.c_void_p),
         ("ln_beta", ctypes.c_void_p), ("w_d1", ctypes.c_void_p), ("b_d1", ctypes.c_float),
         ("w_out", ctypes.c_void_p), ("b_out", ctypes.c_void_p), ("ln_eps", ctypes.c_float),
-        ("alpha_floor", ctypes.c_float),
+        ("alpha_floor", ctypes.c_float), ("w_full", ctypes.c_void_p),
     ]
 
 
@@ -68,6 +68,9 @@ def lib():
             L.oracle_exp2_series.restype = ctypes.c_float
             L.oracle_gelu.argtypes = [ctypes.c_float]
             L.oracle_gelu.restype = ctypes.c_float
+            L.oracle_bf16_round.argtypes = [ctypes.c_float]
+            L.oracle_bf16_round.restype = ctypes.c_float
+            L.oracle_full_linear_row.argtypes = [P, ctypes.c_int, P, ctypes.c_int, P, P, P]
             L.oracle_psum.argtypes = [P, ctypes.c_int]
             L.oracle_psum.restype = ctypes.c_float
             L.oracle_hard_decision.argtypes = [P, ctypes.c_int, P]
@@ -104,6 +107,24 @@ def gelu(x) -> np.ndarray:
     L = lib()
     xs = np.asarray(x, dtype=np.float32).ravel()
     return np.array([L.oracle_gelu(float(v)) for v in xs], dtype=np.float32)
+
+
+def bf16_round(x) -> np.ndarray:
+    L = lib()
+    xs = np.asarray(x, dtype=np.float32).ravel()
+    return np.array([L.oracle_bf16_round(float(v)) for v in xs], dtype=np.float32)
+
+
+def full_linear_row(x, W, b):
+    """The full-precision linear layer of one row: (fp32 sums before the bias, outputs)."""
+    x = np.ascontiguousarray(x, dtype=np.float32)
+    W = np.ascontiguousarray(W, dtype=np.float32)
+    b = np.ascontiguousarray(b, dtype=np.float32)
+    N, K = W.shape
+    s = np.zeros(N, np.float32)
+    out = np.zeros(N, np.float32)
+    lib().oracle_full_linear_row(_p(x), K, _p(W), N, _p(b), _p(s), _p(out))
+    return s, out
 
 
 def exp2_coefficients() -> np.ndarray:
@@ -214,15 +235,21 @@ class _Packed:
         self.w_d1 = np.ascontiguousarray(model.w_d1, dtype=np.float32)
         self.w_out = np.ascontiguousarray(model.w_out, dtype=np.float32)
         self.b_out = np.ascontiguousarray(model.b_out, dtype=np.float32)
+        lm = int(getattr(model, "linear_mode", 0))
+        self.w_full = (np.ascontiguousarray(np.concatenate(
+            [np.asarray(w, np.float32).ravel() for layer in model.w_full for w in layer]))
+            if lm == 1 else np.zeros(1, np.float32))
         if self.w_scale.size == 0:
             self.w_scale = np.zeros(1, np.float32)
             self.ln_gamma = np.zeros(1, np.float32)
             self.ln_beta = np.zeros(1, np.float32)
         self.st = OracleModel(
             model.n, model.k, model.d, model.n_layers, model.heads, model.h_first, model.d_spe, model.ffn_mult,
-            model.activation, int(getattr(model, "mask_mode", 0)), int(getattr(model, "alpha_mode", 0)), _p(self.H), _p(self.emb), _p(self.spe) if self.spe.size else None, _p(self.w),
+            model.activation, int(getattr(model, "mask_mode", 0)), int(getattr(model, "alpha_mode", 0)), lm,
+            _p(self.H), _p(self.emb), _p(self.spe) if self.spe.size else None, _p(self.w),
             _p(self.w_scale), _p(self.bias), _p(self.ln_gamma), _p(self.ln_beta), _p(self.w_d1),
-            float(model.b_d1), _p(self.w_out), _p(self.b_out), float(model.ln_eps), float(model.alpha_floor))
+            float(model.b_d1), _p(self.w_out), _p(self.b_out), float(model.ln_eps), float(model.alpha_floor),
+            _p(self.w_full) if lm == 1 else None)
 
 
 def decode(model, y, nthreads: Optional[int] = None, cap_B: int = 0):

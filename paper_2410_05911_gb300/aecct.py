@@ -41,12 +41,12 @@ class ModelDesc(ctypes.Structure):
         ("heads", ctypes.c_int32), ("h_first", ctypes.c_int32), ("d_spe", ctypes.c_int32),
         ("ffn_mult", ctypes.c_int32), ("activation", ctypes.c_int32), ("cluster_ctas", ctypes.c_int32),
         ("attention_mode", ctypes.c_int32), ("mask_mode", ctypes.c_int32),
-        ("alpha_mode", ctypes.c_int32),
+        ("alpha_mode", ctypes.c_int32), ("linear_mode", ctypes.c_int32),
         ("H", ctypes.c_void_p), ("emb", ctypes.c_void_p), ("spe", ctypes.c_void_p), ("w_packed", ctypes.c_void_p),
         ("w_scale", ctypes.c_void_p), ("bias", ctypes.c_void_p), ("ln_gamma", ctypes.c_void_p),
         ("ln_beta", ctypes.c_void_p), ("w_d1", ctypes.c_void_p), ("b_d1", ctypes.c_float),
         ("w_out", ctypes.c_void_p), ("b_out", ctypes.c_void_p), ("ln_eps", ctypes.c_float),
-        ("alpha_floor", ctypes.c_float), ("wait_limit_cycles", ctypes.c_int64),
+        ("alpha_floor", ctypes.c_float), ("wait_limit_cycles", ctypes.c_int64), ("w_full", ctypes.c_void_p),
     ]
 
 
@@ -126,12 +126,20 @@ class _HostModel:
         self.H = np.ascontiguousarray(model.H, dtype=np.uint8)
         self.emb = np.ascontiguousarray(model.emb, dtype=np.float32)
         self.spe = np.ascontiguousarray(model.spe, dtype=np.float32)
-        packed = []
-        for layer in model.w_tern:
-            for t in layer:
-                packed.append(pack_ternary(t).ravel())
-        self.w_packed = np.ascontiguousarray(np.concatenate(packed) if packed else np.zeros(1, np.uint8))
-        self.w_scale = np.ascontiguousarray(model.w_scale, dtype=np.float32).reshape(-1)
+        linear_mode = int(getattr(model, "linear_mode", 0))
+        # AAP linears: 2-bit ternary codes and scales; full-precision linears (linear_mode 1): fp32
+        # weights in the same per-block order (the arrays the mode does not read stay NULL)
+        w_full = getattr(model, "w_full", None)
+        if linear_mode != 1:
+            packed = [pack_ternary(t).ravel() for layer in model.w_tern for t in layer]
+            self.w_packed = np.ascontiguousarray(np.concatenate(packed) if packed else np.zeros(1, np.uint8))
+            self.w_scale = np.ascontiguousarray(model.w_scale, dtype=np.float32).reshape(-1)
+        else:
+            self.w_packed = np.zeros(0, np.uint8)
+            self.w_scale = np.zeros(0, np.float32)
+        self.w_full = (np.ascontiguousarray(np.concatenate([np.asarray(w, np.float32).ravel()
+                                                            for layer in w_full for w in layer]))
+                       if linear_mode != 0 and w_full is not None else np.zeros(0, np.float32))
         self.bias = np.ascontiguousarray(
             np.concatenate([np.asarray(b, np.float32).ravel() for layer in model.bias for b in layer]))
         self.ln_gamma = np.ascontiguousarray(model.ln_gamma, dtype=np.float32).reshape(-1)
@@ -143,10 +151,10 @@ class _HostModel:
         self.desc = ModelDesc(
             model.n, model.k, model.d, model.n_layers, model.heads, model.h_first, model.d_spe, model.ffn_mult,
             model.activation, int(cluster_ctas), int(attention_mode), int(getattr(model, "mask_mode", 0)),
-            int(getattr(model, "alpha_mode", 0)), ptr(self.H), ptr(self.emb), ptr(self.spe), ptr(self.w_packed),
-            ptr(self.w_scale), ptr(self.bias), ptr(self.ln_gamma), ptr(self.ln_beta), ptr(self.w_d1),
-            float(model.b_d1), ptr(self.w_out), ptr(self.b_out), float(model.ln_eps), float(model.alpha_floor),
-            int(wait_limit_cycles))
+            int(getattr(model, "alpha_mode", 0)), linear_mode, ptr(self.H), ptr(self.emb), ptr(self.spe),
+            ptr(self.w_packed), ptr(self.w_scale), ptr(self.bias), ptr(self.ln_gamma), ptr(self.ln_beta),
+            ptr(self.w_d1), float(model.b_d1), ptr(self.w_out), ptr(self.b_out), float(model.ln_eps),
+            float(model.alpha_floor), int(wait_limit_cycles), ptr(self.w_full))
 
 
 def create_handle(model, cluster_ctas: int = 0, wait_limit_cycles: int = 0, attention_mode: int = 0):

@@ -192,11 +192,12 @@ struct SmemLayout {
   static constexpr uint32_t kRowCacheCol = (D == 128) ? 128u : 256u;
 };
 
-// decoder_kernel.cuh (ACT: 0 = ReLU, instantiated in decoder_kernel.cu; 1 = GELU, in
-// decoder_kernel_gelu.cu)
-template <int D, bool TASKS, int ACT>
+// decoder_kernel.cuh.  ACT: 0 = ReLU, 1 = GELU; LIN: 0 = AAP linears, 1 = full-precision (bf16)
+// linears.  Instantiated in decoder_kernel.cu (0, 0), decoder_kernel_gelu.cu (1, 0),
+// decoder_kernel_fp.cu (0, 1) and decoder_kernel_fp_gelu.cu (1, 1).
+template <int D, bool TASKS, int ACT, int LIN>
 cudaError_t launch_decode(const DecodeParams &p, cudaStream_t stream);
-template <int D, bool TASKS, int ACT>
+template <int D, bool TASKS, int ACT, int LIN>
 cudaError_t prepare_decode_kernel(int cluster_ctas, int *max_active_clusters);
 
 // api.cu diagnostics kernels live in selftest.cu

@@ -34,7 +34,8 @@ struct aecct_handle {
   int C = 1, G = 1, max_clusters = 0;
   bool tasks = false;  // warp-task attention (one CTA per group, d <= 64)
   int alpha_mode = 0;  // 1 = one alpha per quantised matrix of a word
-  int activation = 0;  // 0 = ReLU, 1 = GELU
+  int activation = 0;   // 0 = ReLU, 1 = GELU
+  int linear_mode = 0;  // 0 = AAP ternary linears, 1 = full-precision (bf16) linears
   float ln_eps = 0, alpha_floor = 0, att_scale = 0, b_d1 = 0;
   long long wait_limit = 0;
   int device = 0;
@@ -97,6 +98,15 @@ void free_handle(aecct_handle *h) {
   delete h;
 }
 
+// bf16 encoding of a finite fp32 value, rounded to nearest even (the low 16 bits decide; a tie
+// goes to the even upper half)
+uint16_t bf16_rne_bits(float f) {
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  u += 0x7FFFu + ((u >> 16) & 1u);
+  return static_cast<uint16_t>(u >> 16);
+}
+
 uint16_t f2bf_bits(float f) {
   // exact for the integers -1, 0, 1
   uint32_t u;
@@ -117,8 +127,12 @@ int validate(const aecct_model_desc *d) {
   if (d->attention_mode < 0 || d->attention_mode > 2) return AECCT_ERR_INVALID_ARG;
   if (d->mask_mode < 0 || d->mask_mode > 1) return AECCT_ERR_INVALID_ARG;
   if (d->alpha_mode < 0 || d->alpha_mode > 1) return AECCT_ERR_INVALID_ARG;
-  if (!d->H || !d->emb || !d->w_packed || !d->w_scale || !d->bias || !d->ln_gamma || !d->ln_beta || !d->w_d1 ||
-      !d->w_out || !d->b_out)
+  if (d->linear_mode < 0 || d->linear_mode > 1) return AECCT_ERR_INVALID_ARG;
+  const bool aap = d->linear_mode == 0;
+  if (!aap && d->alpha_mode != 0) return AECCT_ERR_INVALID_ARG;  // alpha belongs to eq. Quant
+  if (aap && (!d->w_packed || !d->w_scale)) return AECCT_ERR_INVALID_ARG;
+  if (!aap && !d->w_full) return AECCT_ERR_INVALID_ARG;
+  if (!d->H || !d->emb || !d->bias || !d->ln_gamma || !d->ln_beta || !d->w_d1 || !d->w_out || !d->b_out)
     return AECCT_ERR_INVALID_ARG;
   if (d->d_spe > 0 && !d->spe) return AECCT_ERR_INVALID_ARG;
   if (!(d->ln_eps >= 0.0f) || !std::isfinite(d->ln_eps)) return AECCT_ERR_INVALID_ARG;
@@ -145,7 +159,13 @@ int validate(const aecct_model_desc *d) {
   if (d->ffn_mult != 4) return AECCT_ERR_UNSUPPORTED;
   const int T = 2 * n - d->k;
   if (T > kMaxCluster * kRows || T > 65535) return AECCT_ERR_UNSUPPORTED;
-  // packed weights: no code 10
+  // packed weights: no code 10; full-precision weights: finite
+  if (!aap) {
+    const size_t nw = (size_t)d->n_layers * 12u * d->d * d->d;
+    for (size_t i = 0; i < nw; ++i)
+      if (!std::isfinite(d->w_full[i])) return AECCT_ERR_INVALID_ARG;
+    return AECCT_OK;
+  }
   const size_t nbytes = (size_t)d->n_layers * 12u * d->d * d->d / 4u;
   for (size_t i = 0; i < nbytes; ++i) {
     const uint8_t b = d->w_packed[i];
@@ -174,21 +194,31 @@ int schedule_chunks(int D, ChunkDesc *out) {
   return D == 32 ? schedule_chunks_t<32>(out) : D == 64 ? schedule_chunks_t<64>(out) : schedule_chunks_t<128>(out);
 }
 
-// the compiled kernel for (d, attention mode, activation): task mode exists for d = 32 and 64
-template <int ACT>
+// the compiled kernel for (d, attention mode, activation ACT, linear mode LIN): task mode exists
+// for d = 32 and 64
+template <int ACT, int LIN>
 cudaError_t prepare_any(int D, bool tasks, int C, int *max_clusters) {
-  if (tasks) return D == 32 ? prepare_decode_kernel<32, true, ACT>(C, max_clusters)
-                            : prepare_decode_kernel<64, true, ACT>(C, max_clusters);
-  if (D == 32) return prepare_decode_kernel<32, false, ACT>(C, max_clusters);
-  if (D == 64) return prepare_decode_kernel<64, false, ACT>(C, max_clusters);
-  return prepare_decode_kernel<128, false, ACT>(C, max_clusters);
+  if (tasks) return D == 32 ? prepare_decode_kernel<32, true, ACT, LIN>(C, max_clusters)
+                            : prepare_decode_kernel<64, true, ACT, LIN>(C, max_clusters);
+  if (D == 32) return prepare_decode_kernel<32, false, ACT, LIN>(C, max_clusters);
+  if (D == 64) return prepare_decode_kernel<64, false, ACT, LIN>(C, max_clusters);
+  return prepare_decode_kernel<128, false, ACT, LIN>(C, max_clusters);
 }
-template <int ACT>
+template <int ACT, int LIN>
 cudaError_t launch_any(int D, bool tasks, const DecodeParams &p, cudaStream_t stream) {
-  if (tasks) return D == 32 ? launch_decode<32, true, ACT>(p, stream) : launch_decode<64, true, ACT>(p, stream);
-  if (D == 32) return launch_decode<32, false, ACT>(p, stream);
-  if (D == 64) return launch_decode<64, false, ACT>(p, stream);
-  return launch_decode<128, false, ACT>(p, stream);
+  if (tasks)
+    return D == 32 ? launch_decode<32, true, ACT, LIN>(p, stream) : launch_decode<64, true, ACT, LIN>(p, stream);
+  if (D == 32) return launch_decode<32, false, ACT, LIN>(p, stream);
+  if (D == 64) return launch_decode<64, false, ACT, LIN>(p, stream);
+  return launch_decode<128, false, ACT, LIN>(p, stream);
+}
+cudaError_t prepare_variant(int act, int lin, int D, bool tasks, int C, int *max_clusters) {
+  if (lin == 0) return act == 0 ? prepare_any<0, 0>(D, tasks, C, max_clusters) : prepare_any<1, 0>(D, tasks, C, max_clusters);
+  return act == 0 ? prepare_any<0, 1>(D, tasks, C, max_clusters) : prepare_any<1, 1>(D, tasks, C, max_clusters);
+}
+cudaError_t launch_variant(int act, int lin, int D, bool tasks, const DecodeParams &p, cudaStream_t stream) {
+  if (lin == 0) return act == 0 ? launch_any<0, 0>(D, tasks, p, stream) : launch_any<1, 0>(D, tasks, p, stream);
+  return act == 0 ? launch_any<0, 1>(D, tasks, p, stream) : launch_any<1, 1>(D, tasks, p, stream);
 }
 
 }  // namespace
@@ -259,8 +289,7 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
     return AECCT_ERR_NO_DEVICE;
   }
   int max_clusters = 0;
-  e = d.activation == 0 ? prepare_any<0>(D, tasks, best_C, &max_clusters)
-                        : prepare_any<1>(D, tasks, best_C, &max_clusters);
+  e = prepare_variant(d.activation, d.linear_mode, D, tasks, best_C, &max_clusters);
   if (e != cudaSuccess) return cuda_fail(e, "kernel occupancy");
   if (max_clusters < 1) {
     g_last_error = "no cluster of this size fits on the device";
@@ -273,6 +302,7 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
   h->ln_eps = d.ln_eps, h->alpha_floor = d.alpha_floor, h->b_d1 = d.b_d1, h->device = dev;
   h->alpha_mode = d.alpha_mode;
   h->activation = d.activation;
+  h->linear_mode = d.linear_mode;
   h->att_scale = static_cast<float>(1.4426950408889634074 / std::sqrt(static_cast<double>(D / kHeads)));
   h->wait_limit = d.wait_limit_cycles ? d.wait_limit_cycles : (1LL << 32);
 
@@ -428,7 +458,8 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
     }
   }
 
-  // ---- weights: 2-bit codes -> bf16 K-major core-matrix chunks, in the order the MMA consumes them
+  // ---- weights: 2-bit codes (or full-precision values rounded to bf16) -> bf16 K-major
+  // core-matrix chunks, in the order the MMA consumes them
   const Gemm gemms[4] = {{3 * D, D}, {D, D}, {F, D}, {D, F}};
   const int nch = schedule_chunks(D, h->chunks);
   const uint32_t off = h->chunks[nch - 1].off + h->chunks[nch - 1].bytes;
@@ -436,26 +467,32 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
   h->layer_bytes = off;
   std::vector<uint16_t> ws((size_t)d.n_layers * off / 2, 0);
   {
-    const size_t per_layer_packed = 12u * (size_t)D * D / 4u;
-    std::vector<int8_t> W[4];
+    const size_t per_layer_packed = 12u * (size_t)D * D / 4u, per_layer_full = 12u * (size_t)D * D;
+    std::vector<uint16_t> W[4];  // bf16 encodings, [N][K] per GEMM
     for (int l = 0; l < d.n_layers; ++l) {
-      const uint8_t *pk = d.w_packed + per_layer_packed * l;
-      // the six matrices in ABI order, unpacked
-      auto unpack = [&](const uint8_t *src, int rows, int cols, int8_t *dst) {
-        for (int r = 0; r < rows; ++r)
-          for (int c = 0; c < cols; ++c) {
-            const uint8_t byte = src[(size_t)r * (cols / 4) + c / 4];
-            dst[(size_t)r * cols + c] = tern((byte >> (2 * (c % 4))) & 3u);
-          }
+      // the six matrices in ABI order, as bf16: ternary codes unpacked (exact), or
+      // full-precision values rounded to nearest even
+      auto unpack = [&](size_t first, int rows, int cols, uint16_t *dst) {
+        if (d.linear_mode == 0) {
+          const uint8_t *src = d.w_packed + per_layer_packed * l + first / 4;
+          for (int r = 0; r < rows; ++r)
+            for (int c = 0; c < cols; ++c) {
+              const uint8_t byte = src[(size_t)r * (cols / 4) + c / 4];
+              dst[(size_t)r * cols + c] = f2bf_bits(static_cast<float>(tern((byte >> (2 * (c % 4))) & 3u)));
+            }
+        } else {
+          const float *src = d.w_full + per_layer_full * l + first;
+          for (size_t i = 0; i < (size_t)rows * cols; ++i) dst[i] = bf16_rne_bits(src[i]);
+        }
       };
       for (int g = 0; g < 4; ++g) W[g].assign((size_t)gemms[g].N * gemms[g].K, 0);
-      const size_t dd4 = (size_t)D * D / 4;
-      unpack(pk, D, D, W[0].data());                                 // W_q -> QKV rows [0, D)
-      unpack(pk + dd4, D, D, W[0].data() + (size_t)D * D);           // W_k -> rows [D, 2D)
-      unpack(pk + 2 * dd4, D, D, W[0].data() + (size_t)2 * D * D);   // W_v -> rows [2D, 3D)
-      unpack(pk + 3 * dd4, D, D, W[1].data());                       // W_o
-      unpack(pk + 4 * dd4, F, D, W[2].data());                       // W_1
-      unpack(pk + 4 * dd4 + (size_t)F * D / 4, D, F, W[3].data());   // W_2
+      const size_t dd = (size_t)D * D;
+      unpack(0, D, D, W[0].data());                        // W_q -> QKV rows [0, D)
+      unpack(dd, D, D, W[0].data() + dd);                  // W_k -> rows [D, 2D)
+      unpack(2 * dd, D, D, W[0].data() + 2 * dd);          // W_v -> rows [2D, 3D)
+      unpack(3 * dd, D, D, W[1].data());                   // W_o
+      unpack(4 * dd, F, D, W[2].data());                   // W_1
+      unpack(4 * dd + (size_t)F * D, D, F, W[3].data());   // W_2
       uint16_t *lw = ws.data() + (size_t)l * off / 2;
       for (int c = 0; c < nch; ++c) {
         const ChunkDesc &ch = h->chunks[c];
@@ -463,8 +500,7 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
         uint8_t *base = reinterpret_cast<uint8_t *>(lw) + ch.off;
         for (int rr = 0; rr < ch.nrows; ++rr)
           for (int cc = 0; cc < ch.kcols; ++cc) {
-            const int8_t v = W[ch.gemm][(size_t)(ch.n0 + rr) * gm.K + ch.k0 + cc];
-            const uint16_t bits = f2bf_bits(static_cast<float>(v));
+            const uint16_t bits = W[ch.gemm][(size_t)(ch.n0 + rr) * gm.K + ch.k0 + cc];
             std::memcpy(base + core_off(rr, cc, ch.kcols), &bits, 2);
           }
       }
@@ -480,7 +516,8 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
     std::memcpy(v + LayerParamLayout::ln1b(D), d.ln_beta + (size_t)l * 2 * D, sizeof(float) * D);
     std::memcpy(v + LayerParamLayout::ln2g(D), d.ln_gamma + (size_t)l * 2 * D + D, sizeof(float) * D);
     std::memcpy(v + LayerParamLayout::ln2b(D), d.ln_beta + (size_t)l * 2 * D + D, sizeof(float) * D);
-    std::memcpy(v + LayerParamLayout::sw(D), d.w_scale + (size_t)l * 6, sizeof(float) * 6);
+    if (d.linear_mode == 0) std::memcpy(v + LayerParamLayout::sw(D), d.w_scale + (size_t)l * 6, sizeof(float) * 6);
+    else for (int i = 0; i < 6; ++i) v[LayerParamLayout::sw(D) + i] = 1.0f;
   }
   const int de = D - d.d_spe;
   if ((rc = dev_upload(h, &h->wstream, reinterpret_cast<const uint8_t *>(ws.data()), ws.size() * 2)) ||
@@ -567,7 +604,7 @@ int aecct_decode(aecct_handle *h, const float *y_dev, int64_t B, uint8_t *bits_d
   p.cap_B = h->cap_B, p.cap_q = h->cap_q, p.cap_acc = h->cap_acc, p.cap_alpha = h->cap_alpha, p.cap_syn = h->cap_syn;
   p.err = h->d_err, p.wait_limit = h->wait_limit;
   cudaError_t e;
-  e = h->activation == 0 ? launch_any<0>(h->d, h->tasks, p, stream) : launch_any<1>(h->d, h->tasks, p, stream);
+  e = launch_variant(h->activation, h->linear_mode, h->d, h->tasks, p, stream);
   if (e != cudaSuccess) return cuda_fail(e, "decode launch");
   if ((e = cudaMemcpyAsync(h->h_err, h->d_err, sizeof(int), cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
     return cuda_fail(e, "status copy");
@@ -688,7 +725,7 @@ int aecct_decode_host_noalloc(aecct_handle *h, const float *y_host, int64_t B, u
   p.ln_eps = h->ln_eps, p.alpha_floor = h->alpha_floor, p.att_scale = h->att_scale, p.alpha_mode = h->alpha_mode;
   p.cap_B = h->cap_B, p.cap_q = h->cap_q, p.cap_acc = h->cap_acc, p.cap_alpha = h->cap_alpha, p.cap_syn = h->cap_syn;
   p.err = err, p.wait_limit = h->wait_limit;
-  e = h->activation == 0 ? launch_any<0>(h->d, h->tasks, p, stream) : launch_any<1>(h->d, h->tasks, p, stream);
+  e = launch_variant(h->activation, h->linear_mode, h->d, h->tasks, p, stream);
   if (e != cudaSuccess) return cuda_fail(e, "decode launch");
   if ((e = cudaMemcpyAsync(bits_host, bits_dev, b * n, cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
     return cuda_fail(e, "copy bits");

@@ -1,18 +1,18 @@
 // decoder_kernel.cu -- instantiations of the decoder kernel with the ReLU feed-forward activation
-// (Sec. 4 item 4).
+// (Sec. 4 item 4), AAP linears (Sec. 4.1).
 #include "decoder_kernel.cuh"
 
 namespace aecct {
 
-template cudaError_t launch_decode<32, false, 0>(const DecodeParams &, cudaStream_t);
-template cudaError_t launch_decode<64, false, 0>(const DecodeParams &, cudaStream_t);
-template cudaError_t launch_decode<128, false, 0>(const DecodeParams &, cudaStream_t);
-template cudaError_t launch_decode<32, true, 0>(const DecodeParams &, cudaStream_t);
-template cudaError_t launch_decode<64, true, 0>(const DecodeParams &, cudaStream_t);
-template cudaError_t prepare_decode_kernel<32, false, 0>(int, int *);
-template cudaError_t prepare_decode_kernel<64, false, 0>(int, int *);
-template cudaError_t prepare_decode_kernel<128, false, 0>(int, int *);
-template cudaError_t prepare_decode_kernel<32, true, 0>(int, int *);
-template cudaError_t prepare_decode_kernel<64, true, 0>(int, int *);
+template cudaError_t launch_decode<32, false, 0, 0>(const DecodeParams &, cudaStream_t);
+template cudaError_t launch_decode<64, false, 0, 0>(const DecodeParams &, cudaStream_t);
+template cudaError_t launch_decode<128, false, 0, 0>(const DecodeParams &, cudaStream_t);
+template cudaError_t launch_decode<32, true, 0, 0>(const DecodeParams &, cudaStream_t);
+template cudaError_t launch_decode<64, true, 0, 0>(const DecodeParams &, cudaStream_t);
+template cudaError_t prepare_decode_kernel<32, false, 0, 0>(int, int *);
+template cudaError_t prepare_decode_kernel<64, false, 0, 0>(int, int *);
+template cudaError_t prepare_decode_kernel<128, false, 0, 0>(int, int *);
+template cudaError_t prepare_decode_kernel<32, true, 0, 0>(int, int *);
+template cudaError_t prepare_decode_kernel<64, true, 0, 0>(int, int *);
 
 }  // namespace aecct

@@ -238,6 +238,26 @@ __device__ __forceinline__ void store_codes(uint32_t tile, int r, int c0, int kd
   }
 }
 
+// write LEN consecutive fp32 values of row r, rounded to bf16 (round to nearest even), into a
+// K-major operand tile (full-precision linears)
+__device__ __forceinline__ uint32_t pack_bf16x2_rn(float a, float b) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);  // a in the low half
+  return *reinterpret_cast<const uint32_t *>(&v);
+}
+template <int LEN>
+__device__ __forceinline__ void store_bf16(uint32_t tile, int r, int c0, int kdim, const float *v) {
+  if constexpr (LEN == 4) {
+    st_shared_v2(tile + core_off(r, c0, kdim), pack_bf16x2_rn(v[0], v[1]), pack_bf16x2_rn(v[2], v[3]));
+  } else {
+    static_assert(LEN % 8 == 0, "bf16 run");
+#pragma unroll
+    for (int j = 0; j < LEN; j += 8)
+      st_shared_v4(tile + core_off(r, c0 + j, kdim), pack_bf16x2_rn(v[j], v[j + 1]),
+                   pack_bf16x2_rn(v[j + 2], v[j + 3]), pack_bf16x2_rn(v[j + 4], v[j + 5]),
+                   pack_bf16x2_rn(v[j + 6], v[j + 7]));
+  }
+}
+
 template <int N>
 __device__ __forceinline__ void ldg_vec(const float *src, float *dst) {
   static_assert(N % 4 == 0, "vector");
@@ -918,7 +938,7 @@ struct Issuer<128, TASKS> {
 // ------------------------------------------------------------------------------------------
 // the kernel
 // ------------------------------------------------------------------------------------------
-template <int D, bool TASKS, int ACT>
+template <int D, bool TASKS, int ACT, int LIN>
 __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid_constant__ DecodeParams p) {
   using L = SmemLayout<D, TASKS>;
   using LP = LayerParamLayout;
@@ -1145,8 +1165,12 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           x[j] = v;
         }
       }
-      // Quant(x) -> QKV operand (Sec. 4.1 eq. Quant)
+      // Quant(x) -> QKV operand (Sec. 4.1 eq. Quant); full-precision linears: x rounded to bf16
       auto quant_x_to_aop = [&]() -> float {
+        if constexpr (LIN == 1) {
+          store_bf16<XS>(aop, r, sl * XS, D, x);
+          return 0.0f;
+        }
         float a = 0.0f;
 #pragma unroll
         for (int j = 0; j < XS; ++j) a = fmaxf(a, fabsf(x[j]));
@@ -1158,6 +1182,12 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         codes<XS>(x, rr, qv);
         store_codes<XS>(aop, r, sl * XS, D, qv);
         return rr;
+      };
+      // dequantisation factor gamma*delta * alpha / Q_b of eq. AAPLinear for the scale at swp;
+      // 1 for full-precision linears (out = acc + b)
+      auto dq_factor = [&](const float *swp) -> float {
+        if constexpr (LIN == 1) return 1.0f;
+        return __fdiv_rn(__fmul_rn(__ldg(swp), alpha_in), 127.0f);
       };
       // x <- LayerNorm(x + (acc * f + bias)) with gamma g and beta be (Post-LN, Sec. 5)
       auto residual_ln = [&](const float *ac, float f, const float *bias, const float *g, const float *be) {
@@ -1182,6 +1212,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         for (int j = 0; j < XS; ++j) x[j] = __fadd_rn(__fmul_rn(__fmul_rn(v[j], rstd), gg[j]), bt[j]);
       };
       auto capture_q = [&](int layer, int gemm, const float *qv, int c0, int len, float alpha) {
+        if constexpr (LIN == 1) return;  // no codes or alpha with full-precision linears
         const int64_t row = ((b * p.n_layers + layer) * 4 + gemm) * T + t;
         if (p.cap_q)
           for (int j = 0; j < len; ++j) p.cap_q[row * W4 + c0 + j] = static_cast<int8_t>(qv[j]);
@@ -1190,7 +1221,8 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
       auto capture_acc = [&](int layer, int gemm, const float *av, int c0, int len) {
         const int64_t row = ((b * p.n_layers + layer) * 4 + gemm) * T + t;
         if (p.cap_acc)
-          for (int j = 0; j < len; ++j) p.cap_acc[row * W4 + c0 + j] = static_cast<int32_t>(av[j]);
+          for (int j = 0; j < len; ++j)
+            p.cap_acc[row * W4 + c0 + j] = LIN == 1 ? __float_as_int(av[j]) : static_cast<int32_t>(av[j]);
       };
 
       {
@@ -1212,9 +1244,9 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         // so that attention runs with the registers it needs
         tmem_st<XS>(tl + 3 * D + sl * XS, x);
         tmem_wait_st();
-        const float fq = __fdiv_rn(__fmul_rn(__ldg(sw + 0), alpha_in), 127.0f);
-        const float fk = __fdiv_rn(__fmul_rn(__ldg(sw + 1), alpha_in), 127.0f);
-        const float fv = __fdiv_rn(__fmul_rn(__ldg(sw + 2), alpha_in), 127.0f);
+        const float fq = dq_factor(sw + 0);
+        const float fk = dq_factor(sw + 1);
+        const float fv = dq_factor(sw + 2);
 #pragma unroll
         for (int hh = 0; hh < 2; ++hh) {
           const int e = sl + 4 * hh;
@@ -1301,17 +1333,21 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
               av[hh * DH + 4 * i + 2] = v.z, av[hh * DH + 4 * i + 3] = v.w;
             }
           }
-          float amax = 0.0f;
+          if constexpr (LIN == 1) {
+            store_bf16<XS>(aop, r, sl * XS, D, av);
+          } else {
+            float amax = 0.0f;
 #pragma unroll
-          for (int j = 0; j < XS; ++j) amax = fmaxf(amax, fabsf(av[j]));
-          float a = word_alpha(row_max(amax));
-          a = (a > p.alpha_floor) ? a : p.alpha_floor;
-          alpha_in = a;
-          const float rr = __fdiv_rn(127.0f, a);
-          float qv[XS];
-          codes<XS>(av, rr, qv);
-          store_codes<XS>(aop, r, sl * XS, D, qv);
-          if (cap) capture_q(l, 1, qv, sl * XS, XS, alpha_in);
+            for (int j = 0; j < XS; ++j) amax = fmaxf(amax, fabsf(av[j]));
+            float a = word_alpha(row_max(amax));
+            a = (a > p.alpha_floor) ? a : p.alpha_floor;
+            alpha_in = a;
+            const float rr = __fdiv_rn(127.0f, a);
+            float qv[XS];
+            codes<XS>(av, rr, qv);
+            store_codes<XS>(aop, r, sl * XS, D, qv);
+            if (cap) capture_q(l, 1, qv, sl * XS, XS, alpha_in);
+          }
         } else {
         cluster_arrive(bar_kvr);
           cluster_wait(bar_kvr, kvr_ph);
@@ -1349,7 +1385,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             for (int i = 0; i < DH; ++i) amax = fmaxf(amax, fabsf(A[hh][i]));
           }
           // Quant(A) -> O operand
-          {
+          if constexpr (LIN == 1) {
+#pragma unroll
+            for (int hh = 0; hh < 2; ++hh) store_bf16<DH>(aop, r, (sl + 4 * hh) * DH, D, A[hh]);
+          } else {
             float a = word_alpha(row_max(amax));
             a = (a > p.alpha_floor) ? a : p.alpha_floor;
             alpha_in = a;
@@ -1373,7 +1412,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         // ---------------- S6: O projection + residual + LayerNorm (Sec. 5, Post-LN)
         wait_acc();
         {
-          const float fo = __fdiv_rn(__fmul_rn(__ldg(sw + 3), alpha_in), 127.0f);
+          const float fo = dq_factor(sw + 3);
           float ac[XS];
           tmem_ld<XS>(tl + sl * XS, ac);
           tmem_ld<XS>(tl + 3 * D + sl * XS, x);
@@ -1394,24 +1433,34 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         // ---------------- S7: FFN1 + ReLU (Sec. 4 item 4) or GELU, Quant(u) -> FFN2 operand
         wait_acc();
         {
-          const float f1 = __fdiv_rn(__fmul_rn(__ldg(sw + 4), alpha_in), 127.0f);
+          const float f1 = dq_factor(sw + 4);
           // ACT 0 = ReLU, 1 = GELU.  u = act(acc f1 + b1) in 32-column chunks of this thread's D
-          // hidden columns; with ReLU at d <= 64 u stays in registers between the row maximum and
-          // the codes, otherwise the second pass recomputes it (same operations, same values).
-          auto ffn1_epilogue = [&](auto act_tag) {
-            constexpr int ACT = decltype(act_tag)::value;
-            constexpr int NCH = D / 32;
-            constexpr bool KEEP = D <= 64 && ACT == 0;
-            auto hidden = [&](int c0, float *u, bool capture) {
-              float ac[32], bb[32];
-              tmem_ld<32>(tl + c0, ac);
-              tmem_wait_ld();
-              if (capture) capture_acc(l, 2, ac, c0, 32);
-              ldg_vec<32>(lp + LP::b1(D) + c0, bb);
-              dequant<32>(ac, f1, bb, u);
+          // hidden columns.  AAP: with ReLU at d <= 64 u stays in registers between the row
+          // maximum and the codes, otherwise the second pass recomputes it (same operations, same
+          // values).  Full-precision linears: one pass, u rounded to bf16.
+          constexpr int NCH = D / 32;
+          constexpr bool KEEP = D <= 64 && ACT == 0;
+          auto hidden = [&](int c0, float *u, bool capture) {
+            float ac[32], bb[32];
+            tmem_ld<32>(tl + c0, ac);
+            tmem_wait_ld();
+            if (capture) capture_acc(l, 2, ac, c0, 32);
+            ldg_vec<32>(lp + LP::b1(D) + c0, bb);
+            dequant<32>(ac, f1, bb, u);
 #pragma unroll
-              for (int j = 0; j < 32; ++j) u[j] = ACT == 0 ? (u[j] > 0.0f ? u[j] : 0.0f) : gelu_as(u[j]);
-            };
+            for (int j = 0; j < 32; ++j) u[j] = ACT == 0 ? (u[j] > 0.0f ? u[j] : 0.0f) : gelu_as(u[j]);
+          };
+          if constexpr (LIN == 1) {
+            // peers have finished reading this CTA's K/V: the shared region may now take u
+            if constexpr (!TASKS) cluster_wait(bar_kvf, kvf_ph);
+#pragma unroll
+            for (int ch = 0; ch < NCH; ++ch) {
+              const int c0 = sl * D + 32 * ch;
+              float u[32];
+              hidden(c0, u, cap);
+              store_bf16<32>(uqt, r, c0, 4 * D, u);
+            }
+          } else {
             float uk[KEEP ? D : 1];
             float umax = 0.0f;
 #pragma unroll
@@ -1446,15 +1495,14 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
               store_codes<32>(uqt, r, c0, 4 * D, qv);
               if (cap) capture_q(l, 3, qv, c0, 32, alpha_in);
             }
-          };
-          ffn1_epilogue(std::integral_constant<int, ACT>{});
+          }
         }
         signal_op(3, l, gi);
 
         // ---------------- S8: FFN2 + residual + LayerNorm
         wait_acc();
         {
-          const float f2 = __fdiv_rn(__fmul_rn(__ldg(sw + 5), alpha_in), 127.0f);
+          const float f2 = dq_factor(sw + 5);
           float ac[XS];
           tmem_ld<XS>(tl + sl * XS, ac);
           tmem_wait_ld();
@@ -1567,10 +1615,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   }
 }
 
-template <int D, bool TASKS, int ACT>
+template <int D, bool TASKS, int ACT, int LIN>
 cudaError_t prepare_decode_kernel(int cluster_ctas, int *max_active_clusters) {
   using L = SmemLayout<D, TASKS>;
-  cudaError_t e = cudaFuncSetAttribute(aecct_decoder_kernel<D, TASKS, ACT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(aecct_decoder_kernel<D, TASKS, ACT, LIN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(L::kTotal));
   if (e != cudaSuccess) return e;
   // ask for the smallest shared-memory carve-out that holds one CTA (1 KB of it is reserved by
@@ -1581,7 +1629,7 @@ cudaError_t prepare_decode_kernel(int cluster_ctas, int *max_active_clusters) {
     return e;
   if (smem_sm > 0) {
     const int pct = static_cast<int>((100ll * (L::kTotal + 1024) + smem_sm - 1) / smem_sm);
-    e = cudaFuncSetAttribute(aecct_decoder_kernel<D, TASKS, ACT>, cudaFuncAttributePreferredSharedMemoryCarveout,
+    e = cudaFuncSetAttribute(aecct_decoder_kernel<D, TASKS, ACT, LIN>, cudaFuncAttributePreferredSharedMemoryCarveout,
                              pct > 100 ? 100 : pct);
     if (e != cudaSuccess) return e;
   }
@@ -1596,10 +1644,10 @@ cudaError_t prepare_decode_kernel(int cluster_ctas, int *max_active_clusters) {
   cfg.dynamicSmemBytes = L::kTotal;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaOccupancyMaxActiveClusters(max_active_clusters, aecct_decoder_kernel<D, TASKS, ACT>, &cfg);
+  return cudaOccupancyMaxActiveClusters(max_active_clusters, aecct_decoder_kernel<D, TASKS, ACT, LIN>, &cfg);
 }
 
-template <int D, bool TASKS, int ACT>
+template <int D, bool TASKS, int ACT, int LIN>
 cudaError_t launch_decode(const DecodeParams &p, cudaStream_t stream) {
   using L = SmemLayout<D, TASKS>;
   cudaLaunchConfig_t cfg = {};
@@ -1614,7 +1662,7 @@ cudaError_t launch_decode(const DecodeParams &p, cudaStream_t stream) {
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, aecct_decoder_kernel<D, TASKS, ACT>, p);
+  return cudaLaunchKernelEx(&cfg, aecct_decoder_kernel<D, TASKS, ACT, LIN>, p);
 }
 
 }  // namespace aecct

@@ -1,0 +1,18 @@
+// decoder_kernel_fp_gelu.cu -- instantiations of the decoder kernel with the GELU feed-forward
+// activation and full-precision (bf16) linears (the ECCT baseline, Sec. 3).
+#include "decoder_kernel.cuh"
+
+namespace aecct {
+
+template cudaError_t launch_decode<32, false, 1, 1>(const DecodeParams &, cudaStream_t);
+template cudaError_t launch_decode<64, false, 1, 1>(const DecodeParams &, cudaStream_t);
+template cudaError_t launch_decode<128, false, 1, 1>(const DecodeParams &, cudaStream_t);
+template cudaError_t launch_decode<32, true, 1, 1>(const DecodeParams &, cudaStream_t);
+template cudaError_t launch_decode<64, true, 1, 1>(const DecodeParams &, cudaStream_t);
+template cudaError_t prepare_decode_kernel<32, false, 1, 1>(int, int *);
+template cudaError_t prepare_decode_kernel<64, false, 1, 1>(int, int *);
+template cudaError_t prepare_decode_kernel<128, false, 1, 1>(int, int *);
+template cudaError_t prepare_decode_kernel<32, true, 1, 1>(int, int *);
+template cudaError_t prepare_decode_kernel<64, true, 1, 1>(int, int *);
+
+}  // namespace aecct

@@ -345,6 +345,8 @@ class ModelTensors:
     alpha_floor: float = 1e-5
     mask_mode: int = 0  # 0 = HPSA rings (Sec. 4.2); 1 = ECCT code-aware mask for all heads (Sec. 3)
     alpha_mode: int = 0  # 0 = one absmax alpha per token (C-1); 1 = one per quantised matrix of a word
+    linear_mode: int = 0  # 0 = AAP ternary linears (Sec. 4.1); 1 = full-precision linears (ECCT, Sec. 3)
+    w_full: Optional[List[List[np.ndarray]]] = None  # linear_mode 1: fp32 weights, same order as w_tern
 
     @property
     def T(self) -> int:
@@ -388,6 +390,7 @@ def random_model(
     ffn_mult: int = 4,
     zero_weights: bool = False,
     binary: bool = False,
+    full_precision: bool = False,
 ) -> ModelTensors:
     """Seeded synthetic AECCT parameters shaped like a trained model.
 
@@ -401,6 +404,9 @@ def random_model(
     binary=True draws the binary-weight variant (App. D): every weight is +1 or -1 and the
     per-tensor scale is the mean |W| of N(0, 1/d_in) weights, sqrt(2 / (pi d_in)), times the
     same jitter.
+
+    full_precision=True also draws fp32 weights W ~ N(0, 1/d_in) per tensor (the full-precision
+    linear layers of the ECCT baseline, Sec. 3) and selects them (linear_mode = 1).
     """
     rng = np.random.Generator(np.random.PCG64(seed))
     T = code.T
@@ -413,8 +419,9 @@ def random_model(
     w_tern: List[List[np.ndarray]] = []
     bias: List[List[np.ndarray]] = []
     w_scale = np.zeros((n_layers, 6), dtype=np.float32)
+    w_full: Optional[List[List[np.ndarray]]] = [] if full_precision else None
     for l in range(n_layers):
-        wl, bl = [], []
+        wl, bl, fl = [], [], []
         for g, (dout, din) in enumerate(shapes):
             size = dout * din
             if zero_weights:
@@ -430,8 +437,12 @@ def random_model(
             base = math.sqrt(2.0 / (math.pi * din)) if binary else ternary_scale_for_zero_fraction(zero_frac, din)
             w_scale[l, g] = base * rng.uniform(0.9, 1.1)
             bl.append((0.1 * rng.standard_normal(dout)).astype(np.float32))
+            if full_precision:
+                fl.append((rng.standard_normal((dout, din)) / math.sqrt(din)).astype(np.float32))
         w_tern.append(wl)
         bias.append(bl)
+        if full_precision:
+            w_full.append(fl)
     ln_gamma = (1.0 + 0.1 * rng.standard_normal((n_layers, 2, d))).astype(np.float32)
     ln_beta = (0.1 * rng.standard_normal((n_layers, 2, d))).astype(np.float32)
     emb = rng.standard_normal((T, d - d_spe)).astype(np.float32)
@@ -445,6 +456,7 @@ def random_model(
         ffn_mult=ffn_mult, activation=activation, H=code.H.copy(), emb=emb, spe=spe,
         w_tern=w_tern, w_scale=w_scale, bias=bias, ln_gamma=ln_gamma, ln_beta=ln_beta,
         w_d1=w_d1, b_d1=b_d1, w_out=w_out, b_out=b_out,
+        linear_mode=1 if full_precision else 0, w_full=w_full,
     )
 
 

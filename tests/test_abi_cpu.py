@@ -68,6 +68,7 @@ def _status(model, **kw):
     (lambda m: setattr(m, "mask_mode", 2), A.AECCT_ERR_INVALID_ARG),
     (lambda m: setattr(m, "mask_mode", -1), A.AECCT_ERR_INVALID_ARG),
     (lambda m: setattr(m, "alpha_mode", 2), A.AECCT_ERR_INVALID_ARG),
+    (lambda m: setattr(m, "linear_mode", 2), A.AECCT_ERR_INVALID_ARG),
     (lambda m: setattr(m, "ffn_mult", 2), A.AECCT_ERR_UNSUPPORTED),
 ])
 def test_create_rejects_invalid_descriptions(mutate, expected):
@@ -101,6 +102,28 @@ def test_create_rejects_invalid_packed_code_and_shapes():
     # NULL description / output pointer
     assert A.load().aecct_create(None, ctypes.byref(h)) == A.AECCT_ERR_INVALID_ARG
     assert A.load().aecct_create(ctypes.byref(hm.desc), None) == A.AECCT_ERR_INVALID_ARG
+
+
+def test_full_precision_description_checks():
+    import ctypes
+    code = I.make_code("bch31_16")
+    m = I.random_model(code, 32, 1, seed=4, full_precision=True)
+    L = A.load()
+    h = ctypes.c_void_p()
+    # alpha belongs to the AAP quantiser: not with full-precision linears
+    m1 = copy.deepcopy(m)
+    m1.alpha_mode = 1
+    assert _status(m1) == A.AECCT_ERR_INVALID_ARG
+    # the fp32 weights are required, and must be finite
+    hm = A._HostModel(m)
+    hm.desc.w_full = None
+    assert L.aecct_create(ctypes.byref(hm.desc), ctypes.byref(h)) == A.AECCT_ERR_INVALID_ARG
+    hm = A._HostModel(m)
+    hm.w_full[7] = np.float32(np.inf)
+    assert L.aecct_create(ctypes.byref(hm.desc), ctypes.byref(h)) == A.AECCT_ERR_INVALID_ARG
+    # the ternary arrays are not read: NULL is fine (create then goes on to the device checks)
+    hm = A._HostModel(m)
+    assert hm.desc.w_packed is None and hm.desc.w_scale is None
 
 
 def test_calls_on_null_handle():

@@ -57,6 +57,42 @@ def test_gelu_special_values_and_odd_part():
     assert (np.abs(d - x) <= 2e-7 * x + 1e-45).all()
 
 
+def test_bf16_round_matches_torch_conversion():
+    # round to nearest even to 8 significant bits: torch's fp32 -> bf16 conversion, with ties
+    # (half an ulp exactly, odd and even kept parts) and values next to them
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(5)
+    base = rng.standard_normal(3000).astype(np.float32)
+    bits = base.view(np.uint32) & np.uint32(0xFFFF0000)
+    ties = (bits | np.uint32(0x8000)).view(np.float32)
+    x = np.concatenate([base, ties, np.nextafter(ties, np.float32(np.inf)), np.nextafter(ties, np.float32(-np.inf)),
+                        np.float32([0.0, -0.0, 1.0, 65504.0, 1e-30, -3.0e38])]).astype(np.float32)
+    want = torch.from_numpy(x).to(torch.bfloat16).to(torch.float32).numpy()
+    assert (O.bf16_round(x).view(np.uint32) == want.view(np.uint32)).all()
+
+
+def test_full_linear_row_is_the_exact_sum_rounded_once():
+    # out_o - b_o = fp32 of the exact rational sum of bf16(x_i) bf16(W_oi)
+    from fractions import Fraction
+    rng = np.random.default_rng(6)
+    K, N = 48, 7
+    x = rng.uniform(-3, 3, K).astype(np.float32)
+    W = (rng.standard_normal((N, K)) / 4).astype(np.float32)
+    b = rng.standard_normal(N).astype(np.float32)
+    s, out = O.full_linear_row(x, W, b)
+    xb, Wb = O.bf16_round(x), O.bf16_round(W).reshape(N, K)
+    assert not (xb == x).all()  # the rounding acts
+    def nearest_f32(q):  # the fp32 value nearest to the rational q, ties to even
+        c = np.float32(float(q))
+        cands = [np.nextafter(c, np.float32(-np.inf)), c, np.nextafter(c, np.float32(np.inf))]
+        return min(cands, key=lambda f: (abs(Fraction(float(f)) - q), int(np.float32(f).view(np.uint32)) & 1))
+
+    for o in range(N):
+        exact = sum(Fraction(float(xb[i])) * Fraction(float(Wb[o, i])) for i in range(K))
+        assert s[o] == nearest_f32(exact)
+        assert out[o] == np.float32(s[o] + b[o])
+
+
 def test_exp2_series_coefficients_are_taylor_terms():
     c = O.exp2_coefficients()
     for kk in range(8):
