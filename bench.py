@@ -304,7 +304,8 @@ def run_cuda(args, rank, world, local_rank):
                 frac=achieved_tops / pk["bf16_tflops"],
                 traffic=args.traffic if args.traffic is not None else
                 (measured_traffic(args.workload, B) if args.variant == "aecct" else None),
-                kernel=f"aecct_decoder_kernel<{w.d}>", work="2*12*T*d^2*N ops per word on the bf16 tensor cores "
+                kernel=f"aecct_decoder_kernel<{w.d}, {int(q['attention_mode'] == 2)}, {model.activation}, "
+                       f"{model.linear_mode}>", work="2*12*T*d^2*N ops per word on the bf16 tensor cores "
                 "(AAP: exact integers; full-precision linears: bf16 products); peak = measured bf16 dense burst")
     cpu = None
     if not args.no_cpu_baseline:
