@@ -689,7 +689,7 @@ struct Issuer {
       }
       wait(bar_full(p % S), (p / S) & 1);
       const uint32_t b_tile = sb + L::kOffW + (p % S) * W::kStageBytes;
-#pragma unroll
+#pragma unroll 1
       for (int ks = 0; ks < c.kcols / 16; ++ks) {
         const uint32_t kabs = c.k0 + 16u * ks;
         mma_bf16_warp(tmem + c.n0, make_sdesc(sb + a_tile + (kabs / 8u) * 128u, 128u, a_sbo),
@@ -836,7 +836,7 @@ struct Issuer<128, TASKS> {
     constexpr uint32_t b_sbo = (c.kcols / 8u) * 128u;
     constexpr uint32_t idesc = make_idesc_bf16(128, c.nrows);
     const uint32_t b_tile = sb + slot(P).off;
-#pragma unroll
+#pragma unroll 1
     for (int ks = 0; ks < c.kcols / 16; ++ks) {
       const uint32_t kabs = c.k0 + 16u * ks;
       mma_bf16_warp(tmem + c.n0, make_sdesc(sb + a_tile + (kabs / 8u) * 128u, 128u, a_sbo),
