@@ -557,7 +557,8 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
             float2 pr[U / 2];
 #pragma unroll
             for (int k = 0; k < U; k += 2)
-              pr[k / 2] = exp2_series2(make_float2(__fsub_rn(sgs[k0 + k], mx), __fsub_rn(sgs[k0 + k + 1], mx)));
+              // sigma - m for two keys: one paired add of -m (the cached scores are not products)
+              pr[k / 2] = exp2_series2(add2(make_float2(sgs[k0 + k], sgs[k0 + k + 1]), make_float2(-mx, -mx)));
 #pragma unroll
             for (int k = 0; k < U; k += 2) {
               if (DENSE || ((CONTIG || k0 + k < nk) && ((seg >> (k0 + k)) & 1u))) fold(pr[k / 2].x, vv[k]);
