@@ -167,3 +167,29 @@ def test_host_buffer_entry_point():
     bits, syn, logits = dec.decode_host(ch.y)
     r = O.decode(model, ch.y)
     assert_same(dict(bits=bits, syndrome=syn, logits=logits), r, "host")
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("label,make,d,layers,B", [
+    # the smallest code: 12 ten-token words per CTA, a batch that leaves a ragged last group
+    ("hamming7_4", lambda: I.make_code("hamming7_4"), 32, 2, 31),
+    # the largest token count this build takes: T = 1020 tokens over a cluster of 8 CTAs
+    ("ldpc680_340", lambda: I.ldpc_regular_code(680, 340, 3, 6, seed=680340), 32, 1, 3),
+    ("ldpc680_340-d64", lambda: I.ldpc_regular_code(680, 340, 3, 6, seed=680340), 64, 1, 2),
+])
+def test_extreme_shapes_exact(label, make, d, layers, B):
+    code = make()
+    model = I.random_model(code, d, layers, seed=17)
+    dec = A.Decoder(model)
+    q = dec.query()
+    if code.T > 896:
+        assert q["cluster_ctas"] == 8
+    ch = I.channel_batch(code, B, 3.0, seed=19)
+    g = gpu_decode(dec, ch.y, cap_B=min(B, 2))
+    r = O.decode(model, ch.y, cap_B=min(B, 2))
+    assert_same(g, r, label)
+    for name in ("q", "acc", "alpha", "syn_in"):
+        a, b = g["capture"][name], r["capture"][name]
+        assert (a.view(np.int32) if a.dtype == np.float32 else a).tolist() == \
+            (b.view(np.int32) if b.dtype == np.float32 else b).tolist(), f"{label}: {name}"
+    dec.close()
