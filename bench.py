@@ -101,6 +101,48 @@ def work_per_word(w: I.Workload):
     return dict(int_ops=2 * 12 * T * d * d * N, io_bytes=4 * w.code.n + w.code.n + (w.code.n - w.code.k))
 
 
+ALU_PEAK_TOPS = 152 * 128 * 2.070e9 / 1e12  # 152 SMs x 128 fp32 lanes x 2070 MHz (an FMA is one op), T ops/s
+
+
+def alu_ops_per_word(code, model) -> float:
+    """Algorithmic fp32 operations per decoded word of the canonical forward pass (an FMA, a
+    compare-select or a divide is one op; the integer core on the tensor cores, integer index
+    work and loads are not counted).  Per block and token, AAP linears with ReLU: Quant of a
+    K-row 4K + 2 (max |x|, floor, 127/alpha, mul + two rounding adds per code), dequant of an
+    N-row 2N + 2, residual + LayerNorm over d 8d + 3, ReLU 1 per hidden unit: 66d + 26 in all.
+    HPSA per (token, head) with kappa keys: kappa (2 d_h + 16) + d_h + 1 (pass 1: d_h FMAs, the
+    chain add, scale, max; pass 2: shift, 11 for exp2, the sum, d_h FMAs; then 1/l and d_h
+    products).  Plus the embedding products and the output head."""
+    H = code.H.astype(np.int64)
+    m, n = H.shape
+    T, d = n + m, model.d
+    dh, heads = d // 8, 8
+    F = model.ffn_mult * d
+    deg_v, deg_c = H.sum(0), H.sum(1)
+    m1 = np.concatenate([deg_v, deg_c])                       # first ring: Tanner neighbours
+    vv = (H.T @ H) > 0
+    cc = (H @ H.T) > 0
+    m2 = np.concatenate([vv.sum(1), cc.sum(1)])               # second ring, with the node itself
+    if getattr(model, "mask_mode", 0) == 1:
+        keys = heads * (m1 + m2).sum()                         # the rings are disjoint: union size = sum
+    else:
+        keys = model.h_first * m1.sum() + (heads - model.h_first) * m2.sum()
+    attn = keys * (2 * dh + 16) + T * heads * (dh + 1)
+    act = 1 if model.activation == 0 else 25                   # GELU: its erf and exp2 steps
+    if getattr(model, "linear_mode", 0) == 0:
+        quant = lambda K: 4 * K + 2                            # noqa: E731
+        deq = lambda N: 2 * N + 2                              # noqa: E731
+    else:                                                      # bf16 rounding, acc + b
+        quant = lambda K: K                                    # noqa: E731
+        deq = lambda N: N                                      # noqa: E731
+    ln = 8 * d + 3
+    per_token = (quant(d) + deq(3 * d) + 4 + quant(d) + deq(d) + ln + quant(d) + deq(F) + act * F + quant(F)
+                 + deq(d) + ln)
+    per_layer = T * per_token + attn
+    head = T * (d - model.d_spe) + T * (2 * d + 1) + n * (T + 1) + n
+    return float(model.n_layers * per_layer + head)
+
+
 class ClockSampler:
     """nvidia-smi clocks and throttle reasons during the timed region."""
 
@@ -300,13 +342,21 @@ def run_cuda(args, rank, world, local_rank):
     pk = peaks()
     wk = work_per_word(w)
     achieved_tops = wk["int_ops"] * B / kernel_s / 1e12
-    roof = dict(bound="tensor", achieved=achieved_tops, peak=pk["bf16_tflops"], unit="TFLOP/s",
-                frac=achieved_tops / pk["bf16_tflops"],
-                traffic=args.traffic if args.traffic is not None else
+    tensor = dict(bound="tensor", achieved=achieved_tops, peak=pk["bf16_tflops"], unit="TFLOP/s",
+                  frac=achieved_tops / pk["bf16_tflops"],
+                  work="2*12*T*d^2*N ops per word on the bf16 tensor cores (AAP: exact integers; "
+                       "full-precision linears: bf16 products); peak = measured bf16 dense burst")
+    alu_tops = alu_ops_per_word(w.code, model) * B / kernel_s / 1e12
+    alu = dict(bound="alu", achieved=alu_tops, peak=ALU_PEAK_TOPS, unit="TFLOP/s", frac=alu_tops / ALU_PEAK_TOPS,
+               work="algorithmic fp32 ops of the canonical forward pass per word (bench.alu_ops_per_word; an FMA "
+                    "is one op); peak = 152 SMs x 128 fp32 lanes x 2070 MHz (derived, not measured)")
+    # d <= 64: the fp32 work (HPSA, epilogues) binds; d = 128: the contraction
+    roof = dict(alu if w.d <= 64 else tensor)
+    roof.update(traffic=args.traffic if args.traffic is not None else
                 (measured_traffic(args.workload, B) if args.variant == "aecct" else None),
                 kernel=f"aecct_decoder_kernel<{w.d}, {int(q['attention_mode'] == 2)}, {model.activation}, "
-                       f"{model.linear_mode}>", work="2*12*T*d^2*N ops per word on the bf16 tensor cores "
-                "(AAP: exact integers; full-precision linears: bf16 products); peak = measured bf16 dense burst")
+                       f"{model.linear_mode}>",
+                other={k: v for k, v in (("tensor", tensor), ("alu", alu)) if v["bound"] != roof["bound"]})
     cpu = None
     if not args.no_cpu_baseline:
         rate, words, secs, cores = cpu_oracle_rate(model, ys_host[0], budget_s=args.cpu_budget)
