@@ -188,6 +188,8 @@ int aecct_synchronize(aecct_handle *h);
  *   acc_dev    int32 [cap_B][n_layers][4][T][W]  integer accumulators sum_i q_i t_oi (first N used)
  *   alpha_dev  fp32  [cap_B][n_layers][4][T]     max(absmax, alpha_floor) of the input row
  *   syn_dev    uint8 [cap_B][n-k]                syndrome s(y) of the channel output (Sec. 3)
+ * With full-precision linears (linear_mode 1) acc_dev receives the bit patterns of the fp32
+ * accumulators, and q_dev and alpha_dev are not written.
  * Any of the four may be NULL.  Unused entries are left untouched. */
 int aecct_set_capture(aecct_handle *h, int64_t cap_B, int8_t *q_dev, int32_t *acc_dev, float *alpha_dev,
                       uint8_t *syn_dev);
