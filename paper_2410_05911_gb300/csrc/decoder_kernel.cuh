@@ -203,10 +203,25 @@ __device__ __forceinline__ float round_even(float x) { return __fsub_rn(__fadd_r
 // before rounding, so the clip of RoundClip can never act and is left out.  The product stays a
 // separately rounded scalar multiply (a paired multiply feeding the rounding add would be fused).
 __device__ __forceinline__ float q_code(float v, float r) { return round_even(__fmul_rn(v, r)); }
-template <int N>
+// the codes of N values.  PAIRED: the products stay separately rounded scalar multiplies and the
+// two rounding adds of a pair of codes run as paired adds (adds of values that are not paired
+// products, so nothing is fused); the kernels whose register allocation this tips into spills
+// (d = 64, warp tasks) keep the scalar form.  Both give the same codes.
+template <int N, bool PAIRED = true>
 __device__ __forceinline__ void codes(const float *v, float r, float *q) {
+  if constexpr (PAIRED) {
+    static_assert(N % 2 == 0, "pairs");
 #pragma unroll
-  for (int j = 0; j < N; ++j) q[j] = q_code(v[j], r);
+    for (int j = 0; j < N; j += 2) {
+      const float2 t = add2(make_float2(__fmul_rn(v[j], r), __fmul_rn(v[j + 1], r)),
+                            make_float2(kRoundMagic, kRoundMagic));
+      const float2 c = add2(t, make_float2(-kRoundMagic, -kRoundMagic));
+      q[j] = c.x, q[j + 1] = c.y;
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < N; ++j) q[j] = q_code(v[j], r);
+  }
 }
 __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
   // a, b are integers in [-127, 127]: their fp32 encodings have 16 zero low bits, so the bf16
@@ -945,6 +960,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   using LP = LayerParamLayout;
   constexpr int DH = D / kHeads;  // head width
   constexpr int XS = D / 4;       // x columns per thread
+  constexpr bool kPairCodes = !(D == 64 && TASKS);  // paired rounding adds (see codes)
   constexpr int S = L::kStages;
   extern __shared__ __align__(1024) uint8_t smem[];
   const uint32_t sb = smem_u32(smem);
@@ -1180,7 +1196,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         alpha_in = a;
         const float rr = __fdiv_rn(127.0f, a);
         float qv[XS];
-        codes<XS>(x, rr, qv);
+        codes<XS, kPairCodes>(x, rr, qv);
         store_codes<XS>(aop, r, sl * XS, D, qv);
         return rr;
       };
@@ -1230,7 +1246,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         const float rr = quant_x_to_aop();
         if (cap) {
           float qv[XS];
-          codes<XS>(x, rr, qv);
+          codes<XS, kPairCodes>(x, rr, qv);
           capture_q(0, 0, qv, sl * XS, XS, alpha_in);
         }
       }
@@ -1345,7 +1361,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             alpha_in = a;
             const float rr = __fdiv_rn(127.0f, a);
             float qv[XS];
-            codes<XS>(av, rr, qv);
+            codes<XS, kPairCodes>(av, rr, qv);
             store_codes<XS>(aop, r, sl * XS, D, qv);
             if (cap) capture_q(l, 1, qv, sl * XS, XS, alpha_in);
           }
@@ -1425,7 +1441,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           const float rr = quant_x_to_aop();
           if (cap) {
             float qv[XS];
-            codes<XS>(x, rr, qv);
+            codes<XS, kPairCodes>(x, rr, qv);
             capture_q(l, 2, qv, sl * XS, XS, alpha_in);
           }
         }
@@ -1492,7 +1508,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
                 hidden(c0, u, false);
               }
               float qv[32];
-              codes<32>(u, rr, qv);
+              codes<32, kPairCodes>(u, rr, qv);
               store_codes<32>(uqt, r, c0, 4 * D, qv);
               if (cap) capture_q(l, 3, qv, c0, 32, alpha_in);
             }
@@ -1514,7 +1530,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           const float rr = quant_x_to_aop();
           if (cap) {
             float qv[XS];
-            codes<XS>(x, rr, qv);
+            codes<XS, kPairCodes>(x, rr, qv);
             capture_q(l + 1, 0, qv, sl * XS, XS, alpha_in);
           }
           signal_op(0, l + 1, gi);
