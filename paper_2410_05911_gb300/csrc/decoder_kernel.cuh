@@ -1453,8 +1453,8 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           const float f1 = dq_factor(sw + 4);
           // ACT 0 = ReLU, 1 = GELU.  u = act(acc f1 + b1) in 32-column chunks of this thread's D
           // hidden columns.  AAP: with ReLU at d <= 64 u stays in registers between the row
-          // maximum and the codes, otherwise the second pass recomputes it (same operations, same
-          // values).  Full-precision linears: one pass, u rounded to bf16.
+          // maximum and the codes; otherwise it is stored over its own accumulators in TMEM and
+          // read back for the codes.  Full-precision linears: one pass, u rounded to bf16.
           constexpr int NCH = D / 32;
           constexpr bool KEEP = D <= 64 && ACT == 0;
           auto hidden = [&](int c0, float *u, bool capture) {
@@ -1490,7 +1490,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
                 umax = fmaxf(umax, fabsf(u[j]));
                 if constexpr (KEEP) uk[32 * ch + j] = u[j];
               }
+              // otherwise u replaces its own accumulators in TMEM (this thread's lane and columns)
+              if constexpr (!KEEP) tmem_st<32>(tl + c0, u);
             }
+            if constexpr (!KEEP) tmem_wait_st();
             float a = word_alpha(row_max(umax));
             a = (a > p.alpha_floor) ? a : p.alpha_floor;
             alpha_in = a;
@@ -1505,7 +1508,8 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
 #pragma unroll
                 for (int j = 0; j < 32; ++j) u[j] = uk[32 * ch + j];
               } else {
-                hidden(c0, u, false);
+                tmem_ld<32>(tl + c0, u);
+                tmem_wait_ld();
               }
               float qv[32];
               codes<32, kPairCodes>(u, rr, qv);
