@@ -203,24 +203,18 @@ __device__ __forceinline__ float round_even(float x) { return __fsub_rn(__fadd_r
 // before rounding, so the clip of RoundClip can never act and is left out.  The product stays a
 // separately rounded scalar multiply (a paired multiply feeding the rounding add would be fused).
 __device__ __forceinline__ float q_code(float v, float r) { return round_even(__fmul_rn(v, r)); }
-// the codes of N values.  PAIRED: the products stay separately rounded scalar multiplies and the
-// two rounding adds of a pair of codes run as paired adds (adds of values that are not paired
-// products, so nothing is fused); the kernels whose register allocation this tips into spills
-// (d = 64, warp tasks) keep the scalar form.  Both give the same codes.
-template <int N, bool PAIRED = true>
+// the codes of N values (N even): the products stay separately rounded scalar multiplies, and
+// the two rounding adds of a pair of codes run as paired adds (adds of values that are not paired
+// products, so nothing is fused); the same codes as q_code
+template <int N>
 __device__ __forceinline__ void codes(const float *v, float r, float *q) {
-  if constexpr (PAIRED) {
-    static_assert(N % 2 == 0, "pairs");
+  static_assert(N % 2 == 0, "pairs");
 #pragma unroll
-    for (int j = 0; j < N; j += 2) {
-      const float2 t = add2(make_float2(__fmul_rn(v[j], r), __fmul_rn(v[j + 1], r)),
-                            make_float2(kRoundMagic, kRoundMagic));
-      const float2 c = add2(t, make_float2(-kRoundMagic, -kRoundMagic));
-      q[j] = c.x, q[j + 1] = c.y;
-    }
-  } else {
-#pragma unroll
-    for (int j = 0; j < N; ++j) q[j] = q_code(v[j], r);
+  for (int j = 0; j < N; j += 2) {
+    const float2 t = add2(make_float2(__fmul_rn(v[j], r), __fmul_rn(v[j + 1], r)),
+                          make_float2(kRoundMagic, kRoundMagic));
+    const float2 c = add2(t, make_float2(-kRoundMagic, -kRoundMagic));
+    q[j] = c.x, q[j + 1] = c.y;
   }
 }
 __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
@@ -960,7 +954,6 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   using LP = LayerParamLayout;
   constexpr int DH = D / kHeads;  // head width
   constexpr int XS = D / 4;       // x columns per thread
-  constexpr bool kPairCodes = !(D == 64 && TASKS);  // paired rounding adds (see codes)
   constexpr int S = L::kStages;
   extern __shared__ __align__(1024) uint8_t smem[];
   const uint32_t sb = smem_u32(smem);
@@ -1196,7 +1189,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         alpha_in = a;
         const float rr = __fdiv_rn(127.0f, a);
         float qv[XS];
-        codes<XS, kPairCodes>(x, rr, qv);
+        codes<XS>(x, rr, qv);
         store_codes<XS>(aop, r, sl * XS, D, qv);
         return rr;
       };
@@ -1246,7 +1239,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         const float rr = quant_x_to_aop();
         if (cap) {
           float qv[XS];
-          codes<XS, kPairCodes>(x, rr, qv);
+          codes<XS>(x, rr, qv);
           capture_q(0, 0, qv, sl * XS, XS, alpha_in);
         }
       }
@@ -1361,7 +1354,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             alpha_in = a;
             const float rr = __fdiv_rn(127.0f, a);
             float qv[XS];
-            codes<XS, kPairCodes>(av, rr, qv);
+            codes<XS>(av, rr, qv);
             store_codes<XS>(aop, r, sl * XS, D, qv);
             if (cap) capture_q(l, 1, qv, sl * XS, XS, alpha_in);
           }
@@ -1441,7 +1434,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           const float rr = quant_x_to_aop();
           if (cap) {
             float qv[XS];
-            codes<XS, kPairCodes>(x, rr, qv);
+            codes<XS>(x, rr, qv);
             capture_q(l, 2, qv, sl * XS, XS, alpha_in);
           }
         }
@@ -1452,11 +1445,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         {
           const float f1 = dq_factor(sw + 4);
           // ACT 0 = ReLU, 1 = GELU.  u = act(acc f1 + b1) in 32-column chunks of this thread's D
-          // hidden columns.  AAP: with ReLU at d <= 64 u stays in registers between the row
-          // maximum and the codes; otherwise it is stored over its own accumulators in TMEM and
-          // read back for the codes.  Full-precision linears: one pass, u rounded to bf16.
+          // hidden columns.  AAP: u is stored over its own accumulators in TMEM (this thread's
+          // lane and columns) between the row maximum and the codes, which leaves the registers
+          // to the rest of the kernel.  Full-precision linears: one pass, u rounded to bf16.
           constexpr int NCH = D / 32;
-          constexpr bool KEEP = D <= 64 && ACT == 0;
           auto hidden = [&](int c0, float *u, bool capture) {
             float ac[32], bb[32];
             tmem_ld<32>(tl + c0, ac);
@@ -1478,7 +1470,6 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
               store_bf16<32>(uqt, r, c0, 4 * D, u);
             }
           } else {
-            float uk[KEEP ? D : 1];
             float umax = 0.0f;
 #pragma unroll
             for (int ch = 0; ch < NCH; ++ch) {
@@ -1486,14 +1477,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
               float u[32];
               hidden(c0, u, cap);
 #pragma unroll
-              for (int j = 0; j < 32; ++j) {
-                umax = fmaxf(umax, fabsf(u[j]));
-                if constexpr (KEEP) uk[32 * ch + j] = u[j];
-              }
-              // otherwise u replaces its own accumulators in TMEM (this thread's lane and columns)
-              if constexpr (!KEEP) tmem_st<32>(tl + c0, u);
+              for (int j = 0; j < 32; ++j) umax = fmaxf(umax, fabsf(u[j]));
+              tmem_st<32>(tl + c0, u);
             }
-            if constexpr (!KEEP) tmem_wait_st();
+            tmem_wait_st();
             float a = word_alpha(row_max(umax));
             a = (a > p.alpha_floor) ? a : p.alpha_floor;
             alpha_in = a;
@@ -1504,15 +1491,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             for (int ch = 0; ch < NCH; ++ch) {
               const int c0 = sl * D + 32 * ch;
               float u[32];
-              if constexpr (KEEP) {
-#pragma unroll
-                for (int j = 0; j < 32; ++j) u[j] = uk[32 * ch + j];
-              } else {
-                tmem_ld<32>(tl + c0, u);
-                tmem_wait_ld();
-              }
+              tmem_ld<32>(tl + c0, u);
+              tmem_wait_ld();
               float qv[32];
-              codes<32, kPairCodes>(u, rr, qv);
+              codes<32>(u, rr, qv);
               store_codes<32>(uqt, r, c0, 4 * D, qv);
               if (cap) capture_q(l, 3, qv, c0, 32, alpha_in);
             }
@@ -1534,7 +1516,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           const float rr = quant_x_to_aop();
           if (cap) {
             float qv[XS];
-            codes<XS, kPairCodes>(x, rr, qv);
+            codes<XS>(x, rr, qv);
             capture_q(l + 1, 0, qv, sl * XS, XS, alpha_in);
           }
           signal_op(0, l + 1, gi);
