@@ -126,11 +126,17 @@ __device__ __forceinline__ float2 exp2_series2(float2 x) {
   return make_float2(r0, r1);
 }
 
-// out[j] = acc[j] * f + b[j]  (eq. AAPLinear dequantisation, f = gamma*delta*alpha/Q_b)
+// out[j] = acc[j] * f + b[j]  (eq. AAPLinear dequantisation, f = gamma*delta*alpha/Q_b): a
+// separately rounded product, then the bias add; the adds of two outputs run as one paired add
+// (the products stay scalar multiplies, so nothing is fused)
 template <int N>
 __device__ __forceinline__ void dequant(const float *acc, float f, const float *b, float *out) {
+  static_assert(N % 2 == 0, "pairs");
 #pragma unroll
-  for (int j = 0; j < N; ++j) out[j] = __fadd_rn(__fmul_rn(acc[j], f), b[j]);
+  for (int j = 0; j < N; j += 2) {
+    const float2 o = add2(make_float2(__fmul_rn(acc[j], f), __fmul_rn(acc[j + 1], f)), make_float2(b[j], b[j + 1]));
+    out[j] = o.x, out[j + 1] = o.y;
+  }
 }
 
 template <int N>
