@@ -1369,11 +1369,16 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           cluster_wait(bar_kvr, kvr_ph);
   
           // ---------------- S5: HPSA (Sec. 4.2)
-          float A[2][DH];
+          // the A of each head goes over the head's Q in TMEM (this thread's lane; that Q has no
+          // other reader), so that the second head's attention runs with the registers of one;
+          // d = 32 (d_h = 4, below the TMEM store width) keeps both in registers
+          constexpr bool kStashA = DH >= 8;
+          float A[kStashA ? 1 : 2][DH];
           float amax = 0.0f;
   #pragma unroll
           for (int hh = 0; hh < 2; ++hh) {
             const int e = sl + 4 * hh;
+            float *Ah = A[kStashA ? 0 : hh];
             float qa[DH], bq[DH];
             tmem_ld<DH>(tl + e * DH, qa);
             tmem_wait_ld();
@@ -1383,7 +1388,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   #pragma unroll
             for (int i = 0; i < DH; ++i) q[i] = __fadd_rn(__fmul_rn(qa[i], fq), bq[i]);
   #pragma unroll
-            for (int i = 0; i < DH; ++i) A[hh][i] = 0.0f;
+            for (int i = 0; i < DH; ++i) Ah[i] = 0.0f;
             {
               const int mk = (e < p.h_first) ? 0 : 1;
               constexpr int U = (DH >= 16) ? 2 : 4;
@@ -1392,18 +1397,34 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
               const uint32_t info = row_cw ? __ldg(p.mask_info[mk] + t) : 0u;
               if (p.C == 1)
                 hpsa_head<DH, U, L::kKvStride, false>(q, info, row_cw, p.mask_list[mk], smem + L::kOffU, s_kvcl,
-                                                      g * T, e * (8 * DH), p.att_scale, tcache, A[hh]);
+                                                      g * T, e * (8 * DH), p.att_scale, tcache, Ah);
               else
                 hpsa_head<DH, U, L::kKvStride, true>(q, info, row_cw, p.mask_list[mk], smem + L::kOffU, s_kvcl,
-                                                     g * T, e * (8 * DH), p.att_scale, tcache, A[hh]);
+                                                     g * T, e * (8 * DH), p.att_scale, tcache, Ah);
             }
   #pragma unroll
-            for (int i = 0; i < DH; ++i) amax = fmaxf(amax, fabsf(A[hh][i]));
+            for (int i = 0; i < DH; ++i) amax = fmaxf(amax, fabsf(Ah[i]));
+            if constexpr (kStashA) tmem_st<DH>(tl + e * DH, Ah);
           }
+          if constexpr (kStashA) tmem_wait_st();
+          // A of head sl + 4 hh, from TMEM or registers
+          auto head_a = [&](int hh, float *out) {
+            if constexpr (kStashA) {
+              tmem_ld<DH>(tl + (sl + 4 * hh) * DH, out);
+              tmem_wait_ld();
+            } else {
+#pragma unroll
+              for (int i = 0; i < DH; ++i) out[i] = A[hh][i];
+            }
+          };
           // Quant(A) -> O operand
           if constexpr (LIN == 1) {
 #pragma unroll
-            for (int hh = 0; hh < 2; ++hh) store_bf16<DH>(aop, r, (sl + 4 * hh) * DH, D, A[hh]);
+            for (int hh = 0; hh < 2; ++hh) {
+              float ah[DH];
+              head_a(hh, ah);
+              store_bf16<DH>(aop, r, (sl + 4 * hh) * DH, D, ah);
+            }
           } else {
             float a = word_alpha(row_max(amax));
             a = (a > p.alpha_floor) ? a : p.alpha_floor;
@@ -1412,9 +1433,9 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   #pragma unroll
             for (int hh = 0; hh < 2; ++hh) {
               const int e = sl + 4 * hh;
-              float qv[DH];
-  #pragma unroll
-              for (int i = 0; i < DH; ++i) qv[i] = q_code(A[hh][i], rr);
+              float ah[DH], qv[DH];
+              head_a(hh, ah);
+              codes<DH>(ah, rr, qv);
               store_codes<DH>(aop, r, e * DH, D, qv);
               if (cap) capture_q(l, 1, qv, e * DH, DH, alpha_in);
             }
