@@ -51,11 +51,27 @@ struct WeightSchedule {
     return f;
   }
   static constexpr int kCPL = first(4);  // chunks per block
+  // N tile and K tile of chunk j of GEMM g.  N tiles go in pairs, a pair's two chunks of one K
+  // range adjacent (two 128-row tiles form one 256-row operand for an N = 256 MMA); an odd last N
+  // tile follows with its K tiles in order.
+  __host__ __device__ static constexpr int tile_of(int g, int j, bool want_n) {
+    const int nt = (gemm_n(g) + tile_n(g) - 1) / tile_n(g), kt = gemm_k(g) / tile_k(g);
+    const int paired = (nt / 2) * 2 * kt;
+    int n = 0, k = 0;
+    if (j < paired) {
+      n = 2 * (j / (2 * kt)) + (j % 2);
+      k = (j % (2 * kt)) / 2;
+    } else {
+      n = nt - 1;
+      k = j - paired;
+    }
+    return want_n ? n : k;
+  }
   __host__ __device__ static constexpr ChunkDesc chunk(int p) {
     int g = 0;
     while (g < 3 && p >= first(g + 1)) ++g;
-    const int j = p - first(g), kt = gemm_k(g) / tile_k(g);
-    const int n0 = (j / kt) * tile_n(g), k0 = (j % kt) * tile_k(g);
+    const int j = p - first(g);
+    const int n0 = tile_of(g, j, true) * tile_n(g), k0 = tile_of(g, j, false) * tile_k(g);
     const int nrows = (gemm_n(g) - n0) < tile_n(g) ? (gemm_n(g) - n0) : tile_n(g);
     uint32_t off = 0;
     for (int q = 0; q < p; ++q) off += chunk_bytes(q);
@@ -64,8 +80,8 @@ struct WeightSchedule {
   __host__ __device__ static constexpr uint32_t chunk_bytes(int p) {
     int g = 0;
     while (g < 3 && p >= first(g + 1)) ++g;
-    const int j = p - first(g), kt = gemm_k(g) / tile_k(g);
-    const int n0 = (j / kt) * tile_n(g);
+    const int j = p - first(g);
+    const int n0 = tile_of(g, j, true) * tile_n(g);
     const int nrows = (gemm_n(g) - n0) < tile_n(g) ? (gemm_n(g) - n0) : tile_n(g);
     return static_cast<uint32_t>(nrows * tile_k(g) * 2);
   }

@@ -859,11 +859,25 @@ struct Issuer<128, TASKS> {
                     make_sdesc(b_tile + ks * 256u, 128u, b_sbo), idesc, kabs > 0 ? 1u : 0u);
     }
   }
-  template <int G, int P0, int P1>
-  __device__ __forceinline__ void mmas_range() const {
-    if constexpr (P0 < P1) {
-      mmas<G, P0>();
-      mmas_range<G, P0 + 1, P1>();
+  // the MMAs of chunks P and P + 1, two 128-row N tiles of one K range that sit next to each other
+  // in shared memory, as N = 256 MMAs (the tensor pipe runs an N = 256 MMA at close to its peak,
+  // two N = 128 ones at about 60% of it)
+  template <int G, int P>
+  __device__ __forceinline__ void mmas_pair() const {
+    constexpr ChunkDesc c = W::chunk(P), c2 = W::chunk(P + 1);
+    static_assert(c.nrows == 128 && c2.nrows == 128 && c2.n0 == c.n0 + 128 && c2.k0 == c.k0 &&
+                      c2.kcols == c.kcols && slot(P + 1).off == slot(P).off + kChunk,
+                  "an N-tile pair: adjacent tiles of one K range");
+    constexpr uint32_t a_tile = (G == 3) ? L::kOffU : L::kOffAop;
+    constexpr uint32_t a_sbo = (G == 3) ? (4u * D / 8u) * 128u : (D / 8u) * 128u;
+    constexpr uint32_t b_sbo = (c.kcols / 8u) * 128u;  // row groups 16..31 continue in chunk P + 1
+    constexpr uint32_t idesc = make_idesc_bf16(128, 256);
+    const uint32_t b_tile = sb + slot(P).off;
+#pragma unroll 1
+    for (int ks = 0; ks < c.kcols / 16; ++ks) {
+      const uint32_t kabs = c.k0 + 16u * ks;
+      mma_bf16_warp(tmem + c.n0, make_sdesc(sb + a_tile + (kabs / 8u) * 128u, 128u, a_sbo),
+                    make_sdesc(b_tile + ks * 256u, 128u, b_sbo), idesc, kabs > 0 ? 1u : 0u);
     }
   }
 
@@ -875,7 +889,10 @@ struct Issuer<128, TASKS> {
     tc_fence_after();
     if constexpr (G == 0) {
       wait(bar(3), 0);  // QKV weights in region U
-      mmas_range<0, 0, 6>();
+      mmas_pair<0, 0>();  // N tiles 0 and 1, K 0..63
+      mmas_pair<0, 2>();  // N tiles 0 and 1, K 64..127
+      mmas<0, 4>();       // N tile 2
+      mmas<0, 5>();
       mma_commit_warp(bar_acc());
       wait(bar_acc(), 0);
     } else if constexpr (G == 1) {
@@ -903,7 +920,10 @@ struct Issuer<128, TASKS> {
         copies<8, 16>(w_cur);
       }
       wait(bar(3), 1);  // FFN1 weights in region U
-      mmas_range<2, 8, 16>();
+      mmas_pair<2, 8>();
+      mmas_pair<2, 10>();
+      mmas_pair<2, 12>();
+      mmas_pair<2, 14>();
       mma_commit_warp(bar_acc());
       wait(bar_acc(), 0);
       copy1<19>(w_cur);  // the operand tile is free: FFN1's MMAs are done
