@@ -1,6 +1,7 @@
 // decoder_kernel.cuh -- the fused AECCT forward pass for sm_103a (kernel template; its
-// instantiations live in decoder_kernel.cu (ReLU) and decoder_kernel_gelu.cu (GELU), two
-// translation units that compile in parallel).
+// instantiations live in decoder_kernel.cu (ReLU, AAP linears), decoder_kernel_gelu.cu (GELU),
+// decoder_kernel_fp.cu and decoder_kernel_fp_gelu.cu (full-precision bf16 linears), translation
+// units that compile in parallel).
 //
 // One persistent kernel decodes the whole batch.  A cluster of C CTAs owns a group of G
 // codewords whose T = 2n-k tokens are packed back to back over the cluster's C x 128 token
@@ -11,7 +12,8 @@
 //   S3-S8  (Sec. 4.1, 4.2, 5) per block:
 //          Quant(x) -> tcgen05.mma QKV (bf16 operands holding exact int8 / ternary values,
 //          fp32 accumulators in TMEM, exact integers) -> dequant -> K,V to shared memory
-//          -> HPSA over CSR neighbour lists (DSMEM reads of peer CTAs) -> Quant(A) -> MMA O
+//          -> HPSA (warp tasks over shared key lists, or per-row neighbour lists with
+//          distributed-shared-memory reads of peer CTAs) -> Quant(A) -> MMA O
 //          -> dequant + residual + LayerNorm -> Quant -> MMA FFN1 -> dequant + ReLU/GELU ->
 //          Quant -> MMA FFN2 -> dequant + residual + LayerNorm
 //   S9/S10 (Sec. 3)        output head, hard decisions, syndrome of the decoded word
