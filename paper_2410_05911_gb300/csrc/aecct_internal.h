@@ -118,6 +118,8 @@ struct LayerParamLayout {
 struct DecodeParams {
   // problem shape
   int n, k, T, m, n_layers, h_first, d_spe;
+  int Tp;          // token rows per codeword: T, or more when the rows of each node type start on a
+                   // 32-row boundary (d = 128 warp tasks); a padding row holds no token (perm 0xFFFF)
   int C;           // CTAs per cluster (they share one group of codewords)
   int G;           // codewords per group
   int n_clusters;  // clusters launched
@@ -139,7 +141,7 @@ struct DecodeParams {
   const float *b_out;    // [n]
   const uint32_t *hbits;  // [m][hwords] row i of H as a bitmask over the variables (bit j%32 of word j/32)
   int hwords;             // ceil(n / 32)
-  const uint16_t *perm;         // [T] row offset within a codeword -> token
+  const uint16_t *perm;         // [Tp] row offset within a codeword -> token (0xFFFF: padding row)
   const uint16_t *pos;          // [T] token -> row offset within its codeword
   // HPSA neighbour lists, 0 = first ring, 1 = second ring.  mask_info[mk][t] = (start << 11) | count:
   // the count row offsets of token t's neighbours (ascending token order) begin at mask_list[mk][start]
@@ -175,11 +177,13 @@ __host__ __device__ constexpr inline uint32_t core_off(uint32_t r, uint32_t c, u
 }
 
 // Shared-memory map.  Region U holds, per block, first the attention operands and then the FFN2
-// operand.  Row mode: per token row 8 heads x (K | V) x d_h fp32.  Task mode: 8 heads x
-// (Q | K | V) x d_h fp32; the attention output of a (row, head) then replaces its Q.
+// operand.  Row mode, and task mode at d = 128: per token row 8 heads x (K | V) x d_h fp32 (Q and
+// the attention output stay in TMEM).  Task mode at d <= 64: 8 heads x (Q | K | V) x d_h fp32;
+// the attention output of a (row, head) then replaces its Q.
 template <int D, bool TASKS = false>
 struct SmemLayout {
-  static constexpr uint32_t kSlot = (TASKS ? 12u : 8u) * (D / 8u);  // bytes of one head of one row
+  static constexpr bool kQInSmem = TASKS && D != 128;
+  static constexpr uint32_t kSlot = (kQInSmem ? 12u : 8u) * (D / 8u);  // bytes of one head of one row
   static constexpr uint32_t kKvStride = 8u * kSlot + 16u;            // token row, + 16 B pad
   static constexpr uint32_t kKvBytes = kRows * kKvStride;
   static constexpr uint32_t kUqBytes = kRows * 4u * D * 2u;  // FFN2 operand: 128 x 4D bf16
@@ -199,12 +203,13 @@ struct SmemLayout {
   static constexpr uint32_t kOffMisc = kOffBar + 256;  // tmem base, abort flag, peer bases, copy count
   static constexpr uint32_t kTotal = kOffMisc + 256;
   // QKV / FFN1 accumulators in [0, 4D) (x parked in [3D, 4D) during attention).  Attention
-  // scores are cached in TMEM between the two softmax passes: task mode in [kTaskCacheCol, 512)
-  // (4 warps per lane quadrant x kTaskCache columns); row mode kRowCache columns per column slice
-  // from kRowCacheCol, each thread in its own row's lane (d = 128: the K and V accumulator
-  // columns [128, 384), dead once K and V are in shared memory; d <= 64: [256, 512)).
+  // scores are cached in TMEM between the two softmax passes: task mode from kTaskCacheCol
+  // (4 warps per lane quadrant x kTaskCache columns: [256, 512) for d <= 64, the dead K and V
+  // accumulator columns [128, 384) for d = 128); row mode kRowCache columns per column slice
+  // from kRowCacheCol, each thread in its own row's lane (d = 128: [128, 384); d <= 64:
+  // [256, 512)).
   static constexpr uint32_t kTmemCols = 512u;
-  static constexpr uint32_t kTaskCacheCol = 256u;
+  static constexpr uint32_t kTaskCacheCol = (D == 128) ? 128u : 256u;
   static constexpr uint32_t kRowCacheCol = (D == 128) ? 128u : 256u;
 };
 

@@ -31,6 +31,7 @@ int cuda_fail(cudaError_t e, const char *what) {
 
 struct aecct_handle {
   int n = 0, k = 0, T = 0, m = 0, d = 0, n_layers = 0, h_first = 0, d_spe = 0;
+  int Tp = 0;  // token rows per codeword (T, or T plus padding rows)
   int C = 1, G = 1, max_clusters = 0;
   bool tasks = false;  // warp-task attention (one CTA per group, d <= 64)
   int alpha_mode = 0;  // 1 = one alpha per quantised matrix of a word
@@ -194,12 +195,13 @@ int schedule_chunks(int D, ChunkDesc *out) {
   return D == 32 ? schedule_chunks_t<32>(out) : D == 64 ? schedule_chunks_t<64>(out) : schedule_chunks_t<128>(out);
 }
 
-// the compiled kernel for (d, attention mode, activation ACT, linear mode LIN): task mode exists
-// for d = 32 and 64
+// the compiled kernel for (d, attention mode, activation ACT, linear mode LIN)
 template <int ACT, int LIN>
 cudaError_t prepare_any(int D, bool tasks, int C, int *max_clusters) {
-  if (tasks) return D == 32 ? prepare_decode_kernel<32, true, ACT, LIN>(C, max_clusters)
-                            : prepare_decode_kernel<64, true, ACT, LIN>(C, max_clusters);
+  if (tasks)
+    return D == 32   ? prepare_decode_kernel<32, true, ACT, LIN>(C, max_clusters)
+           : D == 64 ? prepare_decode_kernel<64, true, ACT, LIN>(C, max_clusters)
+                     : prepare_decode_kernel<128, true, ACT, LIN>(C, max_clusters);
   if (D == 32) return prepare_decode_kernel<32, false, ACT, LIN>(C, max_clusters);
   if (D == 64) return prepare_decode_kernel<64, false, ACT, LIN>(C, max_clusters);
   return prepare_decode_kernel<128, false, ACT, LIN>(C, max_clusters);
@@ -207,7 +209,9 @@ cudaError_t prepare_any(int D, bool tasks, int C, int *max_clusters) {
 template <int ACT, int LIN>
 cudaError_t launch_any(int D, bool tasks, const DecodeParams &p, cudaStream_t stream) {
   if (tasks)
-    return D == 32 ? launch_decode<32, true, ACT, LIN>(p, stream) : launch_decode<64, true, ACT, LIN>(p, stream);
+    return D == 32   ? launch_decode<32, true, ACT, LIN>(p, stream)
+           : D == 64 ? launch_decode<64, true, ACT, LIN>(p, stream)
+                     : launch_decode<128, true, ACT, LIN>(p, stream);
   if (D == 32) return launch_decode<32, false, ACT, LIN>(p, stream);
   if (D == 64) return launch_decode<64, false, ACT, LIN>(p, stream);
   return launch_decode<128, false, ACT, LIN>(p, stream);
@@ -248,70 +252,6 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
   const aecct_model_desc &d = *desc;
   const int n = d.n, k = d.k, m = n - k, T = 2 * n - k, D = d.d, F = 4 * D;
 
-  // Attention mode.  Task mode keeps every codeword inside one CTA (no cluster): it needs T <= 128,
-  // d <= 64 (shared memory for Q, K, V and A), and at most kMaxGroups 32-row query groups.
-  const int g1 = kRows / T;
-  const bool task_ok = T <= kRows && D <= 64 && g1 >= 1 && g1 * ((T + 31) / 32) <= kMaxGroups &&
-                       g1 * n <= kOutBitsBytes && (d.cluster_ctas == 0 || d.cluster_ctas == 1);
-  bool tasks = false;
-  if (d.attention_mode == 2) {
-    if (!task_ok) return AECCT_ERR_UNSUPPORTED;
-    tasks = true;
-  } else if (d.attention_mode == 0) {
-    tasks = task_ok;
-  }
-  // choose the number of CTAs that share a group: by default the fewest that hold one codeword
-  // (an attention read of a key held by another CTA of the cluster costs far more than the
-  // token rows left idle by a looser packing), with as many words per group as fit; an explicit
-  // cluster_ctas is honoured when it can hold a word
-  int best_C = 0, best_G = 0;
-  const int cmin = (T + kRows - 1) / kRows;
-  for (int C = cmin; C <= kMaxCluster && !best_C; ++C) {
-    if (tasks && C != 1) continue;
-    if (d.cluster_ctas && C != d.cluster_ctas) continue;
-    const int G = (C * kRows) / T;
-    if (G < 1) continue;
-    if (((G + C - 1) / C) * n > kOutBitsBytes) continue;
-    best_C = C, best_G = G;
-  }
-  if (!best_C) return d.cluster_ctas ? AECCT_ERR_INVALID_ARG : AECCT_ERR_UNSUPPORTED;
-  if (best_G * ((n + 31) / 32) > 128) return AECCT_ERR_UNSUPPORTED;  // hard-decision bitmasks of a group
-  if (d.alpha_mode == 1 && best_C != 1) return AECCT_ERR_UNSUPPORTED;  // per-word alpha: one CTA per word
-
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return AECCT_ERR_NO_DEVICE;
-  cudaDeviceProp prop;
-  e = cudaGetDeviceProperties(&prop, dev);
-  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDeviceProperties");
-  if (prop.major != 10) {
-    g_last_error = "device is not compute capability 10.x";
-    return AECCT_ERR_NO_DEVICE;
-  }
-  int max_clusters = 0;
-  e = prepare_variant(d.activation, d.linear_mode, D, tasks, best_C, &max_clusters);
-  if (e != cudaSuccess) return cuda_fail(e, "kernel occupancy");
-  if (max_clusters < 1) {
-    g_last_error = "no cluster of this size fits on the device";
-    return AECCT_ERR_UNSUPPORTED;
-  }
-
-  aecct_handle *h = new aecct_handle();
-  h->n = n, h->k = k, h->T = T, h->m = m, h->d = D, h->n_layers = d.n_layers, h->h_first = d.h_first;
-  h->d_spe = d.d_spe, h->C = best_C, h->G = best_G, h->max_clusters = max_clusters, h->tasks = tasks;
-  h->ln_eps = d.ln_eps, h->alpha_floor = d.alpha_floor, h->b_d1 = d.b_d1, h->device = dev;
-  h->alpha_mode = d.alpha_mode;
-  h->activation = d.activation;
-  h->linear_mode = d.linear_mode;
-  h->att_scale = static_cast<float>(1.4426950408889634074 / std::sqrt(static_cast<double>(D / kHeads)));
-  h->wait_limit = d.wait_limit_cycles ? d.wait_limit_cycles : (1LL << 32);
-
-  // ---- H rows as bitmasks over the variables, for the syndromes (parity of popcounts)
-  h->hwords = (n + 31) / 32;
-  std::vector<uint32_t> hbits((size_t)m * h->hwords, 0u);
-  for (int i = 0; i < m; ++i)
-    for (int j = 0; j < n; ++j)
-      if (d.H[(size_t)i * n + j]) hbits[(size_t)i * h->hwords + j / 32] |= 1u << (j % 32);
   // ---- HPSA neighbour lists (Sec. 4.2): token t < n is variable t, token n + i is check i.
   // First ring: Tanner-graph neighbours.  Second ring: same-type nodes at distance two, and the
   // node itself.  Lists are in ascending token order (the order the softmax sums run in).
@@ -358,10 +298,110 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
       nb[1][t] = u;
     }
   }
+
+  // Attention mode.  Task mode keeps every codeword inside one CTA (no cluster).  d <= 64: Q, K, V
+  // and A in shared memory, T <= 128, at most kMaxGroups 32-row query groups.  d = 128: Q and A in
+  // TMEM, one codeword per CTA whose variables start at row 0 and whose checks start on the next
+  // 32-row boundary, so that every query group is one TMEM lane quadrant (Tp = that padded row
+  // count <= 128), one alpha per row.  By default d = 128 takes task mode only when the query
+  // groups' shared key lists are dense enough that walking their unions beats walking each
+  // row's own list.
+  const int g1 = kRows / T;
+  const int npad = ((n + 31) / 32) * 32, Tp128 = npad + m;
+  const bool one_cta = d.cluster_ctas == 0 || d.cluster_ctas == 1;
+  const bool task_ok =
+      D <= 64 ? (T <= kRows && g1 >= 1 && g1 * ((T + 31) / 32) <= kMaxGroups && g1 * n <= kOutBitsBytes && one_cta)
+              : (Tp128 <= kRows && d.alpha_mode == 0 && n <= kOutBitsBytes && one_cta);
+  bool tasks = false;
+  if (d.attention_mode == 2) {
+    if (!task_ok) return AECCT_ERR_UNSUPPORTED;
+    tasks = true;
+  } else if (d.attention_mode == 0) {
+    tasks = task_ok;
+    if (tasks && D == 128) {
+      // share of the lane-key iterations of the task walks that fall on a lane's own keys
+      double useful = 0.0, walked = 0.0;
+      const int hr[2] = {d.h_first, d.heads - d.h_first};
+      for (int r = 0; r < 2; ++r) {
+        for (int t = 0; t < T; ++t) useful += hr[r] * static_cast<double>(nb[r][t].size());
+        for (int type = 0; type < 2; ++type) {
+          const int t0 = type == 0 ? 0 : n, t1 = type == 0 ? n : T;
+          for (int g0 = t0; g0 < t1; g0 += 32) {
+            std::vector<uint8_t> in(T, 0);
+            int u = 0;
+            for (int t = g0; t < std::min(g0 + 32, t1); ++t)
+              for (uint16_t v : nb[r][t]) u += in[v] ? 0 : (in[v] = 1);
+            walked += hr[r] * 32.0 * u;
+          }
+        }
+      }
+      tasks = walked > 0.0 && useful / walked >= 0.35;
+    }
+  }
+  // choose the number of CTAs that share a group: by default the fewest that hold one codeword
+  // (an attention read of a key held by another CTA of the cluster costs far more than the
+  // token rows left idle by a looser packing), with as many words per group as fit; an explicit
+  // cluster_ctas is honoured when it can hold a word
+  int best_C = 0, best_G = 0;
+  const int cmin = (T + kRows - 1) / kRows;
+  for (int C = cmin; C <= kMaxCluster && !best_C; ++C) {
+    if (tasks && C != 1) continue;
+    if (d.cluster_ctas && C != d.cluster_ctas) continue;
+    const int G = (tasks && D == 128) ? 1 : (C * kRows) / T;
+    if (G < 1) continue;
+    if (((G + C - 1) / C) * n > kOutBitsBytes) continue;
+    best_C = C, best_G = G;
+  }
+  if (!best_C) return d.cluster_ctas ? AECCT_ERR_INVALID_ARG : AECCT_ERR_UNSUPPORTED;
+  if (best_G * ((n + 31) / 32) > 128) return AECCT_ERR_UNSUPPORTED;  // hard-decision bitmasks of a group
+  if (d.alpha_mode == 1 && best_C != 1) return AECCT_ERR_UNSUPPORTED;  // per-word alpha: one CTA per word
+
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return AECCT_ERR_NO_DEVICE;
+  cudaDeviceProp prop;
+  e = cudaGetDeviceProperties(&prop, dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDeviceProperties");
+  if (prop.major != 10) {
+    g_last_error = "device is not compute capability 10.x";
+    return AECCT_ERR_NO_DEVICE;
+  }
+  int max_clusters = 0;
+  e = prepare_variant(d.activation, d.linear_mode, D, tasks, best_C, &max_clusters);
+  if (e != cudaSuccess) return cuda_fail(e, "kernel occupancy");
+  if (max_clusters < 1) {
+    g_last_error = "no cluster of this size fits on the device";
+    return AECCT_ERR_UNSUPPORTED;
+  }
+
+  aecct_handle *h = new aecct_handle();
+  h->n = n, h->k = k, h->T = T, h->m = m, h->d = D, h->n_layers = d.n_layers, h->h_first = d.h_first;
+  h->Tp = (tasks && D == 128) ? Tp128 : T;
+  h->d_spe = d.d_spe, h->C = best_C, h->G = best_G, h->max_clusters = max_clusters, h->tasks = tasks;
+  h->ln_eps = d.ln_eps, h->alpha_floor = d.alpha_floor, h->b_d1 = d.b_d1, h->device = dev;
+  h->alpha_mode = d.alpha_mode;
+  h->activation = d.activation;
+  h->linear_mode = d.linear_mode;
+  h->att_scale = static_cast<float>(1.4426950408889634074 / std::sqrt(static_cast<double>(D / kHeads)));
+  h->wait_limit = d.wait_limit_cycles ? d.wait_limit_cycles : (1LL << 32);
+
+  // ---- H rows as bitmasks over the variables, for the syndromes (parity of popcounts)
+  h->hwords = (n + 31) / 32;
+  std::vector<uint32_t> hbits((size_t)m * h->hwords, 0u);
+  for (int i = 0; i < m; ++i)
+    for (int j = 0; j < n; ++j)
+      if (d.H[(size_t)i * n + j]) hbits[(size_t)i * h->hwords + j / 32] |= 1u << (j % 32);
   // Rows of a codeword hold its tokens sorted by attention work (keys over the thread's first-ring
   // and second-ring head), so the 32 rows of a warp loop over similar key counts.
-  std::vector<uint16_t> perm(T), pos(T);
-  {
+  std::vector<uint16_t> perm(h->Tp, 0xFFFFu), pos(T);
+  if (tasks && D == 128) {
+    // variables in rows 0..n-1, checks from the 32-row boundary npad; rows n..npad-1 hold no token
+    for (int t = 0; t < T; ++t) {
+      const int row = t < n ? t : npad + (t - n);
+      perm[row] = static_cast<uint16_t>(t);
+      pos[t] = static_cast<uint16_t>(row);
+    }
+  } else {
     std::vector<int> order(T);
     for (int t = 0; t < T; ++t) order[t] = t;
     const int hf = d.h_first, hs = d.heads - d.h_first;
@@ -406,8 +446,15 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
       int row0, lanes, cwrow0;
     };
     std::vector<Grp> grps;
-    for (int cw = 0; cw < G; ++cw)
-      for (int off0 = 0; off0 < T; off0 += 32) grps.push_back({cw * T + off0, std::min(32, T - off0), cw * T});
+    if (D == 128) {
+      // one codeword; groups of the variables' rows, then of the checks' rows from npad: every group
+      // starts on a lane quadrant (its padding rows, if any, come last)
+      for (int off0 = 0; off0 < n; off0 += 32) grps.push_back({off0, std::min(32, n - off0), 0});
+      for (int off0 = npad; off0 < h->Tp; off0 += 32) grps.push_back({off0, std::min(32, h->Tp - off0), 0});
+    } else {
+      for (int cw = 0; cw < G; ++cw)
+        for (int off0 = 0; off0 < T; off0 += 32) grps.push_back({cw * T + off0, std::min(32, T - off0), cw * T});
+    }
     const int ng = static_cast<int>(grps.size());
     std::vector<int> ucount(ng * 2, 0);
     pgrp.assign((size_t)ng * 4, 0);
@@ -439,7 +486,8 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
         }
       }
     }
-    // tasks (group, head), longest first, each to the least-loaded warp
+    // tasks (group, head), longest first, each to the least-loaded warp (d = 128: to a warp of the
+    // group's TMEM lane quadrant, where its rows' Q and A live)
     std::vector<std::pair<int, int>> tl;  // (cost, task)
     for (int gi = 0; gi < ng; ++gi)
       for (int e = 0; e < kHeads; ++e) tl.push_back({ucount[gi * 2 + (e < d.h_first ? 0 : 1)] + 4, gi * 8 + e});
@@ -451,8 +499,14 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
     std::vector<int> cnt(kEpiWarps, 0);
     for (const auto &tk : tl) {
       int best = -1;
+      const int quad = (grps[tk.second / 8].row0 / 32) & 3;
       for (int w = 0; w < kEpiWarps; ++w)
-        if (cnt[w] < kMaxTasks && (best < 0 || load[w] < load[best])) best = w;
+        if (cnt[w] < kMaxTasks && (D != 128 || (w & 3) == quad) && (best < 0 || load[w] < load[best])) best = w;
+      if (best < 0) {
+        free_handle(h);
+        g_last_error = "attention plan: too many tasks for a warp";
+        return AECCT_ERR_UNSUPPORTED;
+      }
       ptask[(size_t)best * kMaxTasks + cnt[best]++] = static_cast<uint16_t>(tk.second);
       load[best] += tk.first;
     }
@@ -583,6 +637,7 @@ int aecct_decode(aecct_handle *h, const float *y_dev, int64_t B, uint8_t *bits_d
   if (prev != AECCT_OK) return prev;
   DecodeParams p = {};
   p.n = h->n, p.k = h->k, p.T = h->T, p.m = h->m, p.n_layers = h->n_layers, p.h_first = h->h_first;
+  p.Tp = h->Tp;
   p.d_spe = h->d_spe, p.C = h->C, p.G = h->G;
   p.B = B;
   p.n_groups = (B + h->G - 1) / h->G;
@@ -705,6 +760,7 @@ int aecct_decode_host_noalloc(aecct_handle *h, const float *y_host, int64_t B, u
     return cuda_fail(e, "copy y");
   DecodeParams p = {};
   p.n = h->n, p.k = h->k, p.T = h->T, p.m = h->m, p.n_layers = h->n_layers, p.h_first = h->h_first;
+  p.Tp = h->Tp;
   p.d_spe = h->d_spe, p.C = h->C, p.G = h->G;
   p.B = B;
   p.n_groups = (B + h->G - 1) / h->G;

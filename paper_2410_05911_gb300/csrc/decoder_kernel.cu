@@ -9,10 +9,12 @@ template cudaError_t launch_decode<64, false, 0, 0>(const DecodeParams &, cudaSt
 template cudaError_t launch_decode<128, false, 0, 0>(const DecodeParams &, cudaStream_t);
 template cudaError_t launch_decode<32, true, 0, 0>(const DecodeParams &, cudaStream_t);
 template cudaError_t launch_decode<64, true, 0, 0>(const DecodeParams &, cudaStream_t);
+template cudaError_t launch_decode<128, true, 0, 0>(const DecodeParams &, cudaStream_t);
 template cudaError_t prepare_decode_kernel<32, false, 0, 0>(int, int *);
 template cudaError_t prepare_decode_kernel<64, false, 0, 0>(int, int *);
 template cudaError_t prepare_decode_kernel<128, false, 0, 0>(int, int *);
 template cudaError_t prepare_decode_kernel<32, true, 0, 0>(int, int *);
 template cudaError_t prepare_decode_kernel<64, true, 0, 0>(int, int *);
+template cudaError_t prepare_decode_kernel<128, true, 0, 0>(int, int *);
 
 }  // namespace aecct

@@ -461,7 +461,7 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
   };
   auto dot2 = [&](const float4 *ka, const float4 *kb) -> float2 { return make_float2(dot(ka), dot(kb)); };
   const float2 sc = make_float2(scale, scale);
-  constexpr int U = 4;
+  constexpr int U = (DH >= 16) ? 2 : 4;  // keys per step (registers: U x d_h fp32 of K or V)
   // membership bits of a 16-key block (jb is a multiple of 16)
   auto segment = [&](int jb) -> uint32_t {
     const uint32_t word = jb < 64 ? (jb < 32 ? mask.x : mask.y) : (jb < 96 ? mask.z : mask.w);
@@ -1057,7 +1057,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
     uint32_t *bitw = reinterpret_cast<uint32_t *>(smem + L::kOffBitWords);  // [G][hwords] bitmasks
     const int W = p.hwords;
     const uint32_t qbar = 1 + qd;  // named barrier of the 4 warps sharing a lane quadrant
-    const int T = p.T, n = p.n, m = p.m, de = D - p.d_spe;
+    const int T = p.T, Tp = p.Tp, n = p.n, m = p.m, de = D - p.d_spe;
     const int W4 = 4 * D;
     const float inv_d = 1.0f / static_cast<float>(D);
     uint32_t kvr_ph = 0, kvf_ph = 0, zr_ph = 0, zf_ph = 0;
@@ -1082,13 +1082,13 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
       named_bar_sync(5, kEpiThreads);
       if (warp < p.G) {
         float a = 0.0f;
-        for (int i = lane; i < p.T; i += 32) a = fmaxf(a, rowmax_s[warp * p.T + i]);
+        for (int i = lane; i < p.Tp; i += 32) a = fmaxf(a, rowmax_s[warp * p.Tp + i]);
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, o));
         if (lane == 0) wordmax_s[warp] = a;
       }
       named_bar_sync(5, kEpiThreads);
-      const int gw = (static_cast<int>(crank) * kRows + r) / p.T;
+      const int gw = (static_cast<int>(crank) * kRows + r) / p.Tp;
       return gw < p.G ? wordmax_s[gw] : a_row;
     };
     auto row_sum = [&](float v) -> float {
@@ -1169,10 +1169,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
       }
       named_bar_sync(5, kEpiThreads);
       const int rho = static_cast<int>(crank) * kRows + r;
-      const int g = rho / T;
-      const int t = __ldg(p.perm + (rho - g * T));  // token held by this row (rows are ordered by attention work)
+      const int g = rho / Tp;
+      const int t = __ldg(p.perm + (rho - g * Tp));  // token held by this row (0xFFFF: a padding row)
       const int64_t b = gi * p.G + g;
-      const bool row_cw = g < p.G;
+      const bool row_cw = g < p.G && t != 0xFFFF;
       const bool valid = row_cw && b < p.B;
       const bool cap = valid && b < p.cap_B;
       const float *yrow = ybuf + (valid ? g : 0) * n;
@@ -1298,8 +1298,8 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             capture_acc(l, 0, ka, D + e * DH, DH);
             capture_acc(l, 0, va, 2 * D + e * DH, DH);
           }
-          // head slot of this row: row mode (K | V), task mode (Q | K | V)
-          const uint32_t dst = kvl + r * L::kKvStride + e * L::kSlot + (TASKS ? 4 * DH : 0);
+          // head slot of this row: (K | V), or (Q | K | V) in task mode at d <= 64
+          const uint32_t dst = kvl + r * L::kKvStride + e * L::kSlot + (L::kQInSmem ? 4 * DH : 0);
           dequant<DH>(ka, fk, bk, ka);
           dequant<DH>(va, fv, bv, va);
 #pragma unroll
@@ -1307,7 +1307,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             st_shared_f4(dst + 4 * i, ka[i], ka[i + 1], ka[i + 2], ka[i + 3]);
             st_shared_f4(dst + 4 * (DH + i), va[i], va[i + 1], va[i + 2], va[i + 3]);
           }
-          if constexpr (TASKS) {
+          if constexpr (L::kQInSmem) {
             float qa[DH], bq[DH];
             tmem_ld<DH>(tl + e * DH, qa);
             tmem_wait_ld();
@@ -1322,8 +1322,13 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         if constexpr (TASKS) {
           // ---------------- S5: HPSA (Sec. 4.2), task mode: warp tasks over query groups
           named_bar_sync(5, kEpiThreads);  // every Q, K, V row of this CTA is in shared memory
-          // this warp's score cache: its lane quadrant, kTaskCache columns of [kTaskCacheCol, 512)
-          static_assert(L::kTaskCacheCol >= 4u * D && L::kTaskCacheCol + 4u * kTaskCache <= L::kTmemCols, "TMEM");
+          // this warp's score cache: its lane quadrant, kTaskCache columns from kTaskCacheCol
+          static_assert(L::kQInSmem ? (L::kTaskCacheCol >= 4u * D && L::kTaskCacheCol + 4u * kTaskCache <= L::kTmemCols)
+                                    : (L::kTaskCacheCol >= 1u * D && L::kTaskCacheCol + 4u * kTaskCache <= 3u * D),
+                        "TMEM: the cache clears Q/A, the live accumulators and the parked residual");
+          // d = 128: a task's 32 rows are this warp's TMEM lane quadrant (the plan keeps every task on
+          // a warp of its group's quadrant); Q comes from the QKV accumulators of this thread's row
+          // and the output goes back over them
           const uint32_t tcache = tmem + (static_cast<uint32_t>(32 * (warp & 3)) << 16) + L::kTaskCacheCol +
                                   static_cast<uint32_t>(warp >> 2) * kTaskCache;
           for (int k = 0; k < kMaxTasks; ++k) {
@@ -1339,37 +1344,63 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             const uint4 mk = act ? __ldg(p.plan_mask + (grp * 2 + ring) * 32 + lane) : make_uint4(~0u, ~0u, ~0u, ~0u);
             const uint32_t ui = __ldg(p.plan_uinfo + grp * 2 + ring);
             float q[DH], a[DH];
-            const float4 *qp = reinterpret_cast<const float4 *>(smem + L::kOffU + row * L::kKvStride + e * L::kSlot);
+            if constexpr (L::kQInSmem) {
+              const float4 *qp = reinterpret_cast<const float4 *>(smem + L::kOffU + row * L::kKvStride + e * L::kSlot);
 #pragma unroll
-            for (int i = 0; i < DH / 4; ++i) {
-              const float4 v = qp[i];
-              q[4 * i] = v.x, q[4 * i + 1] = v.y, q[4 * i + 2] = v.z, q[4 * i + 3] = v.w;
+              for (int i = 0; i < DH / 4; ++i) {
+                const float4 v = qp[i];
+                q[4 * i] = v.x, q[4 * i + 1] = v.y, q[4 * i + 2] = v.z, q[4 * i + 3] = v.w;
+              }
+            } else {
+              float qa[DH], bq[DH];
+              tmem_ld<DH>(tl + e * DH, qa);
+              tmem_wait_ld();
+              if (cap) capture_acc(l, 0, qa, e * DH, DH);
+              ldg_vec<DH>(lp + LP::bqkv(D) + e * DH, bq);
+              dequant<DH>(qa, fq, bq, q);
             }
             hpsa_task<DH, L::kKvStride>(q, mk, static_cast<int>(ui & 255u), p.plan_ulist + (ui >> 8),
-                                        smem + L::kOffU + gi.z * L::kKvStride, e * L::kSlot + 4 * DH, p.att_scale,
-                                        tcache, a);
-            if (act) {
-              // A of (row, head e) replaces Q of (row, head e): this task was its only reader
-              float4 *ap = reinterpret_cast<float4 *>(smem + L::kOffU + row * L::kKvStride + e * L::kSlot);
+                                        smem + L::kOffU + gi.z * L::kKvStride,
+                                        e * L::kSlot + (L::kQInSmem ? 4 * DH : 0), p.att_scale, tcache, a);
+            if constexpr (L::kQInSmem) {
+              if (act) {
+                // A of (row, head e) replaces Q of (row, head e): this task was its only reader
+                float4 *ap = reinterpret_cast<float4 *>(smem + L::kOffU + row * L::kKvStride + e * L::kSlot);
 #pragma unroll
-              for (int i = 0; i < DH / 4; ++i) ap[i] = make_float4(a[4 * i], a[4 * i + 1], a[4 * i + 2], a[4 * i + 3]);
+                for (int i = 0; i < DH / 4; ++i) ap[i] = make_float4(a[4 * i], a[4 * i + 1], a[4 * i + 2], a[4 * i + 3]);
+              }
+            } else {
+              // every lane's own row: A of (row, head e) over the head's Q accumulators (a lane past
+              // the group's rows writes a padding or empty row, which nothing reads)
+              tmem_st<DH>(tl + e * DH, a);
             }
             __syncwarp();
           }
+          if constexpr (!L::kQInSmem) {
+            tmem_wait_st();
+            tc_fence_before();  // the TMEM stores are ordered before the barrier for the row owners
+          }
           named_bar_sync(5, kEpiThreads);  // A complete; Q, K, V no longer read
           // Quant(A) -> O operand, by row slices
-          // columns [sl XS, sl XS + XS) are heads 2 sl and 2 sl + 1, in their Q slots
+          // columns [sl XS, sl XS + XS) are heads 2 sl and 2 sl + 1, in their Q slots (shared memory)
+          // or over their Q accumulators (TMEM, d = 128)
           float av[XS];
+          if constexpr (L::kQInSmem) {
 #pragma unroll
-          for (int hh = 0; hh < 2; ++hh) {
-            const float4 *ap =
-                reinterpret_cast<const float4 *>(smem + L::kOffU + r * L::kKvStride + (2 * sl + hh) * L::kSlot);
+            for (int hh = 0; hh < 2; ++hh) {
+              const float4 *ap =
+                  reinterpret_cast<const float4 *>(smem + L::kOffU + r * L::kKvStride + (2 * sl + hh) * L::kSlot);
 #pragma unroll
-            for (int i = 0; i < DH / 4; ++i) {
-              const float4 v = ap[i];
-              av[hh * DH + 4 * i] = v.x, av[hh * DH + 4 * i + 1] = v.y;
-              av[hh * DH + 4 * i + 2] = v.z, av[hh * DH + 4 * i + 3] = v.w;
+              for (int i = 0; i < DH / 4; ++i) {
+                const float4 v = ap[i];
+                av[hh * DH + 4 * i] = v.x, av[hh * DH + 4 * i + 1] = v.y;
+                av[hh * DH + 4 * i + 2] = v.z, av[hh * DH + 4 * i + 3] = v.w;
+              }
             }
+          } else {
+            tc_fence_after();  // the tasks' TMEM stores of other warps are ordered by the barrier above
+            tmem_ld<XS>(tl + sl * XS, av);
+            tmem_wait_ld();
           }
           if constexpr (LIN == 1) {
             store_bf16<XS>(aop, r, sl * XS, D, av);
@@ -1419,10 +1450,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
               const uint32_t info = row_cw ? __ldg(p.mask_info[mk] + t) : 0u;
               if (p.C == 1)
                 hpsa_head<DH, U, L::kKvStride, false>(q, info, row_cw, p.mask_list[mk], smem + L::kOffU, s_kvcl,
-                                                      g * T, e * (8 * DH), p.att_scale, tcache, Ah);
+                                                      g * Tp, e * (8 * DH), p.att_scale, tcache, Ah);
               else
                 hpsa_head<DH, U, L::kKvStride, true>(q, info, row_cw, p.mask_list[mk], smem + L::kOffU, s_kvcl,
-                                                     g * T, e * (8 * DH), p.att_scale, tcache, Ah);
+                                                     g * Tp, e * (8 * DH), p.att_scale, tcache, Ah);
             }
   #pragma unroll
             for (int i = 0; i < DH; ++i) amax = fmaxf(amax, fabsf(Ah[i]));
@@ -1593,7 +1624,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         float *ztok = red.buf;
         for (int it = tid; it < n_local * T; it += kEpiThreads) {
           const int li = it / T, tt = it - li * T;
-          const int ru = (static_cast<int>(crank) + li * p.C) * T + __ldg(p.pos + tt);
+          const int ru = (static_cast<int>(crank) + li * p.C) * Tp + __ldg(p.pos + tt);
           ztok[it] = *reinterpret_cast<const float *>(s_zgen[ru >> 7] + static_cast<uint32_t>(ru & 127) * 4u);
         }
         named_bar_sync(5, kEpiThreads);

@@ -91,10 +91,13 @@ def test_create_rejects_invalid_packed_code_and_shapes():
     # a cluster size that cannot hold one codeword
     big = I.workload_model("ldpc384_192")
     assert _status(big, cluster_ctas=2) == A.AECCT_ERR_INVALID_ARG
-    # attention modes: unknown value, and warp tasks where they do not apply (T > 128, d = 128)
+    # attention modes: unknown value, and warp tasks where they do not apply (more than 128 token
+    # rows once each node type starts on a 32-row boundary; d = 128 with one alpha per word)
     assert _status(I.workload_model("bch31_16"), attention_mode=3) == A.AECCT_ERR_INVALID_ARG
     assert _status(I.workload_model("ldpc128_64"), attention_mode=2) == A.AECCT_ERR_UNSUPPORTED
-    assert _status(I.workload_model("bch63_36"), attention_mode=2) == A.AECCT_ERR_UNSUPPORTED
+    m63 = copy.deepcopy(I.workload_model("bch63_36"))
+    m63.alpha_mode = 1
+    assert _status(m63, attention_mode=2) == A.AECCT_ERR_UNSUPPORTED
     # one alpha per word needs one CTA per word
     m2 = copy.deepcopy(I.workload_model("ldpc128_64"))
     m2.alpha_mode = 1

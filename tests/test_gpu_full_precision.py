@@ -26,7 +26,7 @@ CASES = [
     ("bch31_16", 32, 2, dict(), (1, 2)),
     ("polar64_32", 64, 2, dict(), (1, 2)),
     ("ldpc128_64", 128, 2, dict(), (1,)),
-    ("bch63_36", 128, 2, dict(), (1,)),
+    ("bch63_36", 128, 2, dict(), (1, 2)),
     ("bch31_16", 32, 2, dict(activation=1, mask_mode=1), (1, 2)),
     ("polar64_32", 64, 2, dict(activation=1, mask_mode=1), (2,)),
     ("bch63_36", 128, 1, dict(activation=1, mask_mode=1), (1,)),

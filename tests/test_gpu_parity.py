@@ -73,10 +73,11 @@ def test_small_batch_exact_with_integer_core(key):
 
 LAYOUTS = {
     # (cluster_ctas, attention_mode): per-row lists over a packed cluster, one CTA per group,
-    # warp tasks (one CTA per group, d <= 64)
+    # warp tasks (one CTA per group; at d = 128 with Q and A in TMEM and the checks' rows from the
+    # next 32-row boundary)
     "bch31_16": [(0, 1), (1, 1), (0, 2)],
     "polar64_32": [(0, 1), (1, 1), (0, 2)],
-    "bch63_36": [(0, 1), (1, 1)],
+    "bch63_36": [(0, 1), (1, 1), (0, 2), (2, 1)],
 }
 
 

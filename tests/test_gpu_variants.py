@@ -28,7 +28,7 @@ CASES = [
     ("polar64_32", 64, 2, dict(binary=True), (2,)),
     ("bch31_16", 32, 2, dict(binary=True, h_first=6), (1, 2)),
     ("ldpc128_64", 128, 2, dict(h_first=6), (1,)),
-    ("bch63_36", 128, 1, dict(binary=True), (1,)),
+    ("bch63_36", 128, 1, dict(binary=True), (1, 2)),
     ("bch31_16", 32, 2, dict(mask_mode=1), (1, 2)),
     ("polar64_32", 64, 2, dict(mask_mode=1), (1, 2)),
     ("ldpc128_64", 128, 1, dict(mask_mode=1), (1,)),
@@ -39,6 +39,8 @@ CASES = [
     ("polar64_32", 64, 2, dict(activation=1), (1, 2)),
     ("ldpc128_64", 128, 1, dict(activation=1), (1,)),
     ("bch63_36", 128, 2, dict(activation=1, alpha_mode=1), (1,)),
+    ("bch63_36", 128, 2, dict(activation=1, h_first=2), (1, 2)),
+    ("bch63_36", 128, 1, dict(mask_mode=1), (1, 2)),
 ]
 
 
