@@ -63,8 +63,10 @@ typedef struct aecct_handle aecct_handle; /* opaque */
  *   cluster_ctas  0 = choose automatically; otherwise the number of CTAs (1..8) that
  *                 share one group of codewords (tuning knob).
  *   attention_mode 0 = choose automatically; 1 = per-row neighbour lists (any cluster size);
- *                 2 = warp tasks over shared key sets (one CTA per group, d <= 64, at most
- *                 128 tokens).  Every mode computes the same results bit for bit.
+ *                 2 = warp tasks over shared key sets (one CTA per group; d <= 64 with at most
+ *                 128 tokens, or d = 128 with alpha_mode 0 and at most 128 rows once the checks'
+ *                 rows start on the first 32-row boundary after the variables).  Every mode
+ *                 computes the same results bit for bit.
  *   mask_mode     0 = HPSA (Sec. 4.2): heads [0, h_first) first ring, the rest second ring;
  *                 1 = the ECCT code-aware mask (Sec. 3) for every head: the union of the first
  *                 and second rings (which contains each node itself).  Other values are rejected.
