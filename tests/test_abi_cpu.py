@@ -98,6 +98,11 @@ def test_create_rejects_invalid_packed_code_and_shapes():
     m63 = copy.deepcopy(I.workload_model("bch63_36"))
     m63.alpha_mode = 1
     assert _status(m63, attention_mode=2) == A.AECCT_ERR_UNSUPPORTED
+    # d = 128: T = 98 + 28 = 126 tokens, but the 98 variables take rows 0..97, so the checks would
+    # start at row 128
+    c98 = I.ldpc_regular_code(98, 70, 2, 7, seed=0)
+    assert c98.n + c98.H.shape[0] <= 128
+    assert _status(I.random_model(c98, 128, 1, seed=3), attention_mode=2) == A.AECCT_ERR_UNSUPPORTED
     # one alpha per word needs one CTA per word
     m2 = copy.deepcopy(I.workload_model("ldpc128_64"))
     m2.alpha_mode = 1

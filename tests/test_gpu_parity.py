@@ -194,3 +194,32 @@ def test_extreme_shapes_exact(label, make, d, layers, B):
         assert (a.view(np.int32) if a.dtype == np.float32 else a).tolist() == \
             (b.view(np.int32) if b.dtype == np.float32 else b).tolist(), f"{label}: {name}"
     dec.close()
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("label,make,d,layers,B", [
+    # d = 128 warp tasks: the variables start at row 0 and the checks at the next 32-row boundary,
+    # so the rows per word Tp run from 35 (more padding than tokens) to the limit 128
+    ("hamming7_4", lambda: I.make_code("hamming7_4"), 128, 2, 13),
+    ("bch31_16", lambda: I.make_code("bch31_16"), 128, 1, 11),
+    ("polar64_32", lambda: I.make_code("polar64_32"), 128, 1, 7),
+    ("ldpc96_64", lambda: I.ldpc_regular_code(96, 64, 3, 9, seed=9664), 128, 1, 5),
+    # d <= 64 warp tasks pack the tokens: T = 126 of the 128 rows of a CTA
+    ("ldpc98_70", lambda: I.ldpc_regular_code(98, 70, 2, 7, seed=0), 64, 2, 6),
+    ("ldpc98_70-d32", lambda: I.ldpc_regular_code(98, 70, 2, 7, seed=0), 32, 1, 6),
+])
+def test_warp_tasks_row_limits_exact(label, make, d, layers, B):
+    code = make()
+    model = I.random_model(code, d, layers, seed=23)
+    ch = I.channel_batch(code, B, 3.0, seed=29)
+    r = O.decode(model, ch.y, cap_B=min(B, 3))
+    for mode in (1, 2):
+        dec = A.Decoder(model, attention_mode=mode)
+        assert dec.query()["attention_mode"] == mode
+        g = gpu_decode(dec, ch.y, cap_B=min(B, 3))
+        assert_same(g, r, f"{label} mode {mode}")
+        for name in ("q", "acc", "alpha", "syn_in"):
+            a, b = g["capture"][name], r["capture"][name]
+            assert (a.view(np.int32) if a.dtype == np.float32 else a).tolist() == \
+                (b.view(np.int32) if b.dtype == np.float32 else b).tolist(), f"{label} mode {mode}: {name}"
+        dec.close()
