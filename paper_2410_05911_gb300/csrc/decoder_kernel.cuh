@@ -982,6 +982,9 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   using LP = LayerParamLayout;
   constexpr int DH = D / kHeads;  // head width
   constexpr int XS = D / 4;       // x columns per thread
+  // the O and FFN2 biases are loaded before the accumulator waits where the registers allow it
+  // (d <= 64; at d = 128 the 32 extra live registers spill)
+  constexpr bool kEarlyBias = D <= 64;
   constexpr int S = L::kStages;
   extern __shared__ __align__(1024) uint8_t smem[];
   const uint32_t sb = smem_u32(smem);
@@ -1228,9 +1231,8 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         return __fdiv_rn(__fmul_rn(__ldg(swp), alpha_in), 127.0f);
       };
       // x <- LayerNorm(x + (acc * f + bias)) with gamma g and beta be (Post-LN, Sec. 5)
-      auto residual_ln = [&](const float *ac, float f, const float *bias, const float *g, const float *be) {
-        float bb[XS], v[XS];
-        ldg_vec<XS>(bias, bb);
+      auto residual_ln = [&](const float *ac, float f, const float *bb, const float *g, const float *be) {
+        float v[XS];
         dequant<XS>(ac, f, bb, v);
 #pragma unroll
         for (int j = 0; j < XS; ++j) v[j] = __fadd_rn(x[j], v[j]);
@@ -1277,23 +1279,23 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         const float *lp = p.lparams + (size_t)l * LP::stride(D);
         const float *sw = lp + LP::sw(D);
         // ---------------- S4 epilogue: K, V to shared memory
+        const float fq = dq_factor(sw + 0);
+        const float fk = dq_factor(sw + 1);
+        const float fv = dq_factor(sw + 2);
         wait_acc();
         // park the residual row in TMEM columns [3D, 4D) (unused by the QKV and O accumulators)
         // so that attention runs with the registers it needs
         tmem_st<XS>(tl + 3 * D + sl * XS, x);
         tmem_wait_st();
-        const float fq = dq_factor(sw + 0);
-        const float fk = dq_factor(sw + 1);
-        const float fv = dq_factor(sw + 2);
 #pragma unroll
         for (int hh = 0; hh < 2; ++hh) {
           const int e = sl + 4 * hh;
           float ka[DH], va[DH], bk[DH], bv[DH];
+          ldg_vec<DH>(lp + LP::bqkv(D) + D + e * DH, bk);
+          ldg_vec<DH>(lp + LP::bqkv(D) + 2 * D + e * DH, bv);
           tmem_ld<DH>(tl + D + e * DH, ka);
           tmem_ld<DH>(tl + 2 * D + e * DH, va);
           tmem_wait_ld();
-          ldg_vec<DH>(lp + LP::bqkv(D) + D + e * DH, bk);
-          ldg_vec<DH>(lp + LP::bqkv(D) + 2 * D + e * DH, bv);
           if (cap) {
             capture_acc(l, 0, ka, D + e * DH, DH);
             capture_acc(l, 0, va, 2 * D + e * DH, DH);
@@ -1309,10 +1311,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           }
           if constexpr (L::kQInSmem) {
             float qa[DH], bq[DH];
+            ldg_vec<DH>(lp + LP::bqkv(D) + e * DH, bq);
             tmem_ld<DH>(tl + e * DH, qa);
             tmem_wait_ld();
             if (cap) capture_acc(l, 0, qa, e * DH, DH);
-            ldg_vec<DH>(lp + LP::bqkv(D) + e * DH, bq);
             const uint32_t qdst = kvl + r * L::kKvStride + e * L::kSlot;
             dequant<DH>(qa, fq, bq, qa);
 #pragma unroll
@@ -1353,10 +1355,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
               }
             } else {
               float qa[DH], bq[DH];
+              ldg_vec<DH>(lp + LP::bqkv(D) + e * DH, bq);
               tmem_ld<DH>(tl + e * DH, qa);
               tmem_wait_ld();
               if (cap) capture_acc(l, 0, qa, e * DH, DH);
-              ldg_vec<DH>(lp + LP::bqkv(D) + e * DH, bq);
               dequant<DH>(qa, fq, bq, q);
             }
             hpsa_task<DH, L::kKvStride>(q, mk, static_cast<int>(ui & 255u), p.plan_ulist + (ui >> 8),
@@ -1433,10 +1435,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             const int e = sl + 4 * hh;
             float *Ah = A[kStashA ? 0 : hh];
             float qa[DH], bq[DH];
+            ldg_vec<DH>(lp + LP::bqkv(D) + e * DH, bq);
             tmem_ld<DH>(tl + e * DH, qa);
             tmem_wait_ld();
             if (cap) capture_acc(l, 0, qa, e * DH, DH);
-            ldg_vec<DH>(lp + LP::bqkv(D) + e * DH, bq);
             float q[DH];
   #pragma unroll
             for (int i = 0; i < DH; ++i) q[i] = __fadd_rn(__fmul_rn(qa[i], fq), bq[i]);
@@ -1500,15 +1502,17 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         signal_op(1, l, gi);
 
         // ---------------- S6: O projection + residual + LayerNorm (Sec. 5, Post-LN)
-        wait_acc();
         {
           const float fo = dq_factor(sw + 3);
-          float ac[XS];
+          float ac[XS], bb[XS];
+          if constexpr (kEarlyBias) ldg_vec<XS>(lp + LP::bo(D) + sl * XS, bb);
+          wait_acc();
           tmem_ld<XS>(tl + sl * XS, ac);
           tmem_ld<XS>(tl + 3 * D + sl * XS, x);
           tmem_wait_ld();
           if (cap) capture_acc(l, 1, ac, sl * XS, XS);
-          residual_ln(ac, fo, lp + LP::bo(D) + sl * XS, lp + LP::ln1g(D) + sl * XS, lp + LP::ln1b(D) + sl * XS);
+          if constexpr (!kEarlyBias) ldg_vec<XS>(lp + LP::bo(D) + sl * XS, bb);
+          residual_ln(ac, fo, bb, lp + LP::ln1g(D) + sl * XS, lp + LP::ln1b(D) + sl * XS);
         }
         {
           const float rr = quant_x_to_aop();
@@ -1521,9 +1525,9 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         signal_op(2, l, gi);
 
         // ---------------- S7: FFN1 + ReLU (Sec. 4 item 4) or GELU, Quant(u) -> FFN2 operand
-        wait_acc();
         {
           const float f1 = dq_factor(sw + 4);
+          wait_acc();
           // ACT 0 = ReLU, 1 = GELU.  u = act(acc f1 + b1) in 32-column chunks of this thread's D
           // hidden columns.  AAP: u is stored over its own accumulators in TMEM (this thread's
           // lane and columns) between the row maximum and the codes, which leaves the registers
@@ -1583,14 +1587,16 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         signal_op(3, l, gi);
 
         // ---------------- S8: FFN2 + residual + LayerNorm
-        wait_acc();
         {
           const float f2 = dq_factor(sw + 5);
-          float ac[XS];
+          float ac[XS], bb[XS];
+          if constexpr (kEarlyBias) ldg_vec<XS>(lp + LP::b2(D) + sl * XS, bb);
+          wait_acc();
           tmem_ld<XS>(tl + sl * XS, ac);
           tmem_wait_ld();
           if (cap) capture_acc(l, 3, ac, sl * XS, XS);
-          residual_ln(ac, f2, lp + LP::b2(D) + sl * XS, lp + LP::ln2g(D) + sl * XS, lp + LP::ln2b(D) + sl * XS);
+          if constexpr (!kEarlyBias) ldg_vec<XS>(lp + LP::b2(D) + sl * XS, bb);
+          residual_ln(ac, f2, bb, lp + LP::ln2g(D) + sl * XS, lp + LP::ln2b(D) + sl * XS);
         }
         if (l + 1 < p.n_layers) {
           const float rr = quant_x_to_aop();
