@@ -350,7 +350,7 @@ def run_cuda(args, rank, world, local_rank):
     alu = dict(bound="alu", achieved=alu_tops, peak=ALU_PEAK_TOPS, unit="TFLOP/s", frac=alu_tops / ALU_PEAK_TOPS,
                work="algorithmic fp32 ops of the canonical forward pass per word (bench.alu_ops_per_word; an FMA "
                     "is one op); peak = 152 SMs x 128 fp32 lanes x 2070 MHz (derived, not measured)")
-    # d <= 64: the fp32 work (HPSA, epilogues) binds; d = 128: the contraction
+    # d <= 64: the fp32 work (HPSA, epilogues) binds; d = 128: the linear layers' contraction
     roof = dict(alu if w.d <= 64 else tensor)
     roof.update(traffic=args.traffic if args.traffic is not None else
                 (measured_traffic(args.workload, B) if args.variant == "aecct" else None),
