@@ -144,8 +144,11 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out);
  *   logits_dev    fp32 [B][n] or NULL: the network output eps (multiplicative-noise
  *                 prediction, Sec. 3).
  * Runs asynchronously on cuda_stream (a cudaStream_t; NULL = legacy default stream).
- * B == 0 is a no-op.  Errors: INVALID_ARG (B < 0, NULL y/bits with B > 0), CUDA,
- * and TIMEOUT reported for an earlier decode on this handle whose kernel stopped. */
+ * B == 0 is a no-op.  y is expected finite: a NaN or infinity is not checked, and the words
+ * it reaches get unspecified bits and logits (no value steers a memory access, so the
+ * other words of the batch are unaffected).  Errors: INVALID_ARG (B < 0, NULL y/bits with
+ * B > 0), CUDA, and TIMEOUT reported for an earlier decode on this handle whose kernel
+ * stopped. */
 int aecct_decode(aecct_handle *h, const float *y_dev, int64_t B, uint8_t *bits_dev, uint8_t *syndrome_dev,
                  float *logits_dev, void *cuda_stream);
 

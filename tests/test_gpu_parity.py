@@ -223,3 +223,21 @@ def test_warp_tasks_row_limits_exact(label, make, d, layers, B):
             assert (a.view(np.int32) if a.dtype == np.float32 else a).tolist() == \
                 (b.view(np.int32) if b.dtype == np.float32 else b).tolist(), f"{label} mode {mode}: {name}"
         dec.close()
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("key", ["bch31_16", "polar64_32", "bch63_36"])
+def test_non_finite_word_leaves_the_others_exact(key):
+    # a NaN or infinity in one word reaches only that word's rows (every step is row-local or
+    # within one word), so the other words of the batch, including one sharing its CTA, decode
+    # exactly as without it
+    dec, model = decoder(key)
+    w = I.workload(key)
+    ch = I.channel_batch(w.code, 6, 4.0, seed=41)
+    y = ch.y.copy()
+    y[2, 0] = np.nan  # BCH(31,16) packs two words per CTA: words 3 and 4 share a CTA with these
+    y[5, 1] = -np.inf
+    g = gpu_decode(dec, y)
+    keep = [0, 1, 3, 4]
+    r = O.decode(model, ch.y[keep])
+    assert_same({k: v[keep] for k, v in g.items()}, r, key)
