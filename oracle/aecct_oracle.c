@@ -37,7 +37,8 @@
  * its odd-part identity, pairwise sums, quantiser and
  * LayerNorm closed forms, brute-force integer products, masks against Tanner-graph distances,
  * codeword-symmetry invariance, the all-zero-weight closed form, and an independent float64
- * forward pass teacher-forced on the recorded integer core.
+ * forward pass teacher-forced on the recorded integer core.  A planted-mistake test compiles
+ * copies of this file with one mistake each and checks that every copy fails one of those pins.
  */
 #include <math.h>
 #include <pthread.h>

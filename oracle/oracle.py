@@ -58,7 +58,9 @@ def lib():
     global _lib
     with _lock:
         if _lib is None:
-            path = build()
+            # AECCT_ORACLE_LIB names another build of this file (the planted-mistake tests run the
+            # pins against copies of the oracle with one mistake each)
+            path = os.environ.get("AECCT_ORACLE_LIB") or build()
             L = ctypes.CDLL(path)
             P = ctypes.c_void_p
             L.oracle_decode.argtypes = [ctypes.POINTER(OracleModel), P, ctypes.c_int64, P, P, P, ctypes.c_int,
