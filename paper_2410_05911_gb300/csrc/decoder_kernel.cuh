@@ -666,6 +666,8 @@ struct Issuer {
   __device__ __forceinline__ uint32_t bar_empty(int s) const { return sb + L::kOffBar + 8 * (S + s); }
   __device__ __forceinline__ uint32_t bar_op() const { return sb + L::kOffBar + 16 * S; }
   __device__ __forceinline__ uint32_t bar_acc() const { return sb + L::kOffBar + 16 * S + 8; }
+  // the accumulators are complete: let the CTA's other warps (waiting in wait_acc) go
+  __device__ __forceinline__ static void release_acc() { named_bar_arrive(5, kEpiThreads); }
 
   // whole warp: lane 0 polls (the slow path is bounded and raises the abort flag), then the
   // warp reconverges
@@ -739,8 +741,9 @@ struct Issuer {
     chunk_mmas<G, 0>(w_cur);
     mma_commit_warp(bar_acc());
     // warp 0 alone waits for the accumulators; the other warps of the CTA wait in a named
-    // barrier (no spinning), which warp 0 joins after the wait
+    // barrier (no spinning), which warp 0 arrives at after the wait, before its copies
     wait(bar_acc(), G & 1);
+    release_acc();
     // every MMA so far is complete, so the stages they read are free
     refill<(count > S ? first + count : first + S), first + count + S>(w_cur, w_next, has_next);
   }
@@ -783,6 +786,8 @@ struct Issuer<128, TASKS> {
   __device__ __forceinline__ uint32_t bar_empty(int s) const { return sb + L::kOffBar + 8 * (3 + s); }
   __device__ __forceinline__ uint32_t bar_op() const { return sb + L::kOffBar + 48; }
   __device__ __forceinline__ uint32_t bar_acc() const { return sb + L::kOffBar + 56; }
+  // the accumulators are complete: let the CTA's other warps (waiting in wait_acc) go
+  __device__ __forceinline__ static void release_acc() { named_bar_arrive(5, kEpiThreads); }
 
   // slot of chunk P: shared-memory offset, barrier id, uses of that barrier per block, use index
   struct Slot {
@@ -897,6 +902,7 @@ struct Issuer<128, TASKS> {
       mmas<0, 5>();
       mma_commit_warp(bar_acc());
       wait(bar_acc(), 0);
+      release_acc();
     } else if constexpr (G == 1) {
       wait(bar(0), parity<6>(lp));
       mmas<1, 6>();
@@ -913,6 +919,7 @@ struct Issuer<128, TASKS> {
       }
       copy1<18>(w_cur);
       wait(bar_acc(), 1);
+      release_acc();
       copy1<16>(w_cur);  // W0, W1 were O's
       copy1<17>(w_cur);
     } else if constexpr (G == 2) {
@@ -928,6 +935,7 @@ struct Issuer<128, TASKS> {
       mmas_pair<2, 14>();
       mma_commit_warp(bar_acc());
       wait(bar_acc(), 0);
+      release_acc();
       copy1<19>(w_cur);  // the operand tile is free: FFN1's MMAs are done
       copy1<20>(w_cur);
     } else {
@@ -960,6 +968,7 @@ struct Issuer<128, TASKS> {
       mmas<3, 23>();
       mma_commit_warp(bar_acc());
       wait(bar_acc(), 1);
+      release_acc();
       if (has_next) stage_qkv_o(w_next);  // region U and W0, W1 are free again
     }
   }
@@ -1134,10 +1143,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
       }
       __syncwarp();
     };
-    // accumulators of the last GEMM are complete once warp 0 (which waited for them inside
-    // issue_gemm) reaches this barrier
+    // accumulators of the last GEMM are complete once warp 0, which waited for them in its
+    // gemm<G> call and then arrived at this barrier, releases it
     auto wait_acc = [&]() {
-      named_bar_sync(5, kEpiThreads);
+      if (warp != 0) named_bar_sync(5, kEpiThreads);
       tc_fence_after();
     };
     // wait for a cluster-wide phase: thread 0 waits on the mbarrier, the others in a named barrier
