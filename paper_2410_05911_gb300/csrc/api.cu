@@ -608,6 +608,35 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
   return AECCT_OK;
 }
 
+// the kernel arguments of one decode call: the handle's model and plan, this call's buffers
+static DecodeParams decode_params(const aecct_handle *h, int64_t B, const float *y_dev, uint8_t *bits_dev,
+                                  uint8_t *syn_dev, float *logits_dev, int *err_dev) {
+  DecodeParams p = {};
+  p.n = h->n, p.k = h->k, p.T = h->T, p.m = h->m, p.n_layers = h->n_layers, p.h_first = h->h_first;
+  p.Tp = h->Tp;
+  p.d_spe = h->d_spe, p.C = h->C, p.G = h->G;
+  p.B = B;
+  p.n_groups = (B + h->G - 1) / h->G;
+  p.n_clusters = static_cast<int>(p.n_groups < h->max_clusters ? p.n_groups : h->max_clusters);
+  p.y = y_dev, p.bits = bits_dev, p.syn = syn_dev, p.logits = logits_dev;
+  p.wstream = h->wstream, p.layer_bytes = h->layer_bytes;
+  p.lparams = h->lparams, p.emb = h->emb, p.spe = h->spe, p.w_d1 = h->w_d1, p.b_d1 = h->b_d1;
+  p.w_out = h->w_out, p.b_out = h->b_out, p.hbits = h->hbits, p.hwords = h->hwords;
+  p.perm = h->perm, p.pos = h->pos;
+  p.plan_task = h->plan_task;
+  p.plan_grp = reinterpret_cast<const uint4 *>(h->plan_grp);
+  p.plan_uinfo = h->plan_uinfo;
+  p.plan_ulist = reinterpret_cast<const uint4 *>(h->plan_ulist);
+  p.plan_mask = reinterpret_cast<const uint4 *>(h->plan_mask);
+  p.mask_info[0] = h->mask_info[0], p.mask_info[1] = h->mask_info[1];
+  p.mask_list[0] = reinterpret_cast<const uint4 *>(h->mask_list[0]);
+  p.mask_list[1] = reinterpret_cast<const uint4 *>(h->mask_list[1]);
+  p.ln_eps = h->ln_eps, p.alpha_floor = h->alpha_floor, p.att_scale = h->att_scale, p.alpha_mode = h->alpha_mode;
+  p.cap_B = h->cap_B, p.cap_q = h->cap_q, p.cap_acc = h->cap_acc, p.cap_alpha = h->cap_alpha, p.cap_syn = h->cap_syn;
+  p.err = err_dev, p.wait_limit = h->wait_limit;
+  return p;
+}
+
 static int collect_status(aecct_handle *h, bool block) {
   if (!h->ev_pending) {
     const int s = h->pending_status;
@@ -635,29 +664,7 @@ int aecct_decode(aecct_handle *h, const float *y_dev, int64_t B, uint8_t *bits_d
   cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
   const int prev = collect_status(h, false);
   if (prev != AECCT_OK) return prev;
-  DecodeParams p = {};
-  p.n = h->n, p.k = h->k, p.T = h->T, p.m = h->m, p.n_layers = h->n_layers, p.h_first = h->h_first;
-  p.Tp = h->Tp;
-  p.d_spe = h->d_spe, p.C = h->C, p.G = h->G;
-  p.B = B;
-  p.n_groups = (B + h->G - 1) / h->G;
-  p.n_clusters = static_cast<int>(p.n_groups < h->max_clusters ? p.n_groups : h->max_clusters);
-  p.y = y_dev, p.bits = bits_dev, p.syn = syndrome_dev, p.logits = logits_dev;
-  p.wstream = h->wstream, p.layer_bytes = h->layer_bytes;
-  p.lparams = h->lparams, p.emb = h->emb, p.spe = h->spe, p.w_d1 = h->w_d1, p.b_d1 = h->b_d1;
-  p.w_out = h->w_out, p.b_out = h->b_out, p.hbits = h->hbits, p.hwords = h->hwords;
-  p.perm = h->perm, p.pos = h->pos;
-  p.plan_task = h->plan_task;
-  p.plan_grp = reinterpret_cast<const uint4 *>(h->plan_grp);
-  p.plan_uinfo = h->plan_uinfo;
-  p.plan_ulist = reinterpret_cast<const uint4 *>(h->plan_ulist);
-  p.plan_mask = reinterpret_cast<const uint4 *>(h->plan_mask);
-  p.mask_info[0] = h->mask_info[0], p.mask_info[1] = h->mask_info[1];
-  p.mask_list[0] = reinterpret_cast<const uint4 *>(h->mask_list[0]);
-  p.mask_list[1] = reinterpret_cast<const uint4 *>(h->mask_list[1]);
-  p.ln_eps = h->ln_eps, p.alpha_floor = h->alpha_floor, p.att_scale = h->att_scale, p.alpha_mode = h->alpha_mode;
-  p.cap_B = h->cap_B, p.cap_q = h->cap_q, p.cap_acc = h->cap_acc, p.cap_alpha = h->cap_alpha, p.cap_syn = h->cap_syn;
-  p.err = h->d_err, p.wait_limit = h->wait_limit;
+  const DecodeParams p = decode_params(h, B, y_dev, bits_dev, syndrome_dev, logits_dev, h->d_err);
   cudaError_t e;
   e = launch_variant(h->activation, h->linear_mode, h->d, h->tasks, p, stream);
   if (e != cudaSuccess) return cuda_fail(e, "decode launch");
@@ -758,29 +765,7 @@ int aecct_decode_host_noalloc(aecct_handle *h, const float *y_host, int64_t B, u
   if ((e = cudaMemsetAsync(err, 0, sizeof(int), stream)) != cudaSuccess) return cuda_fail(e, "clear status");
   if ((e = cudaMemcpyAsync(y_dev, y_host, sizeof(float) * b * n, cudaMemcpyHostToDevice, stream)) != cudaSuccess)
     return cuda_fail(e, "copy y");
-  DecodeParams p = {};
-  p.n = h->n, p.k = h->k, p.T = h->T, p.m = h->m, p.n_layers = h->n_layers, p.h_first = h->h_first;
-  p.Tp = h->Tp;
-  p.d_spe = h->d_spe, p.C = h->C, p.G = h->G;
-  p.B = B;
-  p.n_groups = (B + h->G - 1) / h->G;
-  p.n_clusters = static_cast<int>(p.n_groups < h->max_clusters ? p.n_groups : h->max_clusters);
-  p.y = y_dev, p.bits = bits_dev, p.syn = syn_dev, p.logits = logits_dev;
-  p.wstream = h->wstream, p.layer_bytes = h->layer_bytes;
-  p.lparams = h->lparams, p.emb = h->emb, p.spe = h->spe, p.w_d1 = h->w_d1, p.b_d1 = h->b_d1;
-  p.w_out = h->w_out, p.b_out = h->b_out, p.hbits = h->hbits, p.hwords = h->hwords;
-  p.perm = h->perm, p.pos = h->pos;
-  p.plan_task = h->plan_task;
-  p.plan_grp = reinterpret_cast<const uint4 *>(h->plan_grp);
-  p.plan_uinfo = h->plan_uinfo;
-  p.plan_ulist = reinterpret_cast<const uint4 *>(h->plan_ulist);
-  p.plan_mask = reinterpret_cast<const uint4 *>(h->plan_mask);
-  p.mask_info[0] = h->mask_info[0], p.mask_info[1] = h->mask_info[1];
-  p.mask_list[0] = reinterpret_cast<const uint4 *>(h->mask_list[0]);
-  p.mask_list[1] = reinterpret_cast<const uint4 *>(h->mask_list[1]);
-  p.ln_eps = h->ln_eps, p.alpha_floor = h->alpha_floor, p.att_scale = h->att_scale, p.alpha_mode = h->alpha_mode;
-  p.cap_B = h->cap_B, p.cap_q = h->cap_q, p.cap_acc = h->cap_acc, p.cap_alpha = h->cap_alpha, p.cap_syn = h->cap_syn;
-  p.err = err, p.wait_limit = h->wait_limit;
+  const DecodeParams p = decode_params(h, B, y_dev, bits_dev, syn_dev, logits_dev, err);
   e = launch_variant(h->activation, h->linear_mode, h->d, h->tasks, p, stream);
   if (e != cudaSuccess) return cuda_fail(e, "decode launch");
   if ((e = cudaMemcpyAsync(bits_host, bits_dev, b * n, cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
@@ -820,8 +805,9 @@ int aecct_query(const aecct_handle *h, int32_t *cluster_ctas, int32_t *words_per
   if (max_clusters) *max_clusters = h->max_clusters;
   if (threads_per_cta) *threads_per_cta = kThreads;
   int sm;
-  if (h->tasks) sm = h->d == 32 ? SmemLayout<32, true>::kTotal : SmemLayout<64, true>::kTotal;
-  else sm = h->d == 32 ? SmemLayout<32>::kTotal : (h->d == 64 ? SmemLayout<64>::kTotal : SmemLayout<128>::kTotal);
+  if (h->d == 32) sm = h->tasks ? SmemLayout<32, true>::kTotal : SmemLayout<32>::kTotal;
+  else if (h->d == 64) sm = h->tasks ? SmemLayout<64, true>::kTotal : SmemLayout<64>::kTotal;
+  else sm = h->tasks ? SmemLayout<128, true>::kTotal : SmemLayout<128>::kTotal;
   if (smem_bytes) *smem_bytes = sm;
   if (attention_mode) *attention_mode = h->tasks ? 2 : 1;
   return AECCT_OK;

@@ -213,9 +213,12 @@ def test_warp_tasks_row_limits_exact(label, make, d, layers, B):
     model = I.random_model(code, d, layers, seed=23)
     ch = I.channel_batch(code, B, 3.0, seed=29)
     r = O.decode(model, ch.y, cap_B=min(B, 3))
+    smem = {}
     for mode in (1, 2):
         dec = A.Decoder(model, attention_mode=mode)
-        assert dec.query()["attention_mode"] == mode
+        q = dec.query()
+        assert q["attention_mode"] == mode
+        smem[mode] = q["smem_bytes"]
         g = gpu_decode(dec, ch.y, cap_B=min(B, 3))
         assert_same(g, r, f"{label} mode {mode}")
         for name in ("q", "acc", "alpha", "syn_in"):
@@ -223,6 +226,8 @@ def test_warp_tasks_row_limits_exact(label, make, d, layers, B):
             assert (a.view(np.int32) if a.dtype == np.float32 else a).tolist() == \
                 (b.view(np.int32) if b.dtype == np.float32 else b).tolist(), f"{label} mode {mode}: {name}"
         dec.close()
+    if d == 128:  # Q stays in TMEM: both modes lay out shared memory alike
+        assert smem[1] == smem[2]
 
 
 @pytest.mark.gpu
