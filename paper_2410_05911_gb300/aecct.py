@@ -166,6 +166,23 @@ def create_handle(model, cluster_ctas: int = 0, wait_limit_cycles: int = 0, atte
     return st, (h if st == AECCT_OK else None)
 
 
+def check_outputs(out, B: int, n: int, m: int, device):
+    """Caller-provided decode outputs (bits, syndrome or None, logits or None).  The kernel writes
+    B full rows of each, so their shapes, types and device are checked here: the C ABI sees only
+    pointers."""
+    import torch
+
+    bits, syn, logits = out
+    for name, t, shape, dtype, required in (("bits", bits, (B, n), torch.uint8, True),
+                                            ("syndrome", syn, (B, m), torch.uint8, False),
+                                            ("logits", logits, (B, n), torch.float32, False)):
+        if t is None and not required:
+            continue
+        if t is None or t.device != device or t.dtype != dtype or tuple(t.shape) != shape or not t.is_contiguous():
+            raise ValueError(f"out {name} must be a contiguous {dtype} tensor of shape {shape} on {device}")
+    return bits, syn, logits
+
+
 class Decoder:
     """A decoder handle on the current CUDA device.
 
@@ -218,7 +235,7 @@ class Decoder:
             syn = torch.empty((B, self.m), dtype=torch.uint8, device=y.device) if want_syndrome else None
             logits = torch.empty((B, self.n), dtype=torch.float32, device=y.device) if want_logits else None
         else:
-            bits, syn, logits = out
+            bits, syn, logits = check_outputs(out, B, self.n, self.m, y.device)
         s = stream if stream is not None else torch.cuda.current_stream(y.device)
         st = self._L.aecct_decode(self._h, y.data_ptr(), B, bits.data_ptr(), syn.data_ptr() if syn is not None else None,
                                   logits.data_ptr() if logits is not None else None, s.cuda_stream)
@@ -227,7 +244,7 @@ class Decoder:
 
     def decode_host(self, y: np.ndarray, want_syndrome: bool = True, want_logits: bool = True):
         """End-to-end call with host arrays: copies in, decodes, copies out, waits."""
-        y = np.ascontiguousarray(y, dtype=np.float32)
+        y = self._host_y(y)
         B = y.shape[0]
         bits = np.empty((B, self.n), np.uint8)
         syn = np.empty((B, self.m), np.uint8) if want_syndrome else None
@@ -241,7 +258,7 @@ class Decoder:
     def decode_host_noalloc(self, y: np.ndarray, want_syndrome: bool = True, want_logits: bool = True):
         """aecct_decode_host_noalloc: host arrays, device staging from the library's static scratch
         (no allocation).  Returns (status, bits, syndrome, logits); calls must not overlap."""
-        y = np.ascontiguousarray(y, dtype=np.float32)
+        y = self._host_y(y)
         B = y.shape[0]
         bits = np.empty((B, self.n), np.uint8)
         syn = np.empty((B, self.m), np.uint8) if want_syndrome else None
@@ -250,6 +267,12 @@ class Decoder:
                                                syn.ctypes.data if syn is not None else None,
                                                logits.ctypes.data if logits is not None else None, None)
         return st, bits, syn, logits
+
+    def _host_y(self, y) -> np.ndarray:
+        y = np.ascontiguousarray(y, dtype=np.float32)
+        if y.ndim != 2 or y.shape[1] != self.n:
+            raise ValueError(f"y must be a float32 array of shape [B, {self.n}]")
+        return y
 
     def synchronize(self) -> int:
         return self._L.aecct_synchronize(self._h)

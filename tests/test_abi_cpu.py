@@ -140,3 +140,24 @@ def test_calls_on_null_handle():
     assert L.aecct_synchronize(None) == A.AECCT_ERR_INVALID_ARG
     assert L.aecct_destroy(None) == A.AECCT_ERR_INVALID_ARG
     assert L.aecct_set_capture(None, 0, None, None, None, None) == A.AECCT_ERR_INVALID_ARG
+
+
+def test_caller_outputs_are_checked_before_the_kernel_writes_them():
+    torch = pytest.importorskip("torch")
+    cpu = torch.device("cpu")
+    B, n, m = 5, 31, 15
+    ok = (torch.empty((B, n), dtype=torch.uint8), torch.empty((B, m), dtype=torch.uint8), None)
+    assert A.check_outputs(ok, B, n, m, cpu)[0] is ok[0]
+    assert A.check_outputs((ok[0], None, torch.empty((B, n))), B, n, m, cpu)[2].shape == (B, n)
+    bad = [
+        (None, None, None),                                                         # bits are required
+        (torch.empty((B - 1, n), dtype=torch.uint8), None, None),                  # too few rows
+        (torch.empty((B, n), dtype=torch.int32), None, None),                      # wrong type
+        (ok[0], torch.empty((B, m + 1), dtype=torch.uint8), None),                 # syndrome too wide
+        (ok[0], None, torch.empty((B, n), dtype=torch.float64)),                   # logits type
+        (torch.empty((n, B), dtype=torch.uint8).t(), None, None),                  # not contiguous
+        (ok[0].to("meta"), None, None),                                            # another device
+    ]
+    for out in bad:
+        with pytest.raises(ValueError):
+            A.check_outputs(out, B, n, m, cpu)
