@@ -3,9 +3,9 @@
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl {cuda,reference}] [--workload KEY]
                   [--variant {aecct,ecct,fp-hpsa}]
 
-A step decodes one batch of the workload (default: Polar(64,32), d = 64, N = 6, 8 heads,
-B = 65,536 received words, BPSK/AWGN at Eb/N0 cycling over 4, 5, 6 dB) through the C ABI
-(aecct_decode).  Inputs are resident in HBM before the timed region; L2 is flushed between
+A step decodes one batch of the workload (default: BCH(63,36), d = 128, N = 10, 8 heads,
+B = 262,144 received words, BPSK/AWGN at Eb/N0 cycling over 4, 5, 6, 7 dB: the largest
+configuration, 92.8 T int ops per batch) through the C ABI (aecct_decode).  Inputs are resident in HBM before the timed region; L2 is flushed between
 steps by writing a 256 MB buffer outside the timed events.  One JSON line is printed by
 rank 0.  Under torchrun each rank decodes its own batch (weak scaling, no collective on the
 data path); the time is the maximum over ranks.
@@ -101,7 +101,37 @@ def work_per_word(w: I.Workload):
     return dict(int_ops=2 * 12 * T * d * d * N, io_bytes=4 * w.code.n + w.code.n + (w.code.n - w.code.k))
 
 
-ALU_PEAK_TOPS = 152 * 128 * 2.070e9 / 1e12  # 152 SMs x 128 fp32 lanes x 2070 MHz (an FMA is one op), T ops/s
+ALU_NOMINAL_TOPS = 152 * 128 * 2.070e9 / 1e12  # 152 SMs x 128 fp32 lanes x 2070 MHz (an FMA is one op), T ops/s
+
+
+def measured_alu_peak():
+    """The fp32 FMA rate measured on this device by the library's diagnostic kernel (scalar and
+    paired f32x2 instructions; the larger), in T ops/s, an FMA counting one op."""
+    from paper_2410_05911_gb300 import aecct
+
+    rates = {"scalar": aecct.selftest_fma_rate(False) / 1e12, "paired": aecct.selftest_fma_rate(True) / 1e12}
+    return max(rates.values()), rates
+
+
+def cpu_model() -> str:
+    """The host CPU's model name (lscpu, else /proc/cpuinfo, else the machine type)."""
+    import platform
+
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith("model name"):
+                    return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    return platform.machine()
 
 
 def alu_ops_per_word(code, model) -> float:
@@ -200,19 +230,35 @@ class ClockSampler:
         return dict(sm_mhz=float(np.median(sm)), sm_max_mhz=mx, reasons=sorted(reasons), samples=len(sm))
 
 
-def cpu_oracle_rate(model, y, budget_s: float = 12.0, chunk: int = 64, max_words: int = 8192):
-    """Oracle decode rate (words/s) on the host cores over a bounded prefix of y."""
+def cpu_oracle_rate(model, y, budget_s: float = 12.0, chunk: int = 64, max_words: int = 8192, threads: int = 0):
+    """Oracle decode rate (words/s) on the host cores over a bounded prefix of y; also returns the
+    oracle's outputs for the words it decoded (the parity sample)."""
     from oracle import oracle as O
 
-    cores = os.cpu_count() or 1
+    cores = threads or os.cpu_count() or 1
+    chunk = max(cores, chunk) if threads == 0 else chunk
     done, t0 = 0, time.perf_counter()
+    outs = []
     while done < min(max_words, y.shape[0]):
-        O.decode(model, y[done:done + chunk], nthreads=cores)
-        done += chunk
+        outs.append(O.decode(model, y[done:done + chunk], nthreads=cores))
+        done += min(chunk, y.shape[0] - done)
         if time.perf_counter() - t0 > budget_s:
             break
     dt = time.perf_counter() - t0
-    return done / dt, done, dt, cores
+    ref = {k: np.concatenate([o[k] for o in outs]) for k in ("bits", "syndrome", "logits")}
+    return done / dt, done, dt, cores, ref
+
+
+def parity_summary(gpu: dict, ref: dict) -> dict:
+    """GPU outputs against the oracle's on the same words: bit-exact logits and decisions, and
+    the tolerance criteria (|d logit| <= 2e-2; decisions equal except where |logit| < 0.05)."""
+    dl = np.abs(gpu["logits"].astype(np.float64) - ref["logits"].astype(np.float64))
+    differ = gpu["bits"] != ref["bits"]
+    return dict(words=int(ref["bits"].shape[0]), bits=int(ref["bits"].size),
+                logits_bit_exact=bool((gpu["logits"].view(np.int32) == ref["logits"].view(np.int32)).all()),
+                max_abs_dlogit=float(dl.max()), bits_differ=int(differ.sum()),
+                bits_differ_away_from_zero=int((differ & (np.abs(ref["logits"]) >= 0.05)).sum()),
+                syndromes_equal=bool((gpu["syndrome"] == ref["syndrome"]).all()))
 
 
 VARIANTS = {
@@ -296,6 +342,9 @@ def run_cuda(args, rank, world, local_rank):
     def step(i):
         dec.decode(ys[i % len(ys)], out=(bits, syn, None), stream=stream)
 
+    # the CUDA-core roofline's denominator, measured before the timed region
+    alu_peak, alu_rates = measured_alu_peak() if rank == 0 else (ALU_NOMINAL_TOPS, {})
+
     for i in range(args.warmup):
         step(i)
     torch.cuda.synchronize()
@@ -347,9 +396,11 @@ def run_cuda(args, rank, world, local_rank):
                   work="2*12*T*d^2*N ops per word on the bf16 tensor cores (AAP: exact integers; "
                        "full-precision linears: bf16 products); peak = measured bf16 dense burst")
     alu_tops = alu_ops_per_word(w.code, model) * B / kernel_s / 1e12
-    alu = dict(bound="alu", achieved=alu_tops, peak=ALU_PEAK_TOPS, unit="TFLOP/s", frac=alu_tops / ALU_PEAK_TOPS,
+    alu = dict(bound="alu", achieved=alu_tops, peak=alu_peak, unit="TFLOP/s", frac=alu_tops / alu_peak,
                work="algorithmic fp32 ops of the canonical forward pass per word (bench.alu_ops_per_word; an FMA "
-                    "is one op); peak = 152 SMs x 128 fp32 lanes x 2070 MHz (derived, not measured)")
+                    "is one op); peak = fp32 FMA rate measured on this GPU by aecct_selftest_fma_rate (the larger "
+                    f"of scalar {alu_rates['scalar']:.1f} and paired {alu_rates['paired']:.1f} T FMA/s; nominal "
+                    f"152 SMs x 128 lanes x 2070 MHz = {ALU_NOMINAL_TOPS:.1f})")
     # d <= 64: the fp32 work (HPSA, epilogues) binds; d = 128: the linear layers' contraction
     roof = dict(alu if w.d <= 64 else tensor)
     roof.update(traffic=args.traffic if args.traffic is not None else
@@ -358,10 +409,21 @@ def run_cuda(args, rank, world, local_rank):
                        f"{model.linear_mode}>",
                 other={k: v for k, v in (("tensor", tensor), ("alu", alu)) if v["bound"] != roof["bound"]})
     cpu = None
+    parity = None
     if not args.no_cpu_baseline:
-        rate, words, secs, cores = cpu_oracle_rate(model, ys_host[0], budget_s=args.cpu_budget)
-        cpu = dict(value=rate, unit=UNIT, cores=cores, kind="oracle",
-                   sample=f"first {words} words of the {w.ebn0_db[0]} dB batch ({secs:.1f} s)")
+        rate, words, secs, cores, ref = cpu_oracle_rate(model, ys_host[0], budget_s=args.cpu_budget)
+        rate1, words1, secs1, _, _ = cpu_oracle_rate(model, ys_host[0], budget_s=args.cpu_budget / 3, chunk=4,
+                                                      threads=1)
+        cpu = dict(value=rate, unit=UNIT, cores=cores, kind="oracle", cpu_model=cpu_model(),
+                   sample=f"first {words} words of the {w.ebn0_db[0]} dB batch ({secs:.1f} s, {cores} threads)",
+                   one_thread=dict(value=rate1, unit=UNIT, sample=f"first {words1} words ({secs1:.1f} s)"))
+        # the GPU's outputs on the oracle's sample, compared with the oracle's
+        g_bits, g_syn, g_logits = dec.decode(ys[0][:words])
+        torch.cuda.synchronize()
+        if dec.synchronize() != aecct.AECCT_OK:
+            raise RuntimeError("parity decode reported an error")
+        parity = parity_summary(dict(bits=g_bits.cpu().numpy(), syndrome=g_syn.cpu().numpy(),
+                                     logits=g_logits.cpu().numpy()), ref)
     line = dict(
         metric=METRIC, value=value, unit=UNIT, n_gpus=world, steps=args.steps, warmup=args.warmup,
         ms_per_step=1e3 * kernel_s, higher_is_better=True, scaling="weak", vs_baseline=None,
@@ -370,7 +432,7 @@ def run_cuda(args, rank, world, local_rank):
                     cluster_ctas=q["cluster_ctas"],
                     words_per_group=q["words_per_group"], l2="flushed between steps (256 MB write)",
                     info_gbit_s=value * w.code.k / 1e9, hbm_io_gbs=value * wk["io_bytes"] / 1e9),
-        e2e=e2e, roofline=roof, cpu_baseline=cpu, gpu_launches=args.steps, clocks=clk.summary())
+        e2e=e2e, roofline=roof, cpu_baseline=cpu, parity=parity, gpu_launches=args.steps, clocks=clk.summary())
     print(json.dumps(line), flush=True)
 
 
@@ -380,7 +442,7 @@ def main():
     ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="cuda", choices=["cuda", "reference"])
-    ap.add_argument("--workload", default="polar64_32", choices=sorted(I.WORKLOADS))
+    ap.add_argument("--workload", default="bch63_36", choices=sorted(I.WORKLOADS))
     ap.add_argument("--batch", type=int, default=0, help="override the batch size (0 = the workload's)")
     ap.add_argument("--variant", default="aecct", choices=sorted(VARIANTS),
                     help="; ".join(f"{k}: {v[2]}" for k, v in VARIANTS.items()))

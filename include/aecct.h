@@ -147,8 +147,8 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out);
  * B == 0 is a no-op.  y is expected finite: a NaN or infinity is not checked, and the words
  * it reaches get unspecified bits and logits (no value steers a memory access, so the
  * other words of the batch are unaffected).  Errors: INVALID_ARG (B < 0, NULL y/bits with
- * B > 0), CUDA, and TIMEOUT reported for an earlier decode on this handle whose kernel
- * stopped. */
+ * B > 0, or a current device other than the one the handle was created on), CUDA, and
+ * TIMEOUT reported for an earlier decode on this handle whose kernel stopped. */
 int aecct_decode(aecct_handle *h, const float *y_dev, int64_t B, uint8_t *bits_dev, uint8_t *syndrome_dev,
                  float *logits_dev, void *cuda_stream);
 
@@ -176,6 +176,9 @@ int aecct_decode_host(aecct_handle *h, const float *y_host, int64_t B, uint8_t *
  *   the staging needs no clearing (y is copied in, every output element is written).
  *   Concurrency: every call uses the same array, so calls that overlap in time (two host threads,
  *   or two streams whose work interleaves on the device) race; serialise them.
+ *   Device: the current device must be the one the handle was created on (the array used is the
+ *   current device's), else AECCT_ERR_INVALID_ARG.
+ * An earlier asynchronous aecct_decode on the handle reports its status first, as in aecct_decode.
  * The call waits for its stream and returns the decode status (AECCT_ERR_TIMEOUT as
  * aecct_synchronize reports it). */
 #define AECCT_NOALLOC_SCRATCH_BYTES (4u << 20)
@@ -228,6 +231,13 @@ const char *aecct_last_error(void);
  */
 int aecct_selftest_mma(const int8_t *a_host, const int8_t *b_host, int32_t K, int32_t N, float *out_host);
 int aecct_selftest_timeout(int64_t limit_cycles, int32_t *status_host);
+
+/* aecct_selftest_fma_rate: the measured fp32 fused multiply-add rate of the current device, the
+ * denominator of the CUDA-core roofline that the benchmark reports.  A grid of 4 CTAs of 512
+ * threads per SM runs 8 independent FMA chains per thread, as scalar fma.rn.f32 (paired = 0) or
+ * as paired fma.rn.f32x2 instructions (paired = 1, two FMAs each); *fma_per_s receives the best
+ * of three timed launches (CUDA events), in FMAs per second.  Clocks are left as they are. */
+int aecct_selftest_fma_rate(int32_t paired, double *fma_per_s);
 
 #ifdef __cplusplus
 }

@@ -25,7 +25,7 @@ AECCT_ERR_NO_DEVICE = -6
 EXPORTED_SYMBOLS = (
     "aecct_create", "aecct_decode", "aecct_decode_host", "aecct_synchronize", "aecct_set_capture",
     "aecct_query", "aecct_destroy", "aecct_status_string", "aecct_last_error", "aecct_selftest_mma",
-    "aecct_selftest_timeout", "aecct_decode_host_noalloc",
+    "aecct_selftest_timeout", "aecct_decode_host_noalloc", "aecct_selftest_fma_rate",
 )
 
 
@@ -83,6 +83,7 @@ def load(build_if_missing: bool = True):
     L.aecct_last_error.restype = ctypes.c_char_p
     L.aecct_selftest_mma.argtypes = [P, P, I32, I32, P]
     L.aecct_selftest_timeout.argtypes = [I64, ctypes.POINTER(I32)]
+    L.aecct_selftest_fma_rate.argtypes = [I32, ctypes.POINTER(ctypes.c_double)]
     for name in EXPORTED_SYMBOLS:
         fn = getattr(L, name)
         if fn.restype is None or fn.restype is ctypes.c_int:
@@ -313,3 +314,10 @@ def selftest_timeout(limit_cycles: int) -> int:
     st = ctypes.c_int32(99)
     _check(load().aecct_selftest_timeout(int(limit_cycles), ctypes.byref(st)), "aecct_selftest_timeout")
     return st.value
+
+
+def selftest_fma_rate(paired: bool) -> float:
+    """Measured fp32 FMAs per second of the current device (scalar or paired f32x2 instructions)."""
+    v = ctypes.c_double()
+    _check(load().aecct_selftest_fma_rate(1 if paired else 0, ctypes.byref(v)), "aecct_selftest_fma_rate")
+    return v.value

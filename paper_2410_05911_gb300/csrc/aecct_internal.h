@@ -224,5 +224,6 @@ cudaError_t prepare_decode_kernel(int cluster_ctas, int *max_active_clusters);
 // api.cu diagnostics kernels live in selftest.cu
 cudaError_t run_selftest_mma(const int8_t *a_host, const int8_t *b_host, int K, int N, float *out_host);
 cudaError_t run_selftest_timeout(long long limit_cycles, int *status_host);
+cudaError_t run_selftest_fma_rate(bool paired, double *fma_per_s);
 
 }  // namespace aecct

@@ -637,6 +637,20 @@ static DecodeParams decode_params(const aecct_handle *h, int64_t B, const float 
   return p;
 }
 
+// The handle's model, plan and status word live on the device that was current at create; a
+// decode launched while another device is current would read them from the wrong GPU.
+static int check_device(const aecct_handle *h, const char *who) {
+  int dev = -1;
+  const cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev != h->device) {
+    g_last_error = std::string(who) + ": the current device is " + std::to_string(dev) +
+                   ", the handle was created on device " + std::to_string(h->device);
+    return AECCT_ERR_INVALID_ARG;
+  }
+  return AECCT_OK;
+}
+
 static int collect_status(aecct_handle *h, bool block) {
   if (!h->ev_pending) {
     const int s = h->pending_status;
@@ -661,6 +675,7 @@ int aecct_decode(aecct_handle *h, const float *y_dev, int64_t B, uint8_t *bits_d
   if (!h || B < 0) return AECCT_ERR_INVALID_ARG;
   if (B == 0) return AECCT_OK;
   if (!y_dev || !bits_dev) return AECCT_ERR_INVALID_ARG;
+  if (const int rc = check_device(h, "aecct_decode")) return rc;
   cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
   const int prev = collect_status(h, false);
   if (prev != AECCT_OK) return prev;
@@ -685,6 +700,7 @@ int aecct_decode_host(aecct_handle *h, const float *y_host, int64_t B, uint8_t *
   if (!h || B < 0) return AECCT_ERR_INVALID_ARG;
   if (B == 0) return AECCT_OK;
   if (!y_host || !bits_host) return AECCT_ERR_INVALID_ARG;
+  if (const int rc = check_device(h, "aecct_decode_host")) return rc;
   cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
   cudaError_t e;
   if (B > h->stage_B) {
@@ -730,9 +746,13 @@ int aecct_decode_host_noalloc(aecct_handle *h, const float *y_host, int64_t B, u
   if (!h || B < 0) return AECCT_ERR_INVALID_ARG;
   if (B == 0) return AECCT_OK;
   if (!y_host || !bits_host) return AECCT_ERR_INVALID_ARG;
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  // the scratch used is the current device's, so the current device must be the handle's
+  if (const int rc = check_device(h, "aecct_decode_host_noalloc")) return rc;
+  // an earlier asynchronous aecct_decode on this handle reports its status first, as in
+  // aecct_decode
+  if (const int prev = collect_status(h, false)) return prev;
+  const int dev = h->device;
+  cudaError_t e;
   if (dev < 0 || dev >= kNoAllocMaxDevices) {
     g_last_error = "aecct_decode_host_noalloc: device index beyond the per-device table";
     return AECCT_ERR_UNSUPPORTED;
@@ -743,8 +763,16 @@ int aecct_decode_host_noalloc(aecct_handle *h, const float *y_host, int64_t B, u
       return cuda_fail(e, "cudaGetSymbolAddress (aecct_decode_host_noalloc scratch)");
     g_noalloc_base[dev] = base;
   }
-  // layout: status word | y | bits | syndromes | logits, each part on a 256-byte boundary
-  const size_t n = static_cast<size_t>(h->n), m = static_cast<size_t>(h->m), b = static_cast<size_t>(B);
+  // layout: status word | y | bits | syndromes | logits, each part on a 256-byte boundary.  A word
+  // takes at least 5n bytes (y and bits), so a B beyond scratch / 5n is refused before any size
+  // product is formed (no size_t wrap-around for huge B).
+  const size_t n = static_cast<size_t>(h->n), m = static_cast<size_t>(h->m);
+  if (static_cast<uint64_t>(B) > AECCT_NOALLOC_SCRATCH_BYTES / (5u * n)) {
+    g_last_error = "aecct_decode_host_noalloc: B = " + std::to_string(B) + " words need more than the " +
+                   std::to_string(AECCT_NOALLOC_SCRATCH_BYTES) + "-byte static scratch holds";
+    return AECCT_ERR_INVALID_ARG;
+  }
+  const size_t b = static_cast<size_t>(B);
   const size_t off_y = 256, off_bits = off_y + round256(sizeof(float) * b * n), off_syn = off_bits + round256(b * n);
   const size_t off_log = off_syn + (syndrome_host ? round256(b * m) : 0);
   const size_t end = off_log + (logits_host ? round256(sizeof(float) * b * n) : 0);
@@ -835,6 +863,12 @@ int aecct_selftest_timeout(int64_t limit_cycles, int32_t *status_host) {
   if (e != cudaSuccess) return cuda_fail(e, "selftest timeout");
   *status_host = st == 1 ? AECCT_ERR_TIMEOUT : (st == 0 ? AECCT_OK : AECCT_ERR_CUDA);
   return AECCT_OK;
+}
+
+int aecct_selftest_fma_rate(int32_t paired, double *fma_per_s) {
+  if (!fma_per_s || (paired != 0 && paired != 1)) return AECCT_ERR_INVALID_ARG;
+  const cudaError_t e = run_selftest_fma_rate(paired != 0, fma_per_s);
+  return e == cudaSuccess ? AECCT_OK : cuda_fail(e, "selftest fma rate");
 }
 
 }  // extern "C"

@@ -164,8 +164,7 @@ struct Ctl {
 static __device__ __noinline__ bool wait_bar_slow(const Ctl c, uint32_t bar, uint32_t parity, bool cluster_scope) {
   const long long t0 = clock64();
   while (true) {
-    for (int i = 0; i < 32; ++i)
-      if (cluster_scope ? mbar_try_wait_acq_cluster(bar, parity) : mbar_try_wait(bar, parity)) return true;
+    if (cluster_scope ? mbar_try_wait_acq_cluster(bar, parity) : mbar_try_wait(bar, parity)) return true;
     if (*c.abort) return false;
     if (clock64() - t0 > c.limit) {
       *c.abort = 1;
@@ -185,11 +184,16 @@ __device__ __forceinline__ bool wait_bar_warp(const Ctl c, uint32_t bar, uint32_
   if ((threadIdx.x & 31) == 0) ok = wait_bar(c, bar, parity, cluster_scope);
   return __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
 }
-// Teardown wait: ignores the abort flag (used to drain copies / MMAs in flight), still bounded.
+// Teardown wait: ignores the abort flag (used to drain copies / MMAs in flight).  Its bound is
+// fixed (about a second) and independent of the caller's wait limit: the copies and MMAs it waits
+// for were all issued on the live path (the issuer stops issuing once a wait gave up), so they
+// finish in microseconds, and a short caller limit must not let the kernel exit while a copy can
+// still land in its shared memory.
+constexpr long long kDrainLimitCycles = 1LL << 31;
 static __device__ __noinline__ bool wait_bar_drain(const Ctl c, uint32_t bar, uint32_t parity) {
   const long long t0 = clock64();
   while (!mbar_try_wait(bar, parity)) {
-    if (clock64() - t0 > c.limit) {
+    if (clock64() - t0 > kDrainLimitCycles) {
       atomicOr(c.err, 1);
       return false;
     }
@@ -662,6 +666,13 @@ struct Issuer {
   Ctl ctl;
   uint32_t *n_issued;  // copies started so far (read by the teardown drain)
 
+  // false once a wait of this CTA gave up: from then on nothing more is issued, so that the
+  // teardown drain knows every copy and MMA in flight (only this warp's lane 0 sets the flag, in
+  // a wait followed by __syncwarp, so every lane reads the same value)
+  __device__ __forceinline__ bool live() const { return *ctl.abort == 0; }
+  __device__ __forceinline__ void commit(uint32_t bar) const {
+    if (live()) mma_commit_warp(bar);
+  }
   __device__ __forceinline__ uint32_t bar_full(int s) const { return sb + L::kOffBar + 8 * s; }
   __device__ __forceinline__ uint32_t bar_empty(int s) const { return sb + L::kOffBar + 8 * (S + s); }
   __device__ __forceinline__ uint32_t bar_op() const { return sb + L::kOffBar + 16 * S; }
@@ -680,6 +691,7 @@ struct Issuer {
   template <int P>
   __device__ __forceinline__ void copy(const uint8_t *src) const {
     constexpr ChunkDesc c = W::chunk(P);
+    if (!live()) return;
     bulk_g2s_expect_warp(sb + L::kOffW + (P % S) * W::kStageBytes, src + c.off, c.bytes, bar_full(P % S));
     if ((threadIdx.x & 31) == 0) ++*n_issued;
   }
@@ -709,13 +721,15 @@ struct Issuer {
       }
       wait(bar_full(p % S), (p / S) & 1);
       const uint32_t b_tile = sb + L::kOffW + (p % S) * W::kStageBytes;
+      if (live()) {
 #pragma unroll 1
-      for (int ks = 0; ks < c.kcols / 16; ++ks) {
-        const uint32_t kabs = c.k0 + 16u * ks;
-        mma_bf16_warp(tmem + c.n0, make_sdesc(sb + a_tile + (kabs / 8u) * 128u, 128u, a_sbo),
-                      make_sdesc(b_tile + ks * 256u, 128u, b_sbo), idesc, kabs > 0 ? 1u : 0u);
+        for (int ks = 0; ks < c.kcols / 16; ++ks) {
+          const uint32_t kabs = c.k0 + 16u * ks;
+          mma_bf16_warp(tmem + c.n0, make_sdesc(sb + a_tile + (kabs / 8u) * 128u, 128u, a_sbo),
+                        make_sdesc(b_tile + ks * 256u, 128u, b_sbo), idesc, kabs > 0 ? 1u : 0u);
+        }
       }
-      if constexpr (kRefillInGemm) mma_commit_warp(bar_empty(p % S));
+      if constexpr (kRefillInGemm) commit(bar_empty(p % S));
       chunk_mmas<G, J + 1>(w_cur);
     }
   }
@@ -739,7 +753,7 @@ struct Issuer {
     wait(bar_op(), G & 1);
     tc_fence_after();
     chunk_mmas<G, 0>(w_cur);
-    mma_commit_warp(bar_acc());
+    commit(bar_acc());
     // warp 0 alone waits for the accumulators; the other warps of the CTA wait in a named
     // barrier (no spinning), which warp 0 arrives at after the wait, before its copies
     wait(bar_acc(), G & 1);
@@ -784,6 +798,12 @@ struct Issuer<128, TASKS> {
     return sb + L::kOffBar + (id < 3 ? 8 * id : 16 * 3 + 7 * 8 + 8 * (id - 3));
   }
   __device__ __forceinline__ uint32_t bar_empty(int s) const { return sb + L::kOffBar + 8 * (3 + s); }
+  // false once a wait of this CTA gave up: nothing more is armed, copied or issued (see the
+  // generic issuer)
+  __device__ __forceinline__ bool live() const { return *ctl.abort == 0; }
+  __device__ __forceinline__ void commit(uint32_t b) const {
+    if (live()) mma_commit_warp(b);
+  }
   __device__ __forceinline__ uint32_t bar_op() const { return sb + L::kOffBar + 48; }
   __device__ __forceinline__ uint32_t bar_acc() const { return sb + L::kOffBar + 56; }
   // the accumulators are complete: let the CTA's other warps (waiting in wait_acc) go
@@ -815,6 +835,7 @@ struct Issuer<128, TASKS> {
   }
   // arm barrier `id` for `bytes` (one arrive), then the copies of chunks P0 .. P1-1 complete it
   __device__ __forceinline__ void arm(int id, uint32_t bytes) const {
+    if (!live()) return;
     asm volatile(
         "{\n\t.reg .pred e;\n\t.reg .b32 r;\n\telect.sync r|e, 0xffffffff;\n\t"
         "@e mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n\t}" ::"r"(bar(id)),
@@ -824,6 +845,10 @@ struct Issuer<128, TASKS> {
   }
   template <int P0, int P1>
   __device__ __forceinline__ void copies(const uint8_t *src) const {
+    if (live()) copies_live<P0, P1>(src);
+  }
+  template <int P0, int P1>
+  __device__ __forceinline__ void copies_live(const uint8_t *src) const {
     if constexpr (P0 < P1) {
       constexpr ChunkDesc c = W::chunk(P0);
       constexpr Slot s = slot(P0);
@@ -833,7 +858,7 @@ struct Issuer<128, TASKS> {
               sb + s.off),
           "l"(src + c.off), "r"(c.bytes), "r"(bar(s.id))
           : "memory");
-      copies<P0 + 1, P1>(src);
+      copies_live<P0 + 1, P1>(src);
     }
   }
   template <int P>
@@ -859,6 +884,7 @@ struct Issuer<128, TASKS> {
     constexpr uint32_t b_sbo = (c.kcols / 8u) * 128u;
     constexpr uint32_t idesc = make_idesc_bf16(128, c.nrows);
     const uint32_t b_tile = sb + slot(P).off;
+    if (!live()) return;
 #pragma unroll 1
     for (int ks = 0; ks < c.kcols / 16; ++ks) {
       const uint32_t kabs = c.k0 + 16u * ks;
@@ -880,6 +906,7 @@ struct Issuer<128, TASKS> {
     constexpr uint32_t b_sbo = (c.kcols / 8u) * 128u;  // row groups 16..31 continue in chunk P + 1
     constexpr uint32_t idesc = make_idesc_bf16(128, 256);
     const uint32_t b_tile = sb + slot(P).off;
+    if (!live()) return;
 #pragma unroll 1
     for (int ks = 0; ks < c.kcols / 16; ++ks) {
       const uint32_t kabs = c.k0 + 16u * ks;
@@ -900,7 +927,7 @@ struct Issuer<128, TASKS> {
       mmas_pair<0, 2>();  // N tiles 0 and 1, K 64..127
       mmas<0, 4>();       // N tile 2
       mmas<0, 5>();
-      mma_commit_warp(bar_acc());
+      commit(bar_acc());
       wait(bar_acc(), 0);
       release_acc();
     } else if constexpr (G == 1) {
@@ -908,7 +935,7 @@ struct Issuer<128, TASKS> {
       mmas<1, 6>();
       wait(bar(1), parity<7>(lp));
       mmas<1, 7>();
-      mma_commit_warp(bar_acc());
+      commit(bar_acc());
       // FFN1 weights into region U: a one-CTA cluster has finished reading its K/V (every warp
       // published the O operand); a larger cluster stages them at FFN1 instead, so that the O
       // epilogue overlaps the peers' attention.  FFN2 chunk 18 into W2 (last read by the
@@ -933,7 +960,7 @@ struct Issuer<128, TASKS> {
       mmas_pair<2, 10>();
       mmas_pair<2, 12>();
       mmas_pair<2, 14>();
-      mma_commit_warp(bar_acc());
+      commit(bar_acc());
       wait(bar_acc(), 0);
       release_acc();
       copy1<19>(w_cur);  // the operand tile is free: FFN1's MMAs are done
@@ -941,13 +968,13 @@ struct Issuer<128, TASKS> {
     } else {
       wait(bar(0), parity<16>(lp));
       mmas<3, 16>();
-      mma_commit_warp(bar_empty(0));
+      commit(bar_empty(0));
       wait(bar(1), parity<17>(lp));
       mmas<3, 17>();
-      mma_commit_warp(bar_empty(1));
+      commit(bar_empty(1));
       wait(bar(2), parity<18>(lp));
       mmas<3, 18>();
-      mma_commit_warp(bar_empty(2));
+      commit(bar_empty(2));
       wait(bar(4), parity<19>(lp));
       mmas<3, 19>();
       wait(bar(5), parity<20>(lp));
@@ -966,7 +993,7 @@ struct Issuer<128, TASKS> {
       mmas<3, 22>();
       wait(bar(2), parity<23>(lp));
       mmas<3, 23>();
-      mma_commit_warp(bar_acc());
+      commit(bar_acc());
       wait(bar_acc(), 1);
       release_acc();
       if (has_next) stage_qkv_o(w_next);  // region U and W0, W1 are free again

@@ -105,6 +105,79 @@ __global__ void selftest_timeout_kernel(long long limit, int *status) {
   if (threadIdx.x == 0) *status = done ? 0 : 1;
 }
 
+// fp32 fused multiply-add rate: every thread runs 8 independent FMA chains (scalar fma.rn.f32,
+// or paired fma.rn.f32x2 with two FMAs per instruction) for `iters` steps; the values stay in
+// [0, 1] (x <- x * 0.5 + 0.25 converges to 0.5), and a comparison nothing satisfies keeps the
+// chains from being removed
+template <bool PAIRED>
+__global__ void __launch_bounds__(512) selftest_fma_kernel(int iters, float *sink) {
+  const float s = 0.5f, c = 0.25f;
+  if constexpr (PAIRED) {
+    uint64_t a[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const float v = 0.001f * static_cast<float>(threadIdx.x + i);
+      asm("mov.b64 %0, {%1, %2};" : "=l"(a[i]) : "f"(v), "f"(-v));
+    }
+    uint64_t sc, cc;
+    asm("mov.b64 %0, {%1, %1};" : "=l"(sc) : "f"(s));
+    asm("mov.b64 %0, {%1, %1};" : "=l"(cc) : "f"(c));
+    for (int it = 0; it < iters; ++it) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) asm volatile("fma.rn.f32x2 %0, %0, %1, %2;" : "+l"(a[i]) : "l"(sc), "l"(cc));
+    }
+    float t = 0.0f;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      float lo, hi;
+      asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(a[i]));
+      t += lo + hi;
+    }
+    if (t == -1.0f) sink[blockIdx.x * blockDim.x + threadIdx.x] = t;
+  } else {
+    float a[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) a[i] = 0.001f * static_cast<float>(threadIdx.x + i);
+    for (int it = 0; it < iters; ++it) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) asm volatile("fma.rn.f32 %0, %0, %1, %2;" : "+f"(a[i]) : "f"(s), "f"(c));
+    }
+    float t = 0.0f;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) t += a[i];
+    if (t == -1.0f) sink[blockIdx.x * blockDim.x + threadIdx.x] = t;
+  }
+}
+
+cudaError_t run_selftest_fma_rate(bool paired, double *fma_per_s) {
+  int dev = 0, sms = 0;
+  cudaError_t e;
+  if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+  if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+  const int blocks = 4 * sms, threads = 512, iters = 1 << 15;
+  float *sink = nullptr;
+  cudaEvent_t t0 = nullptr, t1 = nullptr;
+  float best_ms = 0.0f;
+  if ((e = cudaMalloc(&sink, sizeof(float) * blocks * threads)) != cudaSuccess) return e;
+  if ((e = cudaEventCreate(&t0)) != cudaSuccess || (e = cudaEventCreate(&t1)) != cudaSuccess) goto done;
+  for (int rep = 0; rep < 4; ++rep) {  // the first launch warms up
+    if ((e = cudaEventRecord(t0)) != cudaSuccess) goto done;
+    if (paired) selftest_fma_kernel<true><<<blocks, threads>>>(iters, sink);
+    else selftest_fma_kernel<false><<<blocks, threads>>>(iters, sink);
+    if ((e = cudaGetLastError()) != cudaSuccess) goto done;
+    if ((e = cudaEventRecord(t1)) != cudaSuccess || (e = cudaEventSynchronize(t1)) != cudaSuccess) goto done;
+    float ms = 0.0f;
+    if ((e = cudaEventElapsedTime(&ms, t0, t1)) != cudaSuccess) goto done;
+    if (rep > 0 && (best_ms == 0.0f || ms < best_ms)) best_ms = ms;
+  }
+  *fma_per_s = static_cast<double>(blocks) * threads * iters * 8.0 * (paired ? 2.0 : 1.0) / (best_ms * 1e-3);
+done:
+  if (t0) cudaEventDestroy(t0);
+  if (t1) cudaEventDestroy(t1);
+  cudaFree(sink);
+  return e;
+}
+
 cudaError_t run_selftest_mma(const int8_t *a_host, const int8_t *b_host, int K, int N, float *out_host) {
   int8_t *da = nullptr, *db = nullptr;
   float *dout = nullptr;

@@ -5,9 +5,9 @@ not bit equality:
 
 * block 0's Q, K, V sums, whose bf16 inputs are the same on both sides, agree with the oracle's
   exact sums rounded once to within the fp32 summation bound K 2^-23 sum_i |x_i w_i|;
-* the logits agree within the float tolerance 2e-2 (relative to the largest logit), their median
-  difference is 20 times smaller, and a decoded bit may differ only where the oracle's logit is within
-  that difference of zero;
+* the logits agree within the float tolerance 2e-2 absolute, and the decoded bits are identical
+  except where the oracle's logit is below 0.05 in magnitude, on at least 99.99% of the bits
+  (each case decodes at least 10^4 bits);
 * the syndromes are those of the decoded bits.
 Also the ECCT configuration as a whole: GELU, the code-aware mask on every head (mask_mode 1)
 and full-precision linears.
@@ -54,7 +54,7 @@ def test_full_precision_linears(case):
     mask_mode = var.pop("mask_mode", 0)
     model = I.random_model(code, d, layers, seed=91, full_precision=True, **var)
     model.mask_mode = mask_mode
-    B, capB = 9, 3
+    B, capB = -(-10000 // code.n), 3
     y = I.channel_batch(code, B, 3.0, seed=7).y
     r = O.decode(model, y, cap_B=capB)
     ref = r["logits"].astype(np.float64)
@@ -75,10 +75,10 @@ def test_full_precision_linears(case):
         assert (np.abs(got - want) <= bound).all(), f"mode {mode}: block-0 sums outside the fp32 bound"
         lg = logits.cpu().numpy().astype(np.float64)
         diff = np.abs(lg - ref)
-        scale = 1.0 + np.abs(ref).max()
-        assert diff.max() <= 2e-2 * scale and np.median(diff) <= 1e-3 * scale, f"mode {mode}: {diff.max()}"
+        assert diff.max() <= 2e-2, f"mode {mode}: max |d logit| {diff.max():.3e}, median {np.median(diff):.2e}"
         b = bits.cpu().numpy()
         flip = b != r["bits"]
-        assert (np.abs(ref[flip]) <= diff.max()).all(), f"mode {mode}: a bit differs away from a zero logit"
+        away = flip & (np.abs(ref) >= 0.05)
+        assert away.mean() <= 1e-4, f"mode {mode}: {int(away.sum())} of {flip.size} bits differ where |logit| >= 0.05"
         assert (syn.cpu().numpy() == (b.astype(np.int64) @ model.H.T.astype(np.int64)) % 2).all()
         dec.close()

@@ -129,6 +129,29 @@ def test_full_size_batch_sampled_exact(key):
     # decoding statistics are only reported: synthetic weights carry no trained meaning
 
 
+POINTS = [(key, e) for key in KEYS for e in I.workload(key).ebn0_db]
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("key,ebn0", POINTS, ids=[f"{k}-{e}dB" for k, e in POINTS])
+def test_every_ebn0_point_against_oracle(key, ebn0):
+    # at least 10^4 bits per configuration point (so that the 99.99% decision rule is measurable),
+    # in the default launch configuration: bit-exact logits, decisions and syndromes, which meet
+    # the float criteria (|d logit| <= 2e-2, decisions equal where |logit| >= 0.05) with margin
+    dec, model = decoder(key)
+    w = I.workload(key)
+    B = -(-10000 // w.code.n)
+    ch = I.channel_batch(w.code, B, ebn0, seed=9000 + int(10 * ebn0))
+    g = gpu_decode(dec, ch.y)
+    r = O.decode(model, ch.y)
+    assert g["bits"].size >= 10000
+    dl = np.abs(g["logits"].astype(np.float64) - r["logits"])
+    assert dl.max() <= 2e-2
+    differ = g["bits"] != r["bits"]
+    assert (differ & (np.abs(r["logits"]) >= 0.05)).mean() <= 1e-4
+    assert_same(g, r, f"{key} {ebn0} dB")
+
+
 @pytest.mark.gpu
 def test_edge_batches_and_optional_outputs():
     dec, model = decoder("polar64_32")

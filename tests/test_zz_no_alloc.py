@@ -64,3 +64,23 @@ def test_noalloc_limit_and_refusal():
     st, _, _, _ = dec.decode_host_noalloc(yb, want_logits=False)
     assert st == A.AECCT_OK
     dec.close()
+
+
+@pytest.mark.gpu
+def test_noalloc_reports_timeout_then_recovers():
+    # the status word read back from the scratch: a handle whose waits give up after one cycle
+    # reports AECCT_ERR_TIMEOUT; the word is cleared before the next call, which then succeeds
+    key = "polar64_32"
+    w = I.workload(key)
+    model = I.workload_model(key)
+    y = I.channel_batch(w.code, 2048, w.ebn0_db[0], seed=13).y
+    short = A.Decoder(model, wait_limit_cycles=1)
+    st, _, _, _ = short.decode_host_noalloc(y)
+    assert st == A.AECCT_ERR_TIMEOUT
+    short.close()
+    dec = A.Decoder(model)
+    bits, syn, logits = dec.decode_host(y)
+    st, b2, s2, l2 = dec.decode_host_noalloc(y)
+    assert st == A.AECCT_OK
+    assert (b2 == bits).all() and (s2 == syn).all() and (l2.view(np.int32) == logits.view(np.int32)).all()
+    dec.close()
