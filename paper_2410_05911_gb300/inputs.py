@@ -377,6 +377,56 @@ def ternary_scale_for_zero_fraction(zero_frac: float, d_in: int) -> float:
     return 2.0 * sigma * _inv_norm_cdf(0.5 * (1.0 + zero_frac))
 
 
+@dataclasses.dataclass
+class SpeParams:
+    """Parameters of the spectral positional encoding (Sec. 4.3): W_{2->d_SPE} and the SPE's
+    multi-head self-attention projections (standard form, no biases)."""
+    w_pe: np.ndarray   # [2, d_spe]
+    wq: np.ndarray     # [heads, d_spe, d_e]
+    wk: np.ndarray     # [heads, d_spe, d_e]
+    wv: np.ndarray     # [heads, d_spe, d_e]
+    wo: np.ndarray     # [d_spe, d_spe]
+
+
+def spe_params(H: np.ndarray, d_spe: int, seed: int, heads: int = 4) -> SpeParams:
+    """Seeded SPE parameters standing in for learned ones (float64).  The eigenvalue row of
+    W_{2->d_SPE} is scaled by 1 / (2 max degree), a bound on the Laplacian's largest eigenvalue,
+    and the eigenvector row by sqrt(T) (eigenvector entries are about 1/sqrt(T)), so that both
+    columns of Phi contribute O(1) values; the projections are N(0, 1/d_SPE)."""
+    if d_spe % heads:
+        raise ValueError("d_spe must be a multiple of the SPE heads")
+    m, n = H.shape
+    T = n + m
+    deg = max(int((H != 0).sum(0).max()), int((H != 0).sum(1).max()))
+    rng = np.random.Generator(np.random.PCG64(seed))
+    d_e = d_spe // heads
+    w_pe = rng.standard_normal((2, d_spe))
+    w_pe[0] /= 2.0 * deg
+    w_pe[1] *= math.sqrt(T)
+    s = 1.0 / math.sqrt(d_spe)
+    wq = rng.standard_normal((heads, d_spe, d_e)) * s
+    wk = rng.standard_normal((heads, d_spe, d_e)) * s
+    wv = rng.standard_normal((heads, d_spe, d_e)) * s
+    wo = rng.standard_normal((d_spe, d_spe)) * s
+    return SpeParams(w_pe, wq, wk, wv, wo)
+
+
+_SPE_CACHE: Dict[tuple, np.ndarray] = {}
+
+
+def spe_for_code(H: np.ndarray, d_spe: int, seed: int) -> np.ndarray:
+    """The model's SPE table: the host precompute of Sec. 4.3 (paper_2410_05911_gb300.spe) on
+    seeded SPE parameters, cached per (H, d_spe, seed) within the process."""
+    if d_spe == 0:
+        return np.zeros((H.shape[0] + H.shape[1], 0), np.float32)
+    key = (H.shape, H.tobytes(), d_spe, seed)
+    if key not in _SPE_CACHE:
+        from . import spe
+
+        _SPE_CACHE[key] = spe.spe_table(H, spe_params(H, d_spe, seed))
+    return _SPE_CACHE[key].copy()
+
+
 def random_model(
     code: LinearCode,
     d: int,
@@ -398,8 +448,9 @@ def random_model(
     the rest +1/-1 with equal probability; the scale is the one the paper's quantizer
     would produce on N(0, 1/d_in) weights at that zero fraction, times a per-tensor jitter
     in [0.9, 1.1].  Biases and LayerNorm parameters are small random values so that an
-    indexing mistake changes the output.  The SPE table is a seeded N(0,1) table standing
-    in for the learned one (at inference it is a fixed table).
+    indexing mistake changes the output.  The SPE table is the Tanner-graph spectral encoding
+    of Sec. 4.3 computed on the host from H with seeded SPE parameters (spe_for_code); at
+    inference it is a fixed table.
 
     binary=True draws the binary-weight variant (App. D): every weight is +1 or -1 and the
     per-tensor scale is the mean |W| of N(0, 1/d_in) weights, sqrt(2 / (pi d_in)), times the
@@ -446,7 +497,7 @@ def random_model(
     ln_gamma = (1.0 + 0.1 * rng.standard_normal((n_layers, 2, d))).astype(np.float32)
     ln_beta = (0.1 * rng.standard_normal((n_layers, 2, d))).astype(np.float32)
     emb = rng.standard_normal((T, d - d_spe)).astype(np.float32)
-    spe = rng.standard_normal((T, d_spe)).astype(np.float32)
+    spe = spe_for_code(code.H, d_spe, seed + 7919)
     w_d1 = (rng.standard_normal(d) / math.sqrt(d)).astype(np.float32)
     b_d1 = float(np.float32(0.1 * rng.standard_normal()))
     w_out = (2.0 * rng.standard_normal((T, code.n)) / math.sqrt(T)).astype(np.float32)
