@@ -65,8 +65,12 @@ typedef struct aecct_handle aecct_handle; /* opaque */
  *   attention_mode 0 = choose automatically; 1 = per-row neighbour lists (any cluster size);
  *                 2 = warp tasks over shared key sets (one CTA per group; d <= 64 with at most
  *                 128 tokens, or d = 128 with alpha_mode 0 and at most 128 rows once the checks'
- *                 rows start on the first 32-row boundary after the variables).  Every mode
- *                 computes the same results bit for bit.
+ *                 rows start on the first 32-row boundary after the variables);
+ *                 3 = per-row neighbour lists over per-head staged rows (d = 128, at most 640
+ *                 token rows per group and 256 keys per row): head by head, the group's K and V
+ *                 rows are gathered from every CTA of the cluster into local shared memory, and
+ *                 the 4 threads of a row share its keys.  The default for d = 128 when a group
+ *                 spans more than one CTA.  Every mode computes the same results bit for bit.
  *   mask_mode     0 = HPSA (Sec. 4.2): heads [0, h_first) first ring, the rest second ring;
  *                 1 = the ECCT code-aware mask (Sec. 3) for every head: the union of the first
  *                 and second rings (which contains each node itself).  Other values are rejected.
@@ -205,7 +209,7 @@ int aecct_set_capture(aecct_handle *h, int64_t cap_B, int8_t *q_dev, int32_t *ac
 /* Launch facts of the handle (for benchmarks): CTAs per codeword group, codewords per
  * group, the number of clusters a decode launches at most, threads per CTA, dynamic
  * shared memory bytes per CTA, and the attention mode in use (1 = per-row lists,
- * 2 = warp tasks).  Any pointer may be NULL. */
+ * 2 = warp tasks, 3 = per-row lists over per-head staged rows).  Any pointer may be NULL. */
 int aecct_query(const aecct_handle *h, int32_t *cluster_ctas, int32_t *words_per_group, int32_t *max_clusters,
                 int32_t *threads_per_cta, int32_t *smem_bytes, int32_t *attention_mode);
 

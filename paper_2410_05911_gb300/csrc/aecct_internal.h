@@ -213,13 +213,16 @@ struct SmemLayout {
   static constexpr uint32_t kRowCacheCol = (D == 128) ? 128u : 256u;
 };
 
-// decoder_kernel.cuh.  ACT: 0 = ReLU, 1 = GELU; LIN: 0 = AAP linears, 1 = full-precision (bf16)
-// linears.  Instantiated in decoder_kernel.cu (0, 0), decoder_kernel_gelu.cu (1, 0),
+// decoder_kernel.cuh.  ATT: 0 = per-row neighbour lists, 1 = warp tasks, 2 = per-row lists over
+// per-head staged rows (d = 128); ACT: 0 = ReLU, 1 = GELU; LIN: 0 = AAP linears, 1 = full-precision
+// (bf16) linears.  Instantiated in decoder_kernel.cu (0, 0), decoder_kernel_gelu.cu (1, 0),
 // decoder_kernel_fp.cu (0, 1) and decoder_kernel_fp_gelu.cu (1, 1).
-template <int D, bool TASKS, int ACT, int LIN>
+template <int D, int ATT, int ACT, int LIN>
 cudaError_t launch_decode(const DecodeParams &p, cudaStream_t stream);
-template <int D, bool TASKS, int ACT, int LIN>
+template <int D, int ATT, int ACT, int LIN>
 cudaError_t prepare_decode_kernel(int cluster_ctas, int *max_active_clusters);
+constexpr int kStagedMaxRows = 640;  // staged attention: rows of a group (128 bytes each in 80 KB)
+constexpr int kStagedMaxKeys = 256;  // staged attention: keys per row (TMEM columns [128, 384))
 
 // api.cu diagnostics kernels live in selftest.cu
 cudaError_t run_selftest_mma(const int8_t *a_host, const int8_t *b_host, int K, int N, float *out_host);

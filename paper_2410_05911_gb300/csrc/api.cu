@@ -33,7 +33,7 @@ struct aecct_handle {
   int n = 0, k = 0, T = 0, m = 0, d = 0, n_layers = 0, h_first = 0, d_spe = 0;
   int Tp = 0;  // token rows per codeword (T, or T plus padding rows)
   int C = 1, G = 1, max_clusters = 0;
-  bool tasks = false;  // warp-task attention (one CTA per group, d <= 64)
+  int att = 0;  // kernel attention path: 0 per-row lists, 1 warp tasks, 2 per-row lists over staged rows
   int alpha_mode = 0;  // 1 = one alpha per quantised matrix of a word
   int activation = 0;   // 0 = ReLU, 1 = GELU
   int linear_mode = 0;  // 0 = AAP ternary linears, 1 = full-precision (bf16) linears
@@ -125,7 +125,7 @@ int validate(const aecct_model_desc *d) {
   if (d->ffn_mult <= 0) return AECCT_ERR_INVALID_ARG;
   if (d->activation < 0 || d->activation > 1) return AECCT_ERR_INVALID_ARG;
   if (d->cluster_ctas < 0 || d->cluster_ctas > 64) return AECCT_ERR_INVALID_ARG;
-  if (d->attention_mode < 0 || d->attention_mode > 2) return AECCT_ERR_INVALID_ARG;
+  if (d->attention_mode < 0 || d->attention_mode > 3) return AECCT_ERR_INVALID_ARG;
   if (d->mask_mode < 0 || d->mask_mode > 1) return AECCT_ERR_INVALID_ARG;
   if (d->alpha_mode < 0 || d->alpha_mode > 1) return AECCT_ERR_INVALID_ARG;
   if (d->linear_mode < 0 || d->linear_mode > 1) return AECCT_ERR_INVALID_ARG;
@@ -195,34 +195,36 @@ int schedule_chunks(int D, ChunkDesc *out) {
   return D == 32 ? schedule_chunks_t<32>(out) : D == 64 ? schedule_chunks_t<64>(out) : schedule_chunks_t<128>(out);
 }
 
-// the compiled kernel for (d, attention mode, activation ACT, linear mode LIN)
+// the compiled kernel for (d, attention path ATT, activation ACT, linear mode LIN)
 template <int ACT, int LIN>
-cudaError_t prepare_any(int D, bool tasks, int C, int *max_clusters) {
-  if (tasks)
-    return D == 32   ? prepare_decode_kernel<32, true, ACT, LIN>(C, max_clusters)
-           : D == 64 ? prepare_decode_kernel<64, true, ACT, LIN>(C, max_clusters)
-                     : prepare_decode_kernel<128, true, ACT, LIN>(C, max_clusters);
-  if (D == 32) return prepare_decode_kernel<32, false, ACT, LIN>(C, max_clusters);
-  if (D == 64) return prepare_decode_kernel<64, false, ACT, LIN>(C, max_clusters);
-  return prepare_decode_kernel<128, false, ACT, LIN>(C, max_clusters);
+cudaError_t prepare_any(int D, int att, int C, int *max_clusters) {
+  if (att == 1)
+    return D == 32   ? prepare_decode_kernel<32, 1, ACT, LIN>(C, max_clusters)
+           : D == 64 ? prepare_decode_kernel<64, 1, ACT, LIN>(C, max_clusters)
+                     : prepare_decode_kernel<128, 1, ACT, LIN>(C, max_clusters);
+  if (att == 2) return prepare_decode_kernel<128, 2, ACT, LIN>(C, max_clusters);  // d = 128 only
+  if (D == 32) return prepare_decode_kernel<32, 0, ACT, LIN>(C, max_clusters);
+  if (D == 64) return prepare_decode_kernel<64, 0, ACT, LIN>(C, max_clusters);
+  return prepare_decode_kernel<128, 0, ACT, LIN>(C, max_clusters);
 }
 template <int ACT, int LIN>
-cudaError_t launch_any(int D, bool tasks, const DecodeParams &p, cudaStream_t stream) {
-  if (tasks)
-    return D == 32   ? launch_decode<32, true, ACT, LIN>(p, stream)
-           : D == 64 ? launch_decode<64, true, ACT, LIN>(p, stream)
-                     : launch_decode<128, true, ACT, LIN>(p, stream);
-  if (D == 32) return launch_decode<32, false, ACT, LIN>(p, stream);
-  if (D == 64) return launch_decode<64, false, ACT, LIN>(p, stream);
-  return launch_decode<128, false, ACT, LIN>(p, stream);
+cudaError_t launch_any(int D, int att, const DecodeParams &p, cudaStream_t stream) {
+  if (att == 1)
+    return D == 32   ? launch_decode<32, 1, ACT, LIN>(p, stream)
+           : D == 64 ? launch_decode<64, 1, ACT, LIN>(p, stream)
+                     : launch_decode<128, 1, ACT, LIN>(p, stream);
+  if (att == 2) return launch_decode<128, 2, ACT, LIN>(p, stream);
+  if (D == 32) return launch_decode<32, 0, ACT, LIN>(p, stream);
+  if (D == 64) return launch_decode<64, 0, ACT, LIN>(p, stream);
+  return launch_decode<128, 0, ACT, LIN>(p, stream);
 }
-cudaError_t prepare_variant(int act, int lin, int D, bool tasks, int C, int *max_clusters) {
-  if (lin == 0) return act == 0 ? prepare_any<0, 0>(D, tasks, C, max_clusters) : prepare_any<1, 0>(D, tasks, C, max_clusters);
-  return act == 0 ? prepare_any<0, 1>(D, tasks, C, max_clusters) : prepare_any<1, 1>(D, tasks, C, max_clusters);
+cudaError_t prepare_variant(int act, int lin, int D, int att, int C, int *max_clusters) {
+  if (lin == 0) return act == 0 ? prepare_any<0, 0>(D, att, C, max_clusters) : prepare_any<1, 0>(D, att, C, max_clusters);
+  return act == 0 ? prepare_any<0, 1>(D, att, C, max_clusters) : prepare_any<1, 1>(D, att, C, max_clusters);
 }
-cudaError_t launch_variant(int act, int lin, int D, bool tasks, const DecodeParams &p, cudaStream_t stream) {
-  if (lin == 0) return act == 0 ? launch_any<0, 0>(D, tasks, p, stream) : launch_any<1, 0>(D, tasks, p, stream);
-  return act == 0 ? launch_any<0, 1>(D, tasks, p, stream) : launch_any<1, 1>(D, tasks, p, stream);
+cudaError_t launch_variant(int act, int lin, int D, int att, const DecodeParams &p, cudaStream_t stream) {
+  if (lin == 0) return act == 0 ? launch_any<0, 0>(D, att, p, stream) : launch_any<1, 0>(D, att, p, stream);
+  return act == 0 ? launch_any<0, 1>(D, att, p, stream) : launch_any<1, 1>(D, att, p, stream);
 }
 
 }  // namespace
@@ -356,6 +358,23 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
   if (best_G * ((n + 31) / 32) > 128) return AECCT_ERR_UNSUPPORTED;  // hard-decision bitmasks of a group
   if (d.alpha_mode == 1 && best_C != 1) return AECCT_ERR_UNSUPPORTED;  // per-word alpha: one CTA per word
 
+  // Per-row lists over per-head staged rows (d = 128): a head's K and V rows of the whole group
+  // (128 bytes a row) are gathered into the 80 KB of the operand tile and the weight stages, and
+  // each row's scores take TMEM columns [128, 384).  By default it replaces the per-row walk when
+  // the group spans a cluster, where that walk reads every key through the distributed shared
+  // memory window.
+  size_t max_list = 0;
+  for (int r = 0; r < 2; ++r)
+    for (int t = 0; t < T; ++t) max_list = std::max(max_list, nb[r][t].size());
+  const bool staged_ok = D == 128 && best_G * T <= kStagedMaxRows && max_list <= static_cast<size_t>(kStagedMaxKeys);
+  int att = tasks ? 1 : 0;
+  if (d.attention_mode == 3) {
+    if (!staged_ok) return AECCT_ERR_UNSUPPORTED;
+    att = 2;
+  } else if (d.attention_mode == 0 && !tasks && staged_ok && best_C > 1) {
+    att = 2;
+  }
+
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return AECCT_ERR_NO_DEVICE;
@@ -367,7 +386,7 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
     return AECCT_ERR_NO_DEVICE;
   }
   int max_clusters = 0;
-  e = prepare_variant(d.activation, d.linear_mode, D, tasks, best_C, &max_clusters);
+  e = prepare_variant(d.activation, d.linear_mode, D, att, best_C, &max_clusters);
   if (e != cudaSuccess) return cuda_fail(e, "kernel occupancy");
   if (max_clusters < 1) {
     g_last_error = "no cluster of this size fits on the device";
@@ -377,7 +396,7 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
   aecct_handle *h = new aecct_handle();
   h->n = n, h->k = k, h->T = T, h->m = m, h->d = D, h->n_layers = d.n_layers, h->h_first = d.h_first;
   h->Tp = (tasks && D == 128) ? Tp128 : T;
-  h->d_spe = d.d_spe, h->C = best_C, h->G = best_G, h->max_clusters = max_clusters, h->tasks = tasks;
+  h->d_spe = d.d_spe, h->C = best_C, h->G = best_G, h->max_clusters = max_clusters, h->att = att;
   h->ln_eps = d.ln_eps, h->alpha_floor = d.alpha_floor, h->b_d1 = d.b_d1, h->device = dev;
   h->alpha_mode = d.alpha_mode;
   h->activation = d.activation;
@@ -681,7 +700,7 @@ int aecct_decode(aecct_handle *h, const float *y_dev, int64_t B, uint8_t *bits_d
   if (prev != AECCT_OK) return prev;
   const DecodeParams p = decode_params(h, B, y_dev, bits_dev, syndrome_dev, logits_dev, h->d_err);
   cudaError_t e;
-  e = launch_variant(h->activation, h->linear_mode, h->d, h->tasks, p, stream);
+  e = launch_variant(h->activation, h->linear_mode, h->d, h->att, p, stream);
   if (e != cudaSuccess) return cuda_fail(e, "decode launch");
   if ((e = cudaMemcpyAsync(h->h_err, h->d_err, sizeof(int), cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
     return cuda_fail(e, "status copy");
@@ -794,7 +813,7 @@ int aecct_decode_host_noalloc(aecct_handle *h, const float *y_host, int64_t B, u
   if ((e = cudaMemcpyAsync(y_dev, y_host, sizeof(float) * b * n, cudaMemcpyHostToDevice, stream)) != cudaSuccess)
     return cuda_fail(e, "copy y");
   const DecodeParams p = decode_params(h, B, y_dev, bits_dev, syn_dev, logits_dev, err);
-  e = launch_variant(h->activation, h->linear_mode, h->d, h->tasks, p, stream);
+  e = launch_variant(h->activation, h->linear_mode, h->d, h->att, p, stream);
   if (e != cudaSuccess) return cuda_fail(e, "decode launch");
   if ((e = cudaMemcpyAsync(bits_host, bits_dev, b * n, cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
     return cuda_fail(e, "copy bits");
@@ -833,11 +852,12 @@ int aecct_query(const aecct_handle *h, int32_t *cluster_ctas, int32_t *words_per
   if (max_clusters) *max_clusters = h->max_clusters;
   if (threads_per_cta) *threads_per_cta = kThreads;
   int sm;
-  if (h->d == 32) sm = h->tasks ? SmemLayout<32, true>::kTotal : SmemLayout<32>::kTotal;
-  else if (h->d == 64) sm = h->tasks ? SmemLayout<64, true>::kTotal : SmemLayout<64>::kTotal;
-  else sm = h->tasks ? SmemLayout<128, true>::kTotal : SmemLayout<128>::kTotal;
+  const bool tasks = h->att == 1;
+  if (h->d == 32) sm = tasks ? SmemLayout<32, true>::kTotal : SmemLayout<32>::kTotal;
+  else if (h->d == 64) sm = tasks ? SmemLayout<64, true>::kTotal : SmemLayout<64>::kTotal;
+  else sm = tasks ? SmemLayout<128, true>::kTotal : SmemLayout<128>::kTotal;
   if (smem_bytes) *smem_bytes = sm;
-  if (attention_mode) *attention_mode = h->tasks ? 2 : 1;
+  if (attention_mode) *attention_mode = h->att == 1 ? 2 : (h->att == 2 ? 3 : 1);
   return AECCT_OK;
 }
 

@@ -240,6 +240,11 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t
 __device__ __forceinline__ void st_shared_v2(uint32_t addr, uint32_t a, uint32_t b) {
   asm volatile("st.shared.v2.b32 [%0], {%1, %2};" ::"r"(addr), "r"(a), "r"(b) : "memory");
 }
+__device__ __forceinline__ float4 ld_shared_f4(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(addr) : "memory");
+  return v;
+}
 __device__ __forceinline__ void st_shared_f4(uint32_t addr, float a, float b, float c, float d) {
   asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(a), "f"(b), "f"(c), "f"(d) : "memory");
 }
@@ -652,9 +657,9 @@ struct BlockCtx {
   bool cluster;     // more than one CTA per cluster
 };
 
-template <int D, bool TASKS>
+template <int D, int ATT>
 struct Issuer {
-  using L = SmemLayout<D, TASKS>;
+  using L = SmemLayout<D, ATT == 1>;
   using W = WeightSchedule<D>;
   static constexpr int S = W::kStages;
   static constexpr int CPL = W::kCPL;
@@ -781,10 +786,13 @@ struct Issuer {
 //           W0, W1, W2 again once chunks 16-18 are consumed.
 // A barrier armed u times per block (u odd for W0, W1, A0, A1) completes phase parity
 // (lpar if u is odd) ^ (index of the use within the block), with lpar the block's parity.
-template <bool TASKS>
-struct Issuer<128, TASKS> {
+template <int ATT>
+struct Issuer<128, ATT> {
   static constexpr int D = 128;
-  using L = SmemLayout<D, TASKS>;
+  using L = SmemLayout<D, ATT == 1>;
+  // staged attention (ATT == 2) gathers each head's keys and values into the operand tile and the
+  // weight stages, so O's weights (W0, W1) are fetched after attention (stage_o) instead of with QKV's
+  static constexpr bool kStaged = ATT == 2;
   using W = WeightSchedule<D>;
   static constexpr uint32_t kChunk = W::kStageBytes;
   static_assert(W::kCPL == 24 && W::kStages == 3 && kChunk == 16384, "d = 128 schedule");
@@ -866,10 +874,14 @@ struct Issuer<128, TASKS> {
     arm(slot(P).id, W::chunk(P).bytes);
     copies<P, P + 1>(src);
   }
-  // QKV (region U) and O (W0, W1) of a block
+  // QKV (region U) and O (W0, W1) of a block; staged attention: QKV only
   __device__ __forceinline__ void stage_qkv_o(const uint8_t *src) const {
     arm(3, 6 * kChunk);
     copies<0, 6>(src);
+    if constexpr (!kStaged) stage_o(src);
+  }
+  // O's weights into W0, W1
+  __device__ __forceinline__ void stage_o(const uint8_t *src) const {
     copy1<6>(src);
     copy1<7>(src);
   }
@@ -1012,8 +1024,11 @@ struct Issuer<128, TASKS> {
 // ------------------------------------------------------------------------------------------
 // the kernel
 // ------------------------------------------------------------------------------------------
-template <int D, bool TASKS, int ACT, int LIN>
+template <int D, int ATT, int ACT, int LIN>
 __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid_constant__ DecodeParams p) {
+  // ATT: 0 = per-row neighbour lists, 1 = warp tasks, 2 = per-row lists over per-head staged rows
+  constexpr bool TASKS = ATT == 1, STAGED = ATT == 2;
+  static_assert(!STAGED || D == 128, "staged attention is built for d = 128");
   using L = SmemLayout<D, TASKS>;
   using LP = LayerParamLayout;
   constexpr int DH = D / kHeads;  // head width
@@ -1080,7 +1095,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   const uint32_t tmem = *s_tmem;
   const Ctl ctl{s_abort, p.err, p.wait_limit};
 
-  const Issuer<D, TASKS> issuer{sb, tmem, ctl, s_issued};
+  const Issuer<D, ATT> issuer{sb, tmem, ctl, s_issued};
   if (warp == 0 && cluster_id < p.n_groups) issuer.prologue(p.wstream);
   {
     // ------------------------------------------------------------ CUDA-core warps
@@ -1167,6 +1182,15 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
       if (tid == 0) {
         fence_acq_rel_cluster();
         for (int c = 0; c < p.C; ++c) mbar_arrive_cluster(mapa_cluster(bar, c));
+      }
+      __syncwarp();
+    };
+    // after a CTA-wide barrier: this CTA no longer reads any CTA's K/V of this block
+    auto kvf_signal = [&]() {
+      if (p.C == 1) return;
+      if (tid == 0) {
+        fence_acq_rel_cluster();
+        for (int c = 0; c < p.C; ++c) mbar_arrive_cluster(mapa_cluster(bar_kvf, c));
       }
       __syncwarp();
     };
@@ -1455,10 +1479,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             store_codes<XS>(aop, r, sl * XS, D, qv);
             if (cap) capture_q(l, 1, qv, sl * XS, XS, alpha_in);
           }
-        } else {
-        cluster_arrive(bar_kvr);
+        } else if constexpr (!STAGED) {
+          cluster_arrive(bar_kvr);
           cluster_wait(bar_kvr, kvr_ph);
-  
+
           // ---------------- S5: HPSA (Sec. 4.2)
           // the A of each head goes over the head's Q in TMEM (this thread's lane; that Q has no
           // other reader), so that the second head's attention runs with the registers of one;
@@ -1531,10 +1555,179 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
               if (cap) capture_q(l, 1, qv, e * DH, DH, alpha_in);
             }
           }
+        } else {
+          // ---------------- S5: HPSA (Sec. 4.2), per-row lists over per-head staged rows (d = 128).
+          // Head by head, the K and V rows of the head for every row of the group are gathered from
+          // every CTA of the cluster (coalesced 16-byte reads) into this CTA's operand tile and weight
+          // stages, both idle here.  The row's 4 threads share the head: each takes 4 keys of every
+          // 16-key block for the scores and their exponentials (the row's TMEM lane, columns from
+          // kSc), and then folds every key, in ascending order, into 4 of the 16 features of num.
+          // The arithmetic is the canonical one, key for key and feature for feature.
+          cluster_arrive(bar_kvr);
+          cluster_wait(bar_kvr, kvr_ph);
+          static_assert(L::kOffW == L::kOffAop + L::kAopBytes, "the staging area spans the operand tile and the weight stages");
+          constexpr uint32_t kSc = 128;  // the dead K and V accumulator columns [128, 384)
+          const uint32_t stg = sb + L::kOffAop;  // row rho of the group: 128 bytes at rho * 128, 16-byte slot f at f ^ (rho & 7)
+          const int nrows = p.G * Tp;            // <= 640 (checked at create)
+          const int rowbase = g * Tp;
+          auto dot16 = [&](const float *q, const float4 *kk) -> float {
+            float2 d2 = make_float2(0.0f, 0.0f);
+#pragma unroll
+            for (int i = 0; i < DH / 4; ++i) {
+              d2 = fma2(make_float2(q[4 * i], q[4 * i + 1]), make_float2(kk[i].x, kk[i].y), d2);
+              d2 = fma2(make_float2(q[4 * i + 2], q[4 * i + 3]), make_float2(kk[i].z, kk[i].w), d2);
+            }
+            return __fadd_rn(d2.x, d2.y);
+          };
+          for (int e = 0; e < kHeads; ++e) {
+            {
+              // gather: item it = (row rho, 16-byte slot f of the head's K|V), 10 items per thread at most
+              float4 v[5];
+#pragma unroll
+              for (int half = 0; half < 2; ++half) {
+#pragma unroll
+                for (int j = 0; j < 5; ++j) {
+                  const int it = tid + kEpiThreads * (5 * half + j);
+                  if (it < nrows * 8) {
+                    const int rho = it >> 3, f = it & 7;
+                    v[j] = ld_cluster_f32x4(s_kvcl[rho >> 7] + static_cast<uint32_t>(rho & 127) * L::kKvStride +
+                                            static_cast<uint32_t>(e) * L::kSlot + 16u * f);
+                  }
+                }
+#pragma unroll
+                for (int j = 0; j < 5; ++j) {
+                  const int it = tid + kEpiThreads * (5 * half + j);
+                  if (it < nrows * 8) {
+                    const int rho = it >> 3, f = it & 7;
+                    st_shared_f4(stg + static_cast<uint32_t>(rho) * 128u + static_cast<uint32_t>((f ^ (rho & 7)) << 4),
+                                 v[j].x, v[j].y, v[j].z, v[j].w);
+                  }
+                }
+              }
+            }
+            named_bar_sync(5, kEpiThreads);
+            if (e == kHeads - 1) kvf_signal();  // every read of the cluster's K/V of this block is done
+            const int mk = (e < p.h_first) ? 0 : 1;
+            const uint32_t info = row_cw ? __ldg(p.mask_info[mk] + t) : 0u;
+            const int cnt = static_cast<int>(info & 2047u);
+            const uint4 *lst = p.mask_list[mk] + (info >> 11);
+            const int nmax = __reduce_max_sync(0xffffffffu, cnt);  // the same for the 4 warps of the quadrant
+            float q[DH];
+            {
+              float qa[DH], bq[DH];
+              ldg_vec<DH>(lp + LP::bqkv(D) + e * DH, bq);
+              tmem_ld<DH>(tl + e * DH, qa);
+              tmem_wait_ld();
+              if (cap && sl == (e & 3)) capture_acc(l, 0, qa, e * DH, DH);
+#pragma unroll
+              for (int i = 0; i < DH; ++i) q[i] = __fadd_rn(__fmul_rn(qa[i], fq), bq[i]);
+            }
+            // pass 1: sigma of keys [b + 4 sl, b + 4 sl + 4) of every 16-key block b, and their maximum
+            float mx = -INFINITY;
+            for (int b = 0; b < nmax; b += 16) {
+              const int k0 = b + 4 * sl;
+              if (k0 < nmax) {
+                const uint4 w = (k0 < cnt) ? __ldg(lst + (k0 >> 3)) : make_uint4(0u, 0u, 0u, 0u);
+                const uint32_t lo = (k0 & 4) ? w.z : w.x, hi = (k0 & 4) ? w.w : w.y;
+                const int idx[4] = {static_cast<int>(lo & 0xFFFFu), static_cast<int>(lo >> 16),
+                                    static_cast<int>(hi & 0xFFFFu), static_cast<int>(hi >> 16)};
+                float sg[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                  const int rho = rowbase + idx[i];  // a key past the row's count reads a valid row (offset 0)
+                  const uint32_t rb = stg + static_cast<uint32_t>(rho) * 128u;
+                  float4 kk[DH / 4];
+#pragma unroll
+                  for (int f = 0; f < DH / 4; ++f) kk[f] = ld_shared_f4(rb + static_cast<uint32_t>((f ^ (rho & 7)) << 4));
+                  sg[i] = __fmul_rn(dot16(q, kk), p.att_scale);
+                  if (k0 + i < cnt) mx = fmaxf(mx, sg[i]);
+                }
+                tmem_st4(tl + kSc + k0, sg[0], sg[1], sg[2], sg[3]);
+              }
+            }
+            tmem_wait_st();
+            tc_fence_before();
+            mx = row_max(mx);
+            tc_fence_after();
+            // pass 2: p = 2^(sigma - m) of the same keys, written over their scores
+            for (int b = 0; b < nmax; b += 16) {
+              const int k0 = b + 4 * sl;
+              if (k0 < nmax) {
+                float sg[4];
+                tmem_ld<4>(tl + kSc + k0, sg);
+                tmem_wait_ld();
+                const float2 p01 = exp2_series2(add2(make_float2(sg[0], sg[1]), make_float2(-mx, -mx)));
+                const float2 p23 = exp2_series2(add2(make_float2(sg[2], sg[3]), make_float2(-mx, -mx)));
+                tmem_st4(tl + kSc + k0, p01.x, p01.y, p23.x, p23.y);
+              }
+            }
+            tmem_wait_st();
+            tc_fence_before();
+            named_bar_sync(qbar, 128);
+            tc_fence_after();
+            // l = sum p and num = sum p v over the row's keys in ascending order, features [4 sl, 4 sl + 4)
+            float lsum = 0.0f, num[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+            const uint32_t vslot = static_cast<uint32_t>(DH / 4 + sl);
+            for (int b = 0; b < nmax; b += 16) {
+              float pb[16];
+              tmem_ld<16>(tl + kSc + b, pb);
+              tmem_wait_ld();
+              const uint4 w0 = (b < cnt) ? __ldg(lst + (b >> 3)) : make_uint4(0u, 0u, 0u, 0u);
+              const uint4 w1 = (b + 8 < cnt) ? __ldg(lst + (b >> 3) + 1) : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+              for (int kk = 0; kk < 16; ++kk) {
+                if (b + kk < cnt) {
+                  const int rho = rowbase + idx_at(kk < 8 ? w0 : w1, kk & 7);
+                  const float4 vv = ld_shared_f4(stg + static_cast<uint32_t>(rho) * 128u +
+                                                 ((vslot ^ static_cast<uint32_t>(rho & 7)) << 4));
+                  lsum = __fadd_rn(lsum, pb[kk]);
+                  num[0] = __fmaf_rn(pb[kk], vv.x, num[0]);
+                  num[1] = __fmaf_rn(pb[kk], vv.y, num[1]);
+                  num[2] = __fmaf_rn(pb[kk], vv.z, num[2]);
+                  num[3] = __fmaf_rn(pb[kk], vv.w, num[3]);
+                }
+              }
+            }
+            {
+              const float inv = __fdiv_rn(1.0f, lsum);
+              float a4[4];
+#pragma unroll
+              for (int f = 0; f < 4; ++f) a4[f] = row_cw ? __fmul_rn(num[f], inv) : 0.0f;
+              // A of (row, head e), features [4 sl, 4 sl + 4), over the head's Q (read by all 4 threads
+              // before the quadrant barrier above)
+              tmem_st4(tl + e * DH + 4 * sl, a4[0], a4[1], a4[2], a4[3]);
+            }
+            tmem_wait_st();
+            tc_fence_before();
+            named_bar_sync(5, kEpiThreads);  // the staging area is free for the next head
+            tc_fence_after();
+          }
+          // O's weights into W0, W1 (free again), while the codes of A are made
+          if (warp == 0) issuer.stage_o(p.wstream + static_cast<size_t>(l) * p.layer_bytes);
+          // Quant(A) -> O operand: columns [sl XS, sl XS + XS) = heads 2 sl and 2 sl + 1, from TMEM
+          float av[XS];
+          tmem_ld<XS>(tl + sl * XS, av);
+          tmem_wait_ld();
+          if constexpr (LIN == 1) {
+            store_bf16<XS>(aop, r, sl * XS, D, av);
+          } else {
+            float amax = 0.0f;
+#pragma unroll
+            for (int j = 0; j < XS; ++j) amax = fmaxf(amax, fabsf(av[j]));
+            float a = word_alpha(row_max(amax));
+            a = (a > p.alpha_floor) ? a : p.alpha_floor;
+            alpha_in = a;
+            const float rr = __fdiv_rn(127.0f, a);
+            float qv[XS];
+            codes<XS>(av, rr, qv);
+            store_codes<XS>(aop, r, sl * XS, D, qv);
+            if (cap) capture_q(l, 1, qv, sl * XS, XS, alpha_in);
+          }
         }
         // this CTA no longer reads any K/V of this block (arrived before the O GEMM is issued: the
-        // d = 128 schedule stages FFN1's weights over the K/V region once every CTA has arrived)
-        if constexpr (!TASKS) cluster_arrive(bar_kvf);
+        // d = 128 schedule stages FFN1's weights over the K/V region once every CTA has arrived);
+        // the staged mode has arrived after its last gather
+        if constexpr (ATT == 0) cluster_arrive(bar_kvf);
         signal_op(1, l, gi);
 
         // ---------------- S6: O projection + residual + LayerNorm (Sec. 5, Post-LN)
@@ -1740,10 +1933,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   }
 }
 
-template <int D, bool TASKS, int ACT, int LIN>
+template <int D, int ATT, int ACT, int LIN>
 cudaError_t prepare_decode_kernel(int cluster_ctas, int *max_active_clusters) {
-  using L = SmemLayout<D, TASKS>;
-  cudaError_t e = cudaFuncSetAttribute(aecct_decoder_kernel<D, TASKS, ACT, LIN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  using L = SmemLayout<D, ATT == 1>;
+  cudaError_t e = cudaFuncSetAttribute(aecct_decoder_kernel<D, ATT, ACT, LIN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(L::kTotal));
   if (e != cudaSuccess) return e;
   // ask for the smallest shared-memory carve-out that holds one CTA (1 KB of it is reserved by
@@ -1754,7 +1947,7 @@ cudaError_t prepare_decode_kernel(int cluster_ctas, int *max_active_clusters) {
     return e;
   if (smem_sm > 0) {
     const int pct = static_cast<int>((100ll * (L::kTotal + 1024) + smem_sm - 1) / smem_sm);
-    e = cudaFuncSetAttribute(aecct_decoder_kernel<D, TASKS, ACT, LIN>, cudaFuncAttributePreferredSharedMemoryCarveout,
+    e = cudaFuncSetAttribute(aecct_decoder_kernel<D, ATT, ACT, LIN>, cudaFuncAttributePreferredSharedMemoryCarveout,
                              pct > 100 ? 100 : pct);
     if (e != cudaSuccess) return e;
   }
@@ -1769,12 +1962,12 @@ cudaError_t prepare_decode_kernel(int cluster_ctas, int *max_active_clusters) {
   cfg.dynamicSmemBytes = L::kTotal;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaOccupancyMaxActiveClusters(max_active_clusters, aecct_decoder_kernel<D, TASKS, ACT, LIN>, &cfg);
+  return cudaOccupancyMaxActiveClusters(max_active_clusters, aecct_decoder_kernel<D, ATT, ACT, LIN>, &cfg);
 }
 
-template <int D, bool TASKS, int ACT, int LIN>
+template <int D, int ATT, int ACT, int LIN>
 cudaError_t launch_decode(const DecodeParams &p, cudaStream_t stream) {
-  using L = SmemLayout<D, TASKS>;
+  using L = SmemLayout<D, ATT == 1>;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -1787,7 +1980,7 @@ cudaError_t launch_decode(const DecodeParams &p, cudaStream_t stream) {
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, aecct_decoder_kernel<D, TASKS, ACT, LIN>, p);
+  return cudaLaunchKernelEx(&cfg, aecct_decoder_kernel<D, ATT, ACT, LIN>, p);
 }
 
 }  // namespace aecct

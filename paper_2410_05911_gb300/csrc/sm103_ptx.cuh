@@ -195,6 +195,11 @@ __device__ __forceinline__ void tmem_st8(uint32_t taddr, const float *v) {
                "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7]))
                : "memory");
 }
+__device__ __forceinline__ void tmem_st4(uint32_t taddr, float a, float b, float c, float d) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1, %2, %3, %4};" ::"r"(taddr), "r"(__float_as_uint(a)),
+               "r"(__float_as_uint(b)), "r"(__float_as_uint(c)), "r"(__float_as_uint(d))
+               : "memory");
+}
 // store N (multiple of 8) consecutive columns of this thread's lane
 template <int N>
 __device__ __forceinline__ void tmem_st(uint32_t taddr, const float *v) {

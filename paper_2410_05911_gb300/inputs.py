@@ -441,6 +441,7 @@ def random_model(
     zero_weights: bool = False,
     binary: bool = False,
     full_precision: bool = False,
+    spe_noise: bool = False,
 ) -> ModelTensors:
     """Seeded synthetic AECCT parameters shaped like a trained model.
 
@@ -458,6 +459,10 @@ def random_model(
 
     full_precision=True also draws fp32 weights W ~ N(0, 1/d_in) per tensor (the full-precision
     linear layers of the ECCT baseline, Sec. 3) and selects them (linear_mode = 1).
+
+    spe_noise=True draws the SPE table as seeded N(0, 1) values instead (for shape tests of the
+    decoder at its largest token counts, where the O(T^3) precompute would dominate and the
+    table's content plays no role).
     """
     rng = np.random.Generator(np.random.PCG64(seed))
     T = code.T
@@ -497,7 +502,8 @@ def random_model(
     ln_gamma = (1.0 + 0.1 * rng.standard_normal((n_layers, 2, d))).astype(np.float32)
     ln_beta = (0.1 * rng.standard_normal((n_layers, 2, d))).astype(np.float32)
     emb = rng.standard_normal((T, d - d_spe)).astype(np.float32)
-    spe = spe_for_code(code.H, d_spe, seed + 7919)
+    spe = (rng.standard_normal((T, d_spe)).astype(np.float32) if spe_noise
+           else spe_for_code(code.H, d_spe, seed + 7919))
     w_d1 = (rng.standard_normal(d) / math.sqrt(d)).astype(np.float32)
     b_d1 = float(np.float32(0.1 * rng.standard_normal()))
     w_out = (2.0 * rng.standard_normal((T, code.n)) / math.sqrt(T)).astype(np.float32)

@@ -93,7 +93,11 @@ def test_create_rejects_invalid_packed_code_and_shapes():
     assert _status(big, cluster_ctas=2) == A.AECCT_ERR_INVALID_ARG
     # attention modes: unknown value, and warp tasks where they do not apply (more than 128 token
     # rows once each node type starts on a 32-row boundary; d = 128 with one alpha per word)
-    assert _status(I.workload_model("bch31_16"), attention_mode=3) == A.AECCT_ERR_INVALID_ARG
+    assert _status(I.workload_model("bch31_16"), attention_mode=4) == A.AECCT_ERR_INVALID_ARG
+    # staged rows: d = 128 only, at most 640 token rows per group
+    assert _status(I.workload_model("bch31_16"), attention_mode=3) == A.AECCT_ERR_UNSUPPORTED
+    c680 = I.ldpc_regular_code(680, 340, 3, 6, seed=680340)
+    assert _status(I.random_model(c680, 128, 1, seed=3, spe_noise=True), attention_mode=3) == A.AECCT_ERR_UNSUPPORTED
     assert _status(I.workload_model("ldpc128_64"), attention_mode=2) == A.AECCT_ERR_UNSUPPORTED
     m63 = copy.deepcopy(I.workload_model("bch63_36"))
     m63.alpha_mode = 1
