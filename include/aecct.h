@@ -208,7 +208,7 @@ int aecct_set_capture(aecct_handle *h, int64_t cap_B, int8_t *q_dev, int32_t *ac
 
 /* Launch facts of the handle (for benchmarks): CTAs per codeword group, codewords per
  * group, the number of clusters a decode launches at most, threads per CTA, dynamic
- * shared memory bytes per CTA, and the attention mode in use (1 = per-row lists,
+ * shared memory bytes per CTA (warp tasks: with their plan), and the attention mode in use (1 = per-row lists,
  * 2 = warp tasks, 3 = per-row lists over per-head staged rows).  Any pointer may be NULL. */
 int aecct_query(const aecct_handle *h, int32_t *cluster_ctas, int32_t *words_per_group, int32_t *max_clusters,
                 int32_t *threads_per_cta, int32_t *smem_bytes, int32_t *attention_mode);

@@ -151,11 +151,17 @@ struct DecodeParams {
   // Task-mode attention plan (one CTA per group of codewords, d <= 64).  A task is one head for
   // a query group: up to 32 consecutive rows of one codeword, one per lane.  It walks the union of
   // its lanes' key sets (ascending token order) with per-lane membership bits.
-  const uint16_t *plan_task;   // [16 warps][kMaxTasks]: group * 8 + head; 0xFFFF ends the list
-  const uint4 *plan_grp;       // [groups]: {first row, lanes, first row of the codeword, 0}
-  const uint32_t *plan_uinfo;  // [groups][2 rings]: (start << 8) | count of the union list
-  const uint4 *plan_ulist;     // union lists: 16 row offsets (one byte each) per entry
-  const uint4 *plan_mask;      // [groups][2][32 lanes]: 128 membership bits over the union list
+  // The plan is one blob that every CTA copies into shared memory (after the SmemLayout regions)
+  // at the start of the kernel; the offsets are byte offsets into it, 16-byte aligned:
+  //   task  [16 warps][kMaxTasks] uint16: group * 8 + head; 0xFFFF ends the list
+  //   grp   [groups] uint4: {first row, lanes, first row of the codeword, 0}
+  //   uinfo [groups][2 rings] uint32: (start << 8) | count of the union list
+  //   ulist union lists: 16 row offsets (one byte each) per 16-byte entry
+  //   mask  [groups][2][32 lanes] uint4: 128 membership bits over the union list
+  const uint4 *plan_blob;
+  uint32_t plan_bytes;  // a multiple of 16; 0 without warp tasks
+  uint32_t off_task, off_grp, off_uinfo, off_ulist, off_mask;
+
   float ln_eps, alpha_floor, att_scale;
   int alpha_mode;  // 0 = absmax alpha per token row, 1 = per quantised matrix of a word (C == 1)
   // integer-core capture (device, optional)
@@ -220,7 +226,8 @@ struct SmemLayout {
 template <int D, int ATT, int ACT, int LIN>
 cudaError_t launch_decode(const DecodeParams &p, cudaStream_t stream);
 template <int D, int ATT, int ACT, int LIN>
-cudaError_t prepare_decode_kernel(int cluster_ctas, int *max_active_clusters);
+cudaError_t prepare_decode_kernel(int cluster_ctas, uint32_t plan_bytes, int *max_active_clusters);
+constexpr uint32_t kMaxDynSmem = 232448;  // the largest dynamic shared memory a CTA may opt into (227 KB)
 constexpr int kStagedMaxRows = 640;  // staged attention: rows of a group (128 bytes each in 80 KB)
 constexpr int kStagedMaxKeys = 256;  // staged attention: keys per row (TMEM columns [128, 384))
 

@@ -50,9 +50,8 @@ struct aecct_handle {
   int hwords = 0;
   uint16_t *mask_list[2] = {nullptr, nullptr};
   uint16_t *perm = nullptr, *pos = nullptr;
-  uint16_t *plan_task = nullptr;
-  uint32_t *plan_grp = nullptr, *plan_uinfo = nullptr, *plan_mask = nullptr;
-  uint8_t *plan_ulist = nullptr;
+  uint8_t *plan_blob = nullptr;  // the attention plan (task mode), copied into shared memory by the kernel
+  uint32_t plan_bytes = 0, off_task = 0, off_grp = 0, off_uinfo = 0, off_ulist = 0, off_mask = 0;
   int *d_err = nullptr;
   int *h_err = nullptr;  // pinned
   cudaEvent_t ev = nullptr;
@@ -197,15 +196,15 @@ int schedule_chunks(int D, ChunkDesc *out) {
 
 // the compiled kernel for (d, attention path ATT, activation ACT, linear mode LIN)
 template <int ACT, int LIN>
-cudaError_t prepare_any(int D, int att, int C, int *max_clusters) {
+cudaError_t prepare_any(int D, int att, int C, uint32_t pb, int *max_clusters) {
   if (att == 1)
-    return D == 32   ? prepare_decode_kernel<32, 1, ACT, LIN>(C, max_clusters)
-           : D == 64 ? prepare_decode_kernel<64, 1, ACT, LIN>(C, max_clusters)
-                     : prepare_decode_kernel<128, 1, ACT, LIN>(C, max_clusters);
-  if (att == 2) return prepare_decode_kernel<128, 2, ACT, LIN>(C, max_clusters);  // d = 128 only
-  if (D == 32) return prepare_decode_kernel<32, 0, ACT, LIN>(C, max_clusters);
-  if (D == 64) return prepare_decode_kernel<64, 0, ACT, LIN>(C, max_clusters);
-  return prepare_decode_kernel<128, 0, ACT, LIN>(C, max_clusters);
+    return D == 32   ? prepare_decode_kernel<32, 1, ACT, LIN>(C, pb, max_clusters)
+           : D == 64 ? prepare_decode_kernel<64, 1, ACT, LIN>(C, pb, max_clusters)
+                     : prepare_decode_kernel<128, 1, ACT, LIN>(C, pb, max_clusters);
+  if (att == 2) return prepare_decode_kernel<128, 2, ACT, LIN>(C, pb, max_clusters);  // d = 128 only
+  if (D == 32) return prepare_decode_kernel<32, 0, ACT, LIN>(C, pb, max_clusters);
+  if (D == 64) return prepare_decode_kernel<64, 0, ACT, LIN>(C, pb, max_clusters);
+  return prepare_decode_kernel<128, 0, ACT, LIN>(C, pb, max_clusters);
 }
 template <int ACT, int LIN>
 cudaError_t launch_any(int D, int att, const DecodeParams &p, cudaStream_t stream) {
@@ -218,9 +217,10 @@ cudaError_t launch_any(int D, int att, const DecodeParams &p, cudaStream_t strea
   if (D == 64) return launch_decode<64, 0, ACT, LIN>(p, stream);
   return launch_decode<128, 0, ACT, LIN>(p, stream);
 }
-cudaError_t prepare_variant(int act, int lin, int D, int att, int C, int *max_clusters) {
-  if (lin == 0) return act == 0 ? prepare_any<0, 0>(D, att, C, max_clusters) : prepare_any<1, 0>(D, att, C, max_clusters);
-  return act == 0 ? prepare_any<0, 1>(D, att, C, max_clusters) : prepare_any<1, 1>(D, att, C, max_clusters);
+cudaError_t prepare_variant(int act, int lin, int D, int att, int C, uint32_t pb, int *max_clusters) {
+  if (lin == 0)
+    return act == 0 ? prepare_any<0, 0>(D, att, C, pb, max_clusters) : prepare_any<1, 0>(D, att, C, pb, max_clusters);
+  return act == 0 ? prepare_any<0, 1>(D, att, C, pb, max_clusters) : prepare_any<1, 1>(D, att, C, pb, max_clusters);
 }
 cudaError_t launch_variant(int act, int lin, int D, int att, const DecodeParams &p, cudaStream_t stream) {
   if (lin == 0) return act == 0 ? launch_any<0, 0>(D, att, p, stream) : launch_any<1, 0>(D, att, p, stream);
@@ -385,8 +385,23 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
     g_last_error = "device is not compute capability 10.x";
     return AECCT_ERR_NO_DEVICE;
   }
+  // a bound on the task plan's bytes (it sits in shared memory after the fixed regions)
+  uint32_t plan_bound = 0;
+  if (tasks) {
+    const uint32_t ngb = D == 128 ? static_cast<uint32_t>((n + 31) / 32 + (m + 31) / 32)
+                                  : static_cast<uint32_t>(best_G * ((T + 31) / 32));
+    auto r16 = [](uint32_t v) { return (v + 15u) & ~15u; };
+    plan_bound = r16(2u * kEpiWarps * kMaxTasks) + 16u * ngb +
+                 r16(8u * ngb) + 2u * ngb * r16(static_cast<uint32_t>(T)) + 16u * 2u * 32u * ngb;
+    const uint32_t fixed = D == 32 ? SmemLayout<32, true>::kTotal
+                           : D == 64 ? SmemLayout<64, true>::kTotal : SmemLayout<128, true>::kTotal;
+    if (fixed + plan_bound > kMaxDynSmem) {
+      g_last_error = "the warp-task plan does not fit shared memory";
+      return AECCT_ERR_UNSUPPORTED;
+    }
+  }
   int max_clusters = 0;
-  e = prepare_variant(d.activation, d.linear_mode, D, att, best_C, &max_clusters);
+  e = prepare_variant(d.activation, d.linear_mode, D, att, best_C, plan_bound, &max_clusters);
   if (e != cudaSuccess) return cuda_fail(e, "kernel occupancy");
   if (max_clusters < 1) {
     g_last_error = "no cluster of this size fits on the device";
@@ -592,6 +607,27 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
     if (d.linear_mode == 0) std::memcpy(v + LayerParamLayout::sw(D), d.w_scale + (size_t)l * 6, sizeof(float) * 6);
     else for (int i = 0; i < 6; ++i) v[LayerParamLayout::sw(D) + i] = 1.0f;
   }
+  // the task plan as one blob, each part on a 16-byte boundary
+  std::vector<uint8_t> blob;
+  if (tasks) {
+    auto put = [&](const void *src, size_t bytes) {
+      const uint32_t off = static_cast<uint32_t>(blob.size());
+      blob.insert(blob.end(), static_cast<const uint8_t *>(src), static_cast<const uint8_t *>(src) + bytes);
+      while (blob.size() % 16) blob.push_back(0);
+      return off;
+    };
+    h->off_task = put(ptask.data(), ptask.size() * 2);
+    h->off_grp = put(pgrp.data(), pgrp.size() * 4);
+    h->off_uinfo = put(puinfo.data(), puinfo.size() * 4);
+    h->off_ulist = put(pulist.data(), pulist.size());
+    h->off_mask = put(pmask.data(), pmask.size() * 4);
+    h->plan_bytes = static_cast<uint32_t>(blob.size());
+    if (h->plan_bytes > plan_bound) {
+      free_handle(h);
+      g_last_error = "internal: the task plan exceeds its bound";
+      return AECCT_ERR_UNSUPPORTED;
+    }
+  }
   const int de = D - d.d_spe;
   if ((rc = dev_upload(h, &h->wstream, reinterpret_cast<const uint8_t *>(ws.data()), ws.size() * 2)) ||
       (rc = dev_upload(h, &h->lparams, lpv.data(), lpv.size())) ||
@@ -607,11 +643,7 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
       (rc = dev_upload(h, &h->mask_list[0], mlist[0].data(), mlist[0].size())) ||
       (rc = dev_upload(h, &h->mask_info[1], minfo[1].data(), minfo[1].size())) ||
       (rc = dev_upload(h, &h->mask_list[1], mlist[1].data(), mlist[1].size())) ||
-      (rc = dev_upload(h, &h->plan_task, ptask.data(), ptask.size())) ||
-      (rc = dev_upload(h, &h->plan_grp, pgrp.data(), pgrp.size())) ||
-      (rc = dev_upload(h, &h->plan_uinfo, puinfo.data(), puinfo.size())) ||
-      (rc = dev_upload(h, &h->plan_ulist, pulist.data(), pulist.size())) ||
-      (rc = dev_upload(h, &h->plan_mask, pmask.data(), pmask.size())) ||
+      (rc = dev_upload(h, &h->plan_blob, blob.data(), blob.size())) ||
       (rc = dev_upload<int>(h, &h->d_err, nullptr, 1))) {
     free_handle(h);
     return rc;
@@ -642,11 +674,9 @@ static DecodeParams decode_params(const aecct_handle *h, int64_t B, const float 
   p.lparams = h->lparams, p.emb = h->emb, p.spe = h->spe, p.w_d1 = h->w_d1, p.b_d1 = h->b_d1;
   p.w_out = h->w_out, p.b_out = h->b_out, p.hbits = h->hbits, p.hwords = h->hwords;
   p.perm = h->perm, p.pos = h->pos;
-  p.plan_task = h->plan_task;
-  p.plan_grp = reinterpret_cast<const uint4 *>(h->plan_grp);
-  p.plan_uinfo = h->plan_uinfo;
-  p.plan_ulist = reinterpret_cast<const uint4 *>(h->plan_ulist);
-  p.plan_mask = reinterpret_cast<const uint4 *>(h->plan_mask);
+  p.plan_blob = reinterpret_cast<const uint4 *>(h->plan_blob), p.plan_bytes = h->plan_bytes;
+  p.off_task = h->off_task, p.off_grp = h->off_grp;
+  p.off_uinfo = h->off_uinfo, p.off_ulist = h->off_ulist, p.off_mask = h->off_mask;
   p.mask_info[0] = h->mask_info[0], p.mask_info[1] = h->mask_info[1];
   p.mask_list[0] = reinterpret_cast<const uint4 *>(h->mask_list[0]);
   p.mask_list[1] = reinterpret_cast<const uint4 *>(h->mask_list[1]);
@@ -856,7 +886,7 @@ int aecct_query(const aecct_handle *h, int32_t *cluster_ctas, int32_t *words_per
   if (h->d == 32) sm = tasks ? SmemLayout<32, true>::kTotal : SmemLayout<32>::kTotal;
   else if (h->d == 64) sm = tasks ? SmemLayout<64, true>::kTotal : SmemLayout<64>::kTotal;
   else sm = tasks ? SmemLayout<128, true>::kTotal : SmemLayout<128>::kTotal;
-  if (smem_bytes) *smem_bytes = sm;
+  if (smem_bytes) *smem_bytes = sm + static_cast<int32_t>(h->plan_bytes);
   if (attention_mode) *attention_mode = h->att == 1 ? 2 : (h->att == 2 ? 3 : 1);
   return AECCT_OK;
 }

@@ -453,7 +453,7 @@ __device__ __forceinline__ bool contiguous(const uint4 &w) {
 // Keys go two at a time through f32x2 instructions: the two lanes of a pair are independent
 // computations, and the folds into l and num stay sequential in key order.
 template <int DH, uint32_t STRIDE>
-__device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int cnt, const uint4 *__restrict__ ul,
+__device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int cnt, const uint4 *ul,
                                           const uint8_t *rows, uint32_t kslot, float scale, uint32_t tcache,
                                           float *A) {
   auto kptr = [&](int off) { return reinterpret_cast<const float4 *>(rows + off * STRIDE + kslot); };
@@ -481,7 +481,7 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
   // instead of reloading K and recomputing the dot products (same values, bit for bit).
   float mx = -INFINITY;
   for (int jb = 0; jb < cnt; jb += 16) {
-    const uint4 w = __ldg(ul + (jb >> 4));
+    const uint4 w = ul[jb >> 4];
     const uint32_t seg = segment(jb);
     const int nk = min(16, cnt - jb);
     float sgs[16];
@@ -558,7 +558,7 @@ __device__ __forceinline__ void hpsa_task(const float *q, const uint4 mask, int 
     }
   };
   for (int jb = 0; jb < cnt; jb += 16) {
-    const uint4 w = __ldg(ul + (jb >> 4));
+    const uint4 w = ul[jb >> 4];
     const uint32_t seg = segment(jb);
     const int nk = min(16, cnt - jb);
     if (jb < kTaskCache) {
@@ -1094,6 +1094,11 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   tc_fence_after();
   const uint32_t tmem = *s_tmem;
   const Ctl ctl{s_abort, p.err, p.wait_limit};
+  // the attention plan, into shared memory (read by every task of every block); the first CTA-wide
+  // barrier of the group loop orders it before its readers
+  uint8_t *const splan = smem + L::kTotal;
+  for (uint32_t i = threadIdx.x; i < p.plan_bytes / 16u; i += kThreads)
+    reinterpret_cast<uint4 *>(splan)[i] = __ldg(p.plan_blob + i);
 
   const Issuer<D, ATT> issuer{sb, tmem, ctl, s_issued};
   if (warp == 0 && cluster_id < p.n_groups) issuer.prologue(p.wstream);
@@ -1394,17 +1399,18 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           const uint32_t tcache = tmem + (static_cast<uint32_t>(32 * (warp & 3)) << 16) + L::kTaskCacheCol +
                                   static_cast<uint32_t>(warp >> 2) * kTaskCache;
           for (int k = 0; k < kMaxTasks; ++k) {
-            const uint32_t task = __ldg(p.plan_task + warp * kMaxTasks + k);
+            const uint32_t task = reinterpret_cast<const uint16_t *>(splan + p.off_task)[warp * kMaxTasks + k];
             if (task == 0xFFFFu) break;
             const int grp = static_cast<int>(task >> 3), e = static_cast<int>(task & 7u);
             const int ring = e < p.h_first ? 0 : 1;
-            const uint4 gi = __ldg(p.plan_grp + grp);
+            const uint4 gi = reinterpret_cast<const uint4 *>(splan + p.off_grp)[grp];
             const bool act = lane < static_cast<int>(gi.y);
             const int row = static_cast<int>(gi.x) + (act ? lane : 0);
             // a lane past the group's rows computes on row 0 and its result is dropped; an all-ones
             // mask keeps it from breaking the dense fast path
-            const uint4 mk = act ? __ldg(p.plan_mask + (grp * 2 + ring) * 32 + lane) : make_uint4(~0u, ~0u, ~0u, ~0u);
-            const uint32_t ui = __ldg(p.plan_uinfo + grp * 2 + ring);
+            const uint4 mk = act ? reinterpret_cast<const uint4 *>(splan + p.off_mask)[(grp * 2 + ring) * 32 + lane]
+                                 : make_uint4(~0u, ~0u, ~0u, ~0u);
+            const uint32_t ui = reinterpret_cast<const uint32_t *>(splan + p.off_uinfo)[grp * 2 + ring];
             float q[DH], a[DH];
             if constexpr (L::kQInSmem) {
               const float4 *qp = reinterpret_cast<const float4 *>(smem + L::kOffU + row * L::kKvStride + e * L::kSlot);
@@ -1421,7 +1427,8 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
               if (cap) capture_acc(l, 0, qa, e * DH, DH);
               dequant<DH>(qa, fq, bq, q);
             }
-            hpsa_task<DH, L::kKvStride>(q, mk, static_cast<int>(ui & 255u), p.plan_ulist + (ui >> 8),
+            hpsa_task<DH, L::kKvStride>(q, mk, static_cast<int>(ui & 255u),
+                                        reinterpret_cast<const uint4 *>(splan + p.off_ulist) + (ui >> 8),
                                         smem + L::kOffU + gi.z * L::kKvStride,
                                         e * L::kSlot + (L::kQInSmem ? 4 * DH : 0), p.att_scale, tcache, a);
             if constexpr (L::kQInSmem) {
@@ -1934,10 +1941,11 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
 }
 
 template <int D, int ATT, int ACT, int LIN>
-cudaError_t prepare_decode_kernel(int cluster_ctas, int *max_active_clusters) {
+cudaError_t prepare_decode_kernel(int cluster_ctas, uint32_t plan_bytes, int *max_active_clusters) {
   using L = SmemLayout<D, ATT == 1>;
+  const uint32_t total = L::kTotal + plan_bytes;
   cudaError_t e = cudaFuncSetAttribute(aecct_decoder_kernel<D, ATT, ACT, LIN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(L::kTotal));
+                                       static_cast<int>(total));
   if (e != cudaSuccess) return e;
   // ask for the smallest shared-memory carve-out that holds one CTA (1 KB of it is reserved by
   // the system): the rest of the 256 KB unified array stays L1 for spills and parameter loads
@@ -1946,7 +1954,7 @@ cudaError_t prepare_decode_kernel(int cluster_ctas, int *max_active_clusters) {
   if ((e = cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev)) != cudaSuccess)
     return e;
   if (smem_sm > 0) {
-    const int pct = static_cast<int>((100ll * (L::kTotal + 1024) + smem_sm - 1) / smem_sm);
+    const int pct = static_cast<int>((100ll * (total + 1024) + smem_sm - 1) / smem_sm);
     e = cudaFuncSetAttribute(aecct_decoder_kernel<D, ATT, ACT, LIN>, cudaFuncAttributePreferredSharedMemoryCarveout,
                              pct > 100 ? 100 : pct);
     if (e != cudaSuccess) return e;
@@ -1959,7 +1967,7 @@ cudaError_t prepare_decode_kernel(int cluster_ctas, int *max_active_clusters) {
   attr[0].val.clusterDim.z = 1;
   cfg.gridDim = dim3(cluster_ctas, 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = L::kTotal;
+  cfg.dynamicSmemBytes = total;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaOccupancyMaxActiveClusters(max_active_clusters, aecct_decoder_kernel<D, ATT, ACT, LIN>, &cfg);
@@ -1976,7 +1984,7 @@ cudaError_t launch_decode(const DecodeParams &p, cudaStream_t stream) {
   attr[0].val.clusterDim.z = 1;
   cfg.gridDim = dim3(p.n_clusters * p.C, 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = L::kTotal;
+  cfg.dynamicSmemBytes = L::kTotal + p.plan_bytes;
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = 1;

@@ -251,8 +251,8 @@ def test_warp_tasks_row_limits_exact(label, make, d, layers, B):
             assert (a.view(np.int32) if a.dtype == np.float32 else a).tolist() == \
                 (b.view(np.int32) if b.dtype == np.float32 else b).tolist(), f"{label} mode {mode}: {name}"
         dec.close()
-    if d == 128:  # Q stays in TMEM: every mode lays out shared memory alike
-        assert smem[1] == smem[2] == smem[3]
+    if d == 128:  # Q stays in TMEM: every mode lays out shared memory alike (tasks add their plan)
+        assert smem[1] == smem[3] and 0 < smem[2] - smem[1] <= 8192
 
 
 @pytest.mark.gpu

@@ -41,6 +41,8 @@ CASES = [
     ("bch63_36", 128, 2, dict(activation=1, alpha_mode=1), (1,)),
     ("bch63_36", 128, 2, dict(activation=1, h_first=2), (1, 2)),
     ("bch63_36", 128, 1, dict(mask_mode=1), (1, 2)),
+    ("bch63_36", 128, 1, dict(h_first=6), (1, 2, 3)),
+    ("bch63_36", 128, 1, dict(h_first=1), (2, 3)),
 ]
 
 
