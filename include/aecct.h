@@ -134,7 +134,9 @@ typedef struct {
 
 /* Validate the description, build the HPSA masks from H (Sec. 4.2: first ring = Tanner
  * graph neighbours, second ring = nodes at distance two, plus the node itself), lay the
- * weights out for the tensor cores and copy everything to the current device.  On
+ * weights out for the tensor cores and copy everything to the current device (AAP linears:
+ * the 2-bit codes are copied as they are and expanded into bf16 tensor-core tiles by a kernel
+ * on the device; the call waits for it).  On
  * success *out receives a new handle.  Errors: INVALID_ARG (bad dimension, H not 0/1,
  * zero row/column in H, h_first > heads, d_spe >= d, packed code 10, NULL pointer),
  * UNSUPPORTED (d, heads, ffn_mult or T outside this build), NO_DEVICE, OUT_OF_MEMORY, CUDA. */
@@ -188,6 +190,28 @@ int aecct_decode_host(aecct_handle *h, const float *y_host, int64_t B, uint8_t *
 #define AECCT_NOALLOC_SCRATCH_BYTES (4u << 20)
 int aecct_decode_host_noalloc(aecct_handle *h, const float *y_host, int64_t B, uint8_t *bits_host,
                               uint8_t *syndrome_host, float *logits_host, void *cuda_stream);
+
+/* The AAP weight quantiser of Sec. 4.1 (eq. Ternary), as the training forward applies it to each
+ * weight tensor (biases excluded), on the GPU:
+ *   gamma = Percentile(|W|, 0.5): the median of |W|, interpolated linearly between the two middle
+ *     order statistics (position 0.5 (len - 1)) when len is even;
+ *   scale = gamma * delta (fp32);
+ *   Ternary(W) = RoundClip(W / (scale + eps), -1, 1), an IEEE fp32 division, round to nearest even.
+ * The straight-through estimator of training passes the gradient of scale * Ternary(W) to W
+ * unchanged, so the forward values are all it needs.
+ *   w_dev       DEVICE fp32, the n_tensors tensors back to back (tensor j has len_host[j]
+ *               elements, a multiple of 4, at least 4, at most 2^31; finite values).
+ *   len_host    HOST [n_tensors]; delta_host HOST [n_tensors] (the learnable delta, > 0).
+ *   eps         > 0 (keeps the division finite when gamma delta is 0).
+ *   packed_dev  DEVICE, len/4 bytes per tensor back to back: the 2-bit format of w_packed above
+ *               (weight i of the tensor at bits 2 (i % 4) of byte i / 4: 00 = 0, 01 = +1, 11 = -1).
+ *   scale_dev   DEVICE fp32 [n_tensors]: gamma * delta (the w_scale of aecct_create).
+ *   wq_dev      DEVICE fp32 like w_dev, or NULL: scale * Ternary(W), the weights the training
+ *               forward multiplies with.
+ * Asynchronous on cuda_stream.  Errors: INVALID_ARG (a length or delta out of range, eps <= 0,
+ * a NULL pointer), CUDA. */
+int aecct_aap_ternarize(const float *w_dev, int32_t n_tensors, const int64_t *len_host, const float *delta_host,
+                        float eps, uint8_t *packed_dev, float *scale_dev, float *wq_dev, void *cuda_stream);
 
 /* Wait for the handle's last decode and report whether its kernel stopped on a
  * device-side timeout (AECCT_ERR_TIMEOUT) or a CUDA error occurred. */

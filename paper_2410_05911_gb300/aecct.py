@@ -25,7 +25,7 @@ AECCT_ERR_NO_DEVICE = -6
 EXPORTED_SYMBOLS = (
     "aecct_create", "aecct_decode", "aecct_decode_host", "aecct_synchronize", "aecct_set_capture",
     "aecct_query", "aecct_destroy", "aecct_status_string", "aecct_last_error", "aecct_selftest_mma",
-    "aecct_selftest_timeout", "aecct_decode_host_noalloc", "aecct_selftest_fma_rate",
+    "aecct_selftest_timeout", "aecct_decode_host_noalloc", "aecct_selftest_fma_rate", "aecct_aap_ternarize",
 )
 
 
@@ -84,6 +84,7 @@ def load(build_if_missing: bool = True):
     L.aecct_selftest_mma.argtypes = [P, P, I32, I32, P]
     L.aecct_selftest_timeout.argtypes = [I64, ctypes.POINTER(I32)]
     L.aecct_selftest_fma_rate.argtypes = [I32, ctypes.POINTER(ctypes.c_double)]
+    L.aecct_aap_ternarize.argtypes = [P, I32, P, P, ctypes.c_float, P, P, P, P]
     for name in EXPORTED_SYMBOLS:
         fn = getattr(L, name)
         if fn.restype is None or fn.restype is ctypes.c_int:
@@ -321,3 +322,28 @@ def selftest_fma_rate(paired: bool) -> float:
     v = ctypes.c_double()
     _check(load().aecct_selftest_fma_rate(1 if paired else 0, ctypes.byref(v)), "aecct_selftest_fma_rate")
     return v.value
+
+
+def aap_ternarize(tensors, delta=None, eps: float = 1e-8, want_weights: bool = False, stream=None):
+    """aecct_aap_ternarize: eq. Ternary on the GPU for a list of float32 CUDA tensors (each with a
+    multiple of 4 elements).  Returns (packed uint8 codes per tensor, scales float32 [n], and the
+    weights scale * Ternary(W) per tensor when want_weights)."""
+    import torch
+
+    if not tensors:
+        return [], None, None
+    dev = tensors[0].device
+    flat = torch.cat([t.reshape(-1).to(torch.float32) for t in tensors]).contiguous()
+    lens = np.array([t.numel() for t in tensors], np.int64)
+    deltas = np.asarray(delta if delta is not None else np.ones(len(tensors)), np.float32)
+    packed = torch.empty(int(lens.sum()) // 4, dtype=torch.uint8, device=dev)
+    scale = torch.empty(len(tensors), dtype=torch.float32, device=dev)
+    wq = torch.empty_like(flat) if want_weights else None
+    s = stream if stream is not None else torch.cuda.current_stream(dev)
+    _check(load().aecct_aap_ternarize(flat.data_ptr(), len(tensors), lens.ctypes.data, deltas.ctypes.data, float(eps),
+                                      packed.data_ptr(), scale.data_ptr(), wq.data_ptr() if wq is not None else None,
+                                      s.cuda_stream), "aecct_aap_ternarize")
+    offs = np.concatenate([[0], np.cumsum(lens)])
+    codes = [packed[offs[j] // 4:offs[j + 1] // 4] for j in range(len(tensors))]
+    wqs = [wq[offs[j]:offs[j + 1]].view(tensors[j].shape) for j in range(len(tensors))] if wq is not None else None
+    return codes, scale, wqs

@@ -231,6 +231,13 @@ constexpr uint32_t kMaxDynSmem = 232448;  // the largest dynamic shared memory a
 constexpr int kStagedMaxRows = 640;  // staged attention: rows of a group (128 bytes each in 80 KB)
 constexpr int kStagedMaxKeys = 256;  // staged attention: keys per row (TMEM columns [128, 384))
 
+// aap.cu: the AAP weight quantiser (eq. Ternary) and the GPU expansion of 2-bit weights
+constexpr int kTernarizeMaxTensors = 64;  // tensors per launch (the launcher splits larger calls)
+cudaError_t launch_aap_ternarize(const float *w, int n, const int64_t *len, const float *delta, float eps,
+                                 uint8_t *packed, float *scale, float *wq, cudaStream_t stream);
+cudaError_t launch_unpack_weights(const uint8_t *packed, int n_layers, int D, const ChunkDesc *chunks, int n_chunks,
+                                  uint32_t layer_bytes, uint8_t *wstream, cudaStream_t stream);
+
 // api.cu diagnostics kernels live in selftest.cu
 cudaError_t run_selftest_mma(const int8_t *a_host, const int8_t *b_host, int K, int N, float *out_host);
 cudaError_t run_selftest_timeout(long long limit_cycles, int *status_host);

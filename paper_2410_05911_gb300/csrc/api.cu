@@ -553,8 +553,11 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
   const uint32_t off = h->chunks[nch - 1].off + h->chunks[nch - 1].bytes;
   h->n_chunks = nch;
   h->layer_bytes = off;
-  std::vector<uint16_t> ws((size_t)d.n_layers * off / 2, 0);
-  {
+  // AAP linears: the 2-bit codes go to the device as they are and a kernel expands them there
+  // (aap.cu, unpack_weights_kernel); full-precision linears are rounded to bf16 and laid out here
+  const bool gpu_unpack = d.linear_mode == 0;
+  std::vector<uint16_t> ws(gpu_unpack ? 0 : (size_t)d.n_layers * off / 2, 0);
+  if (!gpu_unpack) {
     const size_t per_layer_packed = 12u * (size_t)D * D / 4u, per_layer_full = 12u * (size_t)D * D;
     std::vector<uint16_t> W[4];  // bf16 encodings, [N][K] per GEMM
     for (int l = 0; l < d.n_layers; ++l) {
@@ -629,7 +632,8 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
     }
   }
   const int de = D - d.d_spe;
-  if ((rc = dev_upload(h, &h->wstream, reinterpret_cast<const uint8_t *>(ws.data()), ws.size() * 2)) ||
+  if ((rc = dev_upload(h, &h->wstream, gpu_unpack ? nullptr : reinterpret_cast<const uint8_t *>(ws.data()),
+                      (size_t)d.n_layers * off)) ||
       (rc = dev_upload(h, &h->lparams, lpv.data(), lpv.size())) ||
       (rc = dev_upload(h, &h->emb, d.emb, (size_t)T * de)) ||
       (rc = dev_upload(h, &h->spe, d.spe, (size_t)T * d.d_spe)) ||
@@ -647,6 +651,19 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
       (rc = dev_upload<int>(h, &h->d_err, nullptr, 1))) {
     free_handle(h);
     return rc;
+  }
+  if (gpu_unpack) {
+    uint8_t *packed = nullptr;
+    const size_t pbytes = (size_t)d.n_layers * 3u * (size_t)D * D;
+    if ((e = cudaMalloc(&packed, pbytes)) == cudaSuccess &&
+        (e = cudaMemcpy(packed, d.w_packed, pbytes, cudaMemcpyHostToDevice)) == cudaSuccess &&
+        (e = launch_unpack_weights(packed, d.n_layers, D, h->chunks, nch, off, h->wstream, nullptr)) == cudaSuccess)
+      e = cudaDeviceSynchronize();
+    cudaFree(packed);
+    if (e != cudaSuccess) {
+      free_handle(h);
+      return cuda_fail(e, "weight unpack");
+    }
   }
   if ((e = cudaMemset(h->d_err, 0, sizeof(int))) != cudaSuccess ||
       (e = cudaHostAlloc(reinterpret_cast<void **>(&h->h_err), sizeof(int), cudaHostAllocDefault)) != cudaSuccess ||
@@ -913,6 +930,21 @@ int aecct_selftest_timeout(int64_t limit_cycles, int32_t *status_host) {
   if (e != cudaSuccess) return cuda_fail(e, "selftest timeout");
   *status_host = st == 1 ? AECCT_ERR_TIMEOUT : (st == 0 ? AECCT_OK : AECCT_ERR_CUDA);
   return AECCT_OK;
+}
+
+int aecct_aap_ternarize(const float *w_dev, int32_t n_tensors, const int64_t *len_host, const float *delta_host,
+                        float eps, uint8_t *packed_dev, float *scale_dev, float *wq_dev, void *cuda_stream) {
+  if (n_tensors < 0 || (n_tensors > 0 && (!w_dev || !len_host || !delta_host || !packed_dev || !scale_dev)))
+    return AECCT_ERR_INVALID_ARG;
+  if (!(eps > 0.0f) || !std::isfinite(eps)) return AECCT_ERR_INVALID_ARG;
+  for (int j = 0; j < n_tensors; ++j) {
+    if (len_host[j] < 4 || len_host[j] % 4 != 0 || len_host[j] > (int64_t(1) << 31)) return AECCT_ERR_INVALID_ARG;
+    if (!(delta_host[j] > 0.0f) || !std::isfinite(delta_host[j])) return AECCT_ERR_INVALID_ARG;
+  }
+  if (n_tensors == 0) return AECCT_OK;
+  const cudaError_t e = launch_aap_ternarize(w_dev, n_tensors, len_host, delta_host, eps, packed_dev, scale_dev, wq_dev,
+                                             static_cast<cudaStream_t>(cuda_stream));
+  return e == cudaSuccess ? AECCT_OK : cuda_fail(e, "aap ternarize launch");
 }
 
 int aecct_selftest_fma_rate(int32_t paired, double *fma_per_s) {

@@ -165,3 +165,21 @@ def test_caller_outputs_are_checked_before_the_kernel_writes_them():
     for out in bad:
         with pytest.raises(ValueError):
             A.check_outputs(out, B, n, m, cpu)
+
+
+def test_aap_ternarize_rejects_bad_arguments_before_any_device_work():
+    L = A.load()
+    lens = np.array([8, 6], np.int64)  # 6 is not a multiple of 4
+    deltas = np.ones(2, np.float32)
+    P = 0x1000  # never dereferenced: the arguments are refused first
+    assert L.aecct_aap_ternarize(P, 2, lens.ctypes.data, deltas.ctypes.data, 1e-8, P, P, None, None) == \
+        A.AECCT_ERR_INVALID_ARG
+    lens = np.array([8, 4], np.int64)
+    assert L.aecct_aap_ternarize(P, 2, lens.ctypes.data, deltas.ctypes.data, 0.0, P, P, None, None) == \
+        A.AECCT_ERR_INVALID_ARG  # eps must be > 0
+    bad = np.array([1.0, -1.0], np.float32)
+    assert L.aecct_aap_ternarize(P, 2, lens.ctypes.data, bad.ctypes.data, 1e-8, P, P, None, None) == \
+        A.AECCT_ERR_INVALID_ARG  # delta must be > 0
+    assert L.aecct_aap_ternarize(None, 2, lens.ctypes.data, deltas.ctypes.data, 1e-8, P, P, None, None) == \
+        A.AECCT_ERR_INVALID_ARG
+    assert L.aecct_aap_ternarize(None, 0, None, None, 1e-8, None, None, None, None) == A.AECCT_OK
