@@ -213,6 +213,25 @@ int aecct_decode_host_noalloc(aecct_handle *h, const float *y_host, int64_t B, u
 int aecct_aap_ternarize(const float *w_dev, int32_t n_tensors, const int64_t *len_host, const float *delta_host,
                         float eps, uint8_t *packed_dev, float *scale_dev, float *wq_dev, void *cuda_stream);
 
+/* The spectral positional encoding of Sec. 4.3 computed on the GPU, in double precision: the table
+ * aecct_create takes as `spe`.  Tanner graph of H (variables 0..n-1, checks n..n+m-1, m = n - k,
+ * T = n + m <= 1024 nodes), Laplacian L = D - A, its eigenpairs (lambda_i, phi_i) in ascending order
+ * (parallel Jacobi rotations) in the canonical basis (per cluster of eigenvalues within 1e-8 max(1,
+ * |lambda|max) of each other: Gram-Schmidt of P e_0, P e_1, ... in node order, P the cluster's
+ * projector, residuals of norm <= 1e-6 skipped; a simple eigenvalue's vector has a positive first
+ * entry above 1e-6 in magnitude), then for every node j:
+ *   X_j = Phi_j W_pe, Phi_j row i = (lambda_i, phi_i[j]);
+ *   MHSA(X_j) = [softmax((X_j Wq_e)(X_j Wk_e)^T / sqrt(d_e)) (X_j Wv_e)]_e Wo, d_e = d_spe / heads;
+ *   SPE_j = the mean of the T rows of MHSA(X_j) (average pooling as the reduction W_{(2n-k)->1}).
+ * All pointers HOST: H [(n-k)][n] 0/1; w_pe [2][d_spe]; wq, wk, wv [heads][d_spe][d_e]; wo
+ * [d_spe][d_spe] (fp64, row-major).  Outputs: spe_out fp32 [T][d_spe]; lam_out [T], U_out [T][T]
+ * (column i = eigenvector i), spe64_out [T][d_spe] fp64, each NULL when not wanted.  Synchronous;
+ * allocates and frees its device memory.  Errors: INVALID_ARG, UNSUPPORTED (a cluster's basis came
+ * out short), CUDA. */
+int aecct_spe_table(const uint8_t *H, int32_t n, int32_t k, int32_t d_spe, int32_t heads, const double *w_pe,
+                    const double *wq, const double *wk, const double *wv, const double *wo, float *spe_out,
+                    double *lam_out, double *U_out, double *spe64_out);
+
 /* Wait for the handle's last decode and report whether its kernel stopped on a
  * device-side timeout (AECCT_ERR_TIMEOUT) or a CUDA error occurred. */
 int aecct_synchronize(aecct_handle *h);

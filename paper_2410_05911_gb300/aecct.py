@@ -26,6 +26,7 @@ EXPORTED_SYMBOLS = (
     "aecct_create", "aecct_decode", "aecct_decode_host", "aecct_synchronize", "aecct_set_capture",
     "aecct_query", "aecct_destroy", "aecct_status_string", "aecct_last_error", "aecct_selftest_mma",
     "aecct_selftest_timeout", "aecct_decode_host_noalloc", "aecct_selftest_fma_rate", "aecct_aap_ternarize",
+    "aecct_spe_table",
 )
 
 
@@ -85,6 +86,7 @@ def load(build_if_missing: bool = True):
     L.aecct_selftest_timeout.argtypes = [I64, ctypes.POINTER(I32)]
     L.aecct_selftest_fma_rate.argtypes = [I32, ctypes.POINTER(ctypes.c_double)]
     L.aecct_aap_ternarize.argtypes = [P, I32, P, P, ctypes.c_float, P, P, P, P]
+    L.aecct_spe_table.argtypes = [P, I32, I32, I32, I32, P, P, P, P, P, P, P, P, P]
     for name in EXPORTED_SYMBOLS:
         fn = getattr(L, name)
         if fn.restype is None or fn.restype is ctypes.c_int:
@@ -347,3 +349,22 @@ def aap_ternarize(tensors, delta=None, eps: float = 1e-8, want_weights: bool = F
     codes = [packed[offs[j] // 4:offs[j + 1] // 4] for j in range(len(tensors))]
     wqs = [wq[offs[j]:offs[j + 1]].view(tensors[j].shape) for j in range(len(tensors))] if wq is not None else None
     return codes, scale, wqs
+
+
+def spe_table(H: np.ndarray, params, want_eigen: bool = False):
+    """aecct_spe_table: the SPE table of Sec. 4.3 computed on the GPU for parity-check matrix H and the
+    SPE parameters (w_pe, wq, wk, wv, wo).  Returns the fp32 table [T, d_spe], and with want_eigen
+    also (the fp64 table, eigenvalues [T], canonical eigenvectors [T, T])."""
+    H = np.ascontiguousarray(H, np.uint8)
+    m, n = H.shape
+    T = n + m
+    heads, d_spe = params.wq.shape[0], params.w_pe.shape[1]
+    ws = [np.ascontiguousarray(w, np.float64) for w in (params.w_pe, params.wq, params.wk, params.wv, params.wo)]
+    out = np.zeros((T, d_spe), np.float32)
+    lam = np.zeros(T) if want_eigen else None
+    U = np.zeros((T, T)) if want_eigen else None
+    t64 = np.zeros((T, d_spe)) if want_eigen else None
+    ptr = lambda a: a.ctypes.data if a is not None else None  # noqa: E731
+    _check(load().aecct_spe_table(H.ctypes.data, n, n - m, d_spe, heads, *[w.ctypes.data for w in ws], out.ctypes.data,
+                                  ptr(lam), ptr(U), ptr(t64)), "aecct_spe_table")
+    return (out, t64, lam, U) if want_eigen else out

@@ -15,7 +15,7 @@ CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(OUT_DIR, "libaecct.so")
 SOURCES = ["api.cu", "decoder_kernel.cu", "decoder_kernel_gelu.cu", "decoder_kernel_fp.cu", "decoder_kernel_fp_gelu.cu",
-           "selftest.cu", "aap.cu"]
+           "selftest.cu", "aap.cu", "spe.cu"]
 HEADERS = ["aecct_internal.h", "sm103_ptx.cuh", "decoder_kernel.cuh", os.path.join("..", "..", "include", "aecct.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--fmad=false",

@@ -238,6 +238,14 @@ cudaError_t launch_aap_ternarize(const float *w, int n, const int64_t *len, cons
 cudaError_t launch_unpack_weights(const uint8_t *packed, int n_layers, int D, const ChunkDesc *chunks, int n_chunks,
                                   uint32_t layer_bytes, uint8_t *wstream, cudaStream_t stream);
 
+// spe.cu: the spectral positional encoding (Sec. 4.3) on the GPU
+constexpr int kSpeMaxHeads = 8;
+constexpr int kSpeMaxTokens = 1024;
+cudaError_t run_spe_table(const uint8_t *H, int n, int m, int d_spe, int heads, const double *w_pe, const double *wq,
+                          const double *wk, const double *wv, const double *wo, double cluster_tol, double vanish_tol,
+                          float *spe_host, double *lam_host, double *U_host, double *spe64_host, int *sweeps,
+                          int *status_host);
+
 // api.cu diagnostics kernels live in selftest.cu
 cudaError_t run_selftest_mma(const int8_t *a_host, const int8_t *b_host, int K, int N, float *out_host);
 cudaError_t run_selftest_timeout(long long limit_cycles, int *status_host);

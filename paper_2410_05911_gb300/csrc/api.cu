@@ -932,6 +932,26 @@ int aecct_selftest_timeout(int64_t limit_cycles, int32_t *status_host) {
   return AECCT_OK;
 }
 
+int aecct_spe_table(const uint8_t *H, int32_t n, int32_t k, int32_t d_spe, int32_t heads, const double *w_pe,
+                    const double *wq, const double *wk, const double *wv, const double *wo, float *spe_out,
+                    double *lam_out, double *U_out, double *spe64_out) {
+  if (!H || !w_pe || !wq || !wk || !wv || !wo || !spe_out) return AECCT_ERR_INVALID_ARG;
+  if (n <= 0 || k <= 0 || k >= n || n + (n - k) > kSpeMaxTokens) return AECCT_ERR_INVALID_ARG;
+  if (heads < 1 || heads > kSpeMaxHeads || d_spe < heads || d_spe % heads != 0) return AECCT_ERR_INVALID_ARG;
+  const int m = n - k;
+  for (size_t i = 0; i < static_cast<size_t>(m) * n; ++i)
+    if (H[i] > 1) return AECCT_ERR_INVALID_ARG;
+  int sweeps = 0, status = 0;
+  const cudaError_t e = run_spe_table(H, n, m, d_spe, heads, w_pe, wq, wk, wv, wo, 1e-8, 1e-6, spe_out, lam_out, U_out,
+                                      spe64_out, &sweeps, &status);
+  if (e != cudaSuccess) return cuda_fail(e, "spe table");
+  if (status) {
+    g_last_error = "spe table: a cluster of equal eigenvalues did not yield a full canonical basis";
+    return AECCT_ERR_UNSUPPORTED;
+  }
+  return AECCT_OK;
+}
+
 int aecct_aap_ternarize(const float *w_dev, int32_t n_tensors, const int64_t *len_host, const float *delta_host,
                         float eps, uint8_t *packed_dev, float *scale_dev, float *wq_dev, void *cuda_stream) {
   if (n_tensors < 0 || (n_tensors > 0 && (!w_dev || !len_host || !delta_host || !packed_dev || !scale_dev)))
