@@ -1574,8 +1574,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           cluster_wait(bar_kvr, kvr_ph);
           static_assert(L::kOffW == L::kOffAop + L::kAopBytes, "the staging area spans the operand tile and the weight stages");
           constexpr uint32_t kSc = 128;  // the dead K and V accumulator columns [128, 384)
-          const uint32_t stg = sb + L::kOffAop;  // row rho of the group: 128 bytes at rho * 128, 16-byte slot f at f ^ (rho & 7)
-          const int nrows = p.G * Tp;            // <= 640 (checked at create)
+          const int nrows = p.G * Tp;  // <= 640 (checked at create)
+          // two staging buffers when two heads' rows fit the 80 KB: head e + 1 is gathered while
+          // nobody reads head e - 1's buffer any more, so one CTA barrier per head suffices
+          const bool dbuf = 2 * nrows * 128 <= static_cast<int>(L::kAopBytes + 3 * L::kStageBytes);
           const int rowbase = g * Tp;
           auto dot16 = [&](const float *q, const float4 *kk) -> float {
             float2 d2 = make_float2(0.0f, 0.0f);
@@ -1587,6 +1589,8 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             return __fadd_rn(d2.x, d2.y);
           };
           for (int e = 0; e < kHeads; ++e) {
+            // row rho of the group: 128 bytes at rho * 128, 16-byte slot f at f ^ (rho & 7)
+            const uint32_t stg = sb + L::kOffAop + ((dbuf && (e & 1)) ? static_cast<uint32_t>(nrows) * 128u : 0u);
             {
               // gather: item it = (row rho, 16-byte slot f of the head's K|V), 10 items per thread at most
               float4 v[5];
@@ -1706,7 +1710,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             }
             tmem_wait_st();
             tc_fence_before();
-            named_bar_sync(5, kEpiThreads);  // the staging area is free for the next head
+            // the staging area is free for the next head (two buffers: the next head's gather barrier
+            // orders this head's reads before the gather after it; the last head's barrier orders
+            // the attention outputs in TMEM before Quant(A))
+            if (!dbuf || e == kHeads - 1) named_bar_sync(5, kEpiThreads);
             tc_fence_after();
           }
           // O's weights into W0, W1 (free again), while the codes of A are made
