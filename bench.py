@@ -64,16 +64,17 @@ def kernel_sources_digest() -> str:
 
 
 def measured_traffic(workload: str, batch: int):
-    """DRAM bytes per launch from the committed ncu record of this workload, scaled to `batch`
-    words, or None when there is no record or the kernel sources changed since it was taken."""
+    """DRAM bytes of one launch from the committed ncu record of this workload at this batch, or
+    None when there is no record for it or the kernel sources changed since it was taken (the
+    weights are read once per launch whatever the batch, so a record does not scale to another)."""
     path = os.path.join(ROOT, "profiles", f"aecct_decoder_kernel{I.WORKLOADS[workload]['d']}_{workload}_dram.json")
     if not os.path.exists(path):
         return None
     with open(path) as f:
         rec = json.load(f)
-    if rec.get("sources_sha256") != kernel_sources_digest() or rec.get("workload") != workload:
+    if rec.get("sources_sha256") != kernel_sources_digest() or rec.get("workload") != workload or rec.get("batch") != batch:
         return None
-    return (rec["dram_bytes_read"] + rec["dram_bytes_write"]) * batch / rec["batch"]
+    return rec["dram_bytes_read"] + rec["dram_bytes_write"]
 
 
 def max_over_ranks(x: float, world: int, device=None) -> float:

@@ -41,16 +41,17 @@ def test_polar_alu_ops_figure():
     assert abs(ops / 1e6 - 7.33) < 0.005
 
 
-def test_traffic_record_gated_on_kernel_sources(monkeypatch):
+def test_traffic_record_gated_on_kernel_sources_and_batch(monkeypatch, tmp_path):
     import json
-    import os
-    path = os.path.join(bench.ROOT, "profiles", "aecct_decoder_kernel64_polar64_32_dram.json")
-    with open(path) as f:
-        sha = json.load(f)["sources_sha256"]
-    monkeypatch.setattr(bench, "kernel_sources_digest", lambda: sha)
-    rec = bench.measured_traffic("polar64_32", 16384)
-    assert rec is not None and rec > 4.19e6  # at least the y a 16,384-word launch must read
-    assert bench.measured_traffic("polar64_32", 32768) == pytest.approx(2 * rec)
-    assert bench.measured_traffic("bch31_16", 16384) is None  # no record for this workload
+    os_ = __import__("os")
+    os_.makedirs(tmp_path / "profiles")
+    rec = dict(workload="bch63_36", batch=262144, dram_bytes_read=9.0e6, dram_bytes_write=1.0e6, sources_sha256="a" * 64)
+    with open(tmp_path / "profiles" / "aecct_decoder_kernel128_bch63_36_dram.json", "w") as f:
+        json.dump(rec, f)
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    monkeypatch.setattr(bench, "kernel_sources_digest", lambda: "a" * 64)
+    assert bench.measured_traffic("bch63_36", 262144) == 10.0e6
+    assert bench.measured_traffic("bch63_36", 4096) is None      # another batch: not scaled
+    assert bench.measured_traffic("polar64_32", 65536) is None   # no record for this workload
     monkeypatch.setattr(bench, "kernel_sources_digest", lambda: "0" * 64)
-    assert bench.measured_traffic("polar64_32", 16384) is None
+    assert bench.measured_traffic("bch63_36", 262144) is None    # the kernel changed since
