@@ -170,6 +170,10 @@ struct DecodeParams {
   int32_t *cap_acc;
   float *cap_alpha;
   uint8_t *cap_syn;
+  // staged attention (d = 128): K and V of every row, per cluster, in global memory (L2), read back
+  // head by head with bulk copies: [cluster][8 heads][K, V][C * 128 rows][16 floats], 16-byte
+  // piece f of row rho at f ^ ((rho >> 1) & 3)
+  float *kv_scratch;
   // control
   int *err;  // device word, bit 0 = a bounded wait timed out
   long long wait_limit;
@@ -228,7 +232,7 @@ cudaError_t launch_decode(const DecodeParams &p, cudaStream_t stream);
 template <int D, int ATT, int ACT, int LIN>
 cudaError_t prepare_decode_kernel(int cluster_ctas, uint32_t plan_bytes, int *max_active_clusters);
 constexpr uint32_t kMaxDynSmem = 232448;  // the largest dynamic shared memory a CTA may opt into (227 KB)
-constexpr int kStagedMaxRows = 640;  // staged attention: rows of a group (128 bytes each in 80 KB)
+constexpr int kStagedMaxRows = 640;  // staged attention: rows of a group (64 bytes of K and of V each, 40 KB + 40 KB)
 constexpr int kStagedMaxKeys = 256;  // staged attention: keys per row (TMEM columns [128, 384))
 
 // aap.cu: the AAP weight quantiser (eq. Ternary) and the GPU expansion of 2-bit weights

@@ -50,6 +50,7 @@ struct aecct_handle {
   int hwords = 0;
   uint16_t *mask_list[2] = {nullptr, nullptr};
   uint16_t *perm = nullptr, *pos = nullptr;
+  float *kv_scratch = nullptr;  // staged attention: K and V rows per cluster
   uint8_t *plan_blob = nullptr;  // the attention plan (task mode), copied into shared memory by the kernel
   uint32_t plan_bytes = 0, off_task = 0, off_grp = 0, off_uinfo = 0, off_ulist = 0, off_mask = 0;
   int *d_err = nullptr;
@@ -648,6 +649,8 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
       (rc = dev_upload(h, &h->mask_info[1], minfo[1].data(), minfo[1].size())) ||
       (rc = dev_upload(h, &h->mask_list[1], mlist[1].data(), mlist[1].size())) ||
       (rc = dev_upload(h, &h->plan_blob, blob.data(), blob.size())) ||
+      (rc = dev_upload<float>(h, &h->kv_scratch, nullptr,
+                              att == 2 ? (size_t)max_clusters * best_C * kRows * kHeads * 2 * 16 : 1)) ||
       (rc = dev_upload<int>(h, &h->d_err, nullptr, 1))) {
     free_handle(h);
     return rc;
@@ -699,6 +702,7 @@ static DecodeParams decode_params(const aecct_handle *h, int64_t B, const float 
   p.mask_list[1] = reinterpret_cast<const uint4 *>(h->mask_list[1]);
   p.ln_eps = h->ln_eps, p.alpha_floor = h->alpha_floor, p.att_scale = h->att_scale, p.alpha_mode = h->alpha_mode;
   p.cap_B = h->cap_B, p.cap_q = h->cap_q, p.cap_acc = h->cap_acc, p.cap_alpha = h->cap_alpha, p.cap_syn = h->cap_syn;
+  p.kv_scratch = h->kv_scratch;
   p.err = err_dev, p.wait_limit = h->wait_limit;
   return p;
 }

@@ -1056,7 +1056,9 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   volatile int *s_abort = reinterpret_cast<volatile int *>(smem + L::kOffMisc + 4);
   uint32_t *s_kvcl = reinterpret_cast<uint32_t *>(smem + L::kOffMisc + 8);   // [8] shared::cluster K/V bases per CTA
   uint64_t *s_zgen = reinterpret_cast<uint64_t *>(smem + L::kOffMisc + 72);   // [8] generic z bases per CTA
-  uint32_t *s_issued = reinterpret_cast<uint32_t *>(smem + L::kOffMisc + 136);  // [6] weight copies / phases armed
+  uint32_t *s_issued = reinterpret_cast<uint32_t *>(smem + L::kOffMisc + 136);  // [10] weight copies / phases armed
+  // staged attention: the barriers of the K and V buffers (buffer set 0; set 1 when two heads fit)
+  const uint32_t bar_sk = bar_fin + 32, bar_sv = bar_fin + 40;  // + 16: set 1
 
   if (tid == 0) {
     for (int s = 0; s < S; ++s) {
@@ -1071,9 +1073,9 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
     mbar_init(bar_zf, p.C);
     mbar_init(bar_fin, 1);
     if constexpr (D == 128)  // region U and the two operand-tile halves (d = 128 weight schedule)
-      for (int i = 0; i < 3; ++i) mbar_init(bar_fin + 8 + 8 * i, 1);
+      for (int i = 0; i < 7; ++i) mbar_init(bar_fin + 8 + 8 * i, 1);
     *s_abort = 0;
-    for (int i = 0; i < 6; ++i) s_issued[i] = 0;
+    for (int i = 0; i < 10; ++i) s_issued[i] = 0;
     // base of the K/V area of every CTA of the cluster as a shared::cluster address, and generic
     // base of its z area: this CTA's own through its plain shared-memory window, the others
     // through the distributed shared window
@@ -1365,14 +1367,28 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             capture_acc(l, 0, ka, D + e * DH, DH);
             capture_acc(l, 0, va, 2 * D + e * DH, DH);
           }
-          // head slot of this row: (K | V), or (Q | K | V) in task mode at d <= 64
-          const uint32_t dst = kvl + r * L::kKvStride + e * L::kSlot + (L::kQInSmem ? 4 * DH : 0);
           dequant<DH>(ka, fk, bk, ka);
           dequant<DH>(va, fv, bv, va);
+          if constexpr (STAGED) {
+            // K and V of this row and head, head-major in region U ([head][K, V][128 rows][64 B],
+            // 16-byte piece f of row r at f ^ ((r >> 1) & 3)): the layout of the cluster's scratch
+            // in global memory, where bulk copies take them next
+            const uint32_t kd = kvl + ((static_cast<uint32_t>(e) * 2u) * kRows + r) * 64u;
+            const uint32_t vd = kd + kRows * 64u;
 #pragma unroll
-          for (int i = 0; i < DH; i += 4) {
-            st_shared_f4(dst + 4 * i, ka[i], ka[i + 1], ka[i + 2], ka[i + 3]);
-            st_shared_f4(dst + 4 * (DH + i), va[i], va[i + 1], va[i + 2], va[i + 3]);
+            for (int f = 0; f < DH / 4; ++f) {
+              const uint32_t g = static_cast<uint32_t>((f ^ ((r >> 1) & 3)) << 4);
+              st_shared_f4(kd + g, ka[4 * f], ka[4 * f + 1], ka[4 * f + 2], ka[4 * f + 3]);
+              st_shared_f4(vd + g, va[4 * f], va[4 * f + 1], va[4 * f + 2], va[4 * f + 3]);
+            }
+          } else {
+            // head slot of this row: (K | V), or (Q | K | V) in task mode at d <= 64
+            const uint32_t dst = kvl + r * L::kKvStride + e * L::kSlot + (L::kQInSmem ? 4 * DH : 0);
+#pragma unroll
+            for (int i = 0; i < DH; i += 4) {
+              st_shared_f4(dst + 4 * i, ka[i], ka[i + 1], ka[i + 2], ka[i + 3]);
+              st_shared_f4(dst + 4 * (DH + i), va[i], va[i + 1], va[i + 2], va[i + 3]);
+            }
           }
           if constexpr (L::kQInSmem) {
             float qa[DH], bq[DH];
@@ -1564,21 +1580,68 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           }
         } else {
           // ---------------- S5: HPSA (Sec. 4.2), per-row lists over per-head staged rows (d = 128).
-          // Head by head, the K and V rows of the head for every row of the group are gathered from
-          // every CTA of the cluster (coalesced 16-byte reads) into this CTA's operand tile and weight
-          // stages, both idle here.  The row's 4 threads share the head: each takes 4 keys of every
-          // 16-key block for the scores and their exponentials (the row's TMEM lane, columns from
-          // kSc), and then folds every key, in ascending order, into 4 of the 16 features of num.
-          // The arithmetic is the canonical one, key for key and feature for feature.
+          // Every CTA of the cluster has left the K and V rows of its token rows in the cluster's
+          // scratch in global memory (L2).  Head by head, one bulk copy brings the K rows of the
+          // head for every row of the group into a K buffer and another the V rows into a V buffer
+          // (the operand tile and the weight stages, idle here: 40 KB each).  The next head's K is
+          // fetched while this head's exponentials and fold run, its V while its scores run.  The
+          // row's 4 threads share the head: each takes 4 keys of every 16-key block for the scores
+          // and their exponentials (the row's TMEM lane, columns from kSc), and then folds every
+          // key, in ascending order, into 4 of the 16 features of num.  The arithmetic is the
+          // canonical one, key for key and feature for feature.
+          // this CTA's K and V rows, from region U to the cluster's scratch in global memory: 16 bulk
+          // copies (one per head and kind, 8 KB each) by thread 0, complete before the cluster
+          // learns that they are there
+          fence_proxy_async_smem();  // this thread's K / V stores, before the bulk copies read them
+          named_bar_sync(5, kEpiThreads);
+          if (tid == 0 && !*s_abort) {
+            const int R = p.C * kRows;
+            for (int ek = 0; ek < 2 * kHeads; ++ek)
+              bulk_s2g(p.kv_scratch + (static_cast<size_t>(cluster_id) * 2 * kHeads + ek) * R * DH +
+                           static_cast<size_t>(crank) * kRows * DH,
+                       kvl + static_cast<uint32_t>(ek) * kRows * 64u, kRows * 64u);
+            bulk_commit_group();
+            bulk_wait_group_0();
+            fence_proxy_async_global();
+          }
           cluster_arrive(bar_kvr);
           cluster_wait(bar_kvr, kvr_ph);
-          static_assert(L::kOffW == L::kOffAop + L::kAopBytes, "the staging area spans the operand tile and the weight stages");
+          static_assert(L::kOffW == L::kOffAop + L::kAopBytes && L::kAopBytes + 3 * L::kStageBytes >= 2 * 40960,
+                        "the K and V buffers span the operand tile and the weight stages");
           constexpr uint32_t kSc = 128;  // the dead K and V accumulator columns [128, 384)
+          // row rho of the group: 64 bytes at rho * 64, 16-byte piece f at f ^ ((rho >> 1) & 3)
           const int nrows = p.G * Tp;  // <= 640 (checked at create)
-          // two staging buffers when two heads' rows fit the 80 KB: head e + 1 is gathered while
-          // nobody reads head e - 1's buffer any more, so one CTA barrier per head suffices
-          const bool dbuf = 2 * nrows * 128 <= static_cast<int>(L::kAopBytes + 3 * L::kStageBytes);
           const int rowbase = g * Tp;
+          const uint32_t fetch_bytes = static_cast<uint32_t>(nrows) * 64u;
+          // two sets of K and V buffers when they fit (LDPC(128,64): 4 x 12 KB): head e uses set
+          // e & 1 and the next-but-one head is fetched after head e, so each head needs one CTA
+          // barrier; one set otherwise (40 KB each), the next head fetched into each buffer as
+          // soon as its reads are over
+          const bool dbuf = 4u * fetch_bytes <= 81920u;
+          const float *kvs = p.kv_scratch + static_cast<size_t>(cluster_id) * kHeads * 2 * (p.C * kRows) * DH;
+          auto buf_of = [&](int e, int kind) -> uint32_t {
+            return dbuf ? sb + L::kOffAop + (static_cast<uint32_t>(e & 1) * 2u + kind) * fetch_bytes
+                        : sb + L::kOffAop + static_cast<uint32_t>(kind) * 40960u;
+          };
+          auto bar_of = [&](int e, int kind) -> uint32_t {
+            return (kind ? bar_sv : bar_sk) + ((dbuf && (e & 1)) ? 16u : 0u);
+          };
+          // phase parity of head e's barrier: one completion per head (one set), per two heads (two)
+          auto par_of = [&](int e) -> uint32_t { return static_cast<uint32_t>(dbuf ? (e >> 1) & 1 : e & 1); };
+          // thread 0: the bulk copy of head e's K (kind 0) or V (kind 1) rows (nothing once a wait
+          // gave up, so that the teardown knows every copy in flight)
+          auto fetch = [&](int e, int kind) {
+            if (*s_abort) return;
+            const uint32_t bar = bar_of(e, kind);
+            mbar_arrive_expect_tx(bar, fetch_bytes);
+            bulk_g2s(buf_of(e, kind), kvs + (static_cast<size_t>(e) * 2 + kind) * (p.C * kRows) * DH, fetch_bytes,
+                     bar);
+            ++s_issued[6 + kind + ((dbuf && (e & 1)) ? 2 : 0)];
+          };
+          if (tid == 0) {
+            fetch(0, 0), fetch(0, 1);
+            if (dbuf) fetch(1, 0), fetch(1, 1);
+          }
           auto dot16 = [&](const float *q, const float4 *kk) -> float {
             float2 d2 = make_float2(0.0f, 0.0f);
 #pragma unroll
@@ -1589,35 +1652,9 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             return __fadd_rn(d2.x, d2.y);
           };
           for (int e = 0; e < kHeads; ++e) {
-            // row rho of the group: 128 bytes at rho * 128, 16-byte slot f at f ^ (rho & 7)
-            const uint32_t stg = sb + L::kOffAop + ((dbuf && (e & 1)) ? static_cast<uint32_t>(nrows) * 128u : 0u);
-            {
-              // gather: item it = (row rho, 16-byte slot f of the head's K|V), 10 items per thread at most
-              float4 v[5];
-#pragma unroll
-              for (int half = 0; half < 2; ++half) {
-#pragma unroll
-                for (int j = 0; j < 5; ++j) {
-                  const int it = tid + kEpiThreads * (5 * half + j);
-                  if (it < nrows * 8) {
-                    const int rho = it >> 3, f = it & 7;
-                    v[j] = ld_cluster_f32x4(s_kvcl[rho >> 7] + static_cast<uint32_t>(rho & 127) * L::kKvStride +
-                                            static_cast<uint32_t>(e) * L::kSlot + 16u * f);
-                  }
-                }
-#pragma unroll
-                for (int j = 0; j < 5; ++j) {
-                  const int it = tid + kEpiThreads * (5 * half + j);
-                  if (it < nrows * 8) {
-                    const int rho = it >> 3, f = it & 7;
-                    st_shared_f4(stg + static_cast<uint32_t>(rho) * 128u + static_cast<uint32_t>((f ^ (rho & 7)) << 4),
-                                 v[j].x, v[j].y, v[j].z, v[j].w);
-                  }
-                }
-              }
-            }
-            named_bar_sync(5, kEpiThreads);
-            if (e == kHeads - 1) kvf_signal();  // every read of the cluster's K/V of this block is done
+            // the barriers complete 8 (one set) or 4 (two sets) times a block: an even number
+            const uint32_t ph = par_of(e);
+            const uint32_t kbuf = buf_of(e, 0), vbuf = buf_of(e, 1);
             const int mk = (e < p.h_first) ? 0 : 1;
             const uint32_t info = row_cw ? __ldg(p.mask_info[mk] + t) : 0u;
             const int cnt = static_cast<int>(info & 2047u);
@@ -1633,6 +1670,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
 #pragma unroll
               for (int i = 0; i < DH; ++i) q[i] = __fadd_rn(__fmul_rn(qa[i], fq), bq[i]);
             }
+            wait_bar_warp(ctl, bar_of(e, 0), ph, false);  // this head's K rows have landed
             // pass 1: sigma of keys [b + 4 sl, b + 4 sl + 4) of every 16-key block b, and their maximum
             float mx = -INFINITY;
             for (int b = 0; b < nmax; b += 16) {
@@ -1646,10 +1684,11 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                   const int rho = rowbase + idx[i];  // a key past the row's count reads a valid row (offset 0)
-                  const uint32_t rb = stg + static_cast<uint32_t>(rho) * 128u;
+                  const uint32_t rb = kbuf + static_cast<uint32_t>(rho) * 64u;
                   float4 kk[DH / 4];
 #pragma unroll
-                  for (int f = 0; f < DH / 4; ++f) kk[f] = ld_shared_f4(rb + static_cast<uint32_t>((f ^ (rho & 7)) << 4));
+                  for (int f = 0; f < DH / 4; ++f)
+                    kk[f] = ld_shared_f4(rb + static_cast<uint32_t>((f ^ ((rho >> 1) & 3)) << 4));
                   sg[i] = __fmul_rn(dot16(q, kk), p.att_scale);
                   if (k0 + i < cnt) mx = fmaxf(mx, sg[i]);
                 }
@@ -1660,6 +1699,11 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             tc_fence_before();
             mx = row_max(mx);
             tc_fence_after();
+            if (!dbuf) {
+              // every thread is past its reads of the K buffer: fetch the next head's K into it
+              named_bar_sync(5, kEpiThreads);
+              if (tid == 0 && e + 1 < kHeads) fetch(e + 1, 0);
+            }
             // pass 2: p = 2^(sigma - m) of the same keys, written over their scores
             for (int b = 0; b < nmax; b += 16) {
               const int k0 = b + 4 * sl;
@@ -1676,9 +1720,9 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             tc_fence_before();
             named_bar_sync(qbar, 128);
             tc_fence_after();
+            wait_bar_warp(ctl, bar_of(e, 1), ph, false);  // this head's V rows have landed
             // l = sum p and num = sum p v over the row's keys in ascending order, features [4 sl, 4 sl + 4)
             float lsum = 0.0f, num[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-            const uint32_t vslot = static_cast<uint32_t>(DH / 4 + sl);
             for (int b = 0; b < nmax; b += 16) {
               float pb[16];
               tmem_ld<16>(tl + kSc + b, pb);
@@ -1689,8 +1733,8 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
               for (int kk = 0; kk < 16; ++kk) {
                 if (b + kk < cnt) {
                   const int rho = rowbase + idx_at(kk < 8 ? w0 : w1, kk & 7);
-                  const float4 vv = ld_shared_f4(stg + static_cast<uint32_t>(rho) * 128u +
-                                                 ((vslot ^ static_cast<uint32_t>(rho & 7)) << 4));
+                  const float4 vv = ld_shared_f4(vbuf + static_cast<uint32_t>(rho) * 64u +
+                                                 static_cast<uint32_t>((sl ^ ((rho >> 1) & 3)) << 4));
                   lsum = __fadd_rn(lsum, pb[kk]);
                   num[0] = __fmaf_rn(pb[kk], vv.x, num[0]);
                   num[1] = __fmaf_rn(pb[kk], vv.y, num[1]);
@@ -1705,17 +1749,23 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
 #pragma unroll
               for (int f = 0; f < 4; ++f) a4[f] = row_cw ? __fmul_rn(num[f], inv) : 0.0f;
               // A of (row, head e), features [4 sl, 4 sl + 4), over the head's Q (read by all 4 threads
-              // before the quadrant barrier above)
+              // before the barriers above)
               tmem_st4(tl + e * DH + 4 * sl, a4[0], a4[1], a4[2], a4[3]);
             }
             tmem_wait_st();
             tc_fence_before();
-            // the staging area is free for the next head (two buffers: the next head's gather barrier
-            // orders this head's reads before the gather after it; the last head's barrier orders
-            // the attention outputs in TMEM before Quant(A))
-            if (!dbuf || e == kHeads - 1) named_bar_sync(5, kEpiThreads);
+            // every thread is past its reads of this head's buffers: fetch the next head's V (one
+            // set) or the next-but-one head's K and V (two sets) into them (after the last head the
+            // attention outputs in TMEM are ordered before Quant(A))
+            named_bar_sync(5, kEpiThreads);
             tc_fence_after();
+            if (tid == 0) {
+              if (!dbuf && e + 1 < kHeads) fetch(e + 1, 1);
+              if (dbuf && e + 2 < kHeads) fetch(e + 2, 0), fetch(e + 2, 1);
+            }
           }
+          // every read of the cluster's K/V scratch of this block is done
+          kvf_signal();
           // O's weights into W0, W1 (free again), while the codes of A are made
           if (warp == 0) issuer.stage_o(p.wstream + static_cast<size_t>(l) * p.layer_bytes);
           // Quant(A) -> O operand: columns [sl XS, sl XS + XS) = heads 2 sl and 2 sl + 1, from TMEM
@@ -1935,6 +1985,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
     if (lane == 0) {
       wait_bar_drain(ctl, bar_fin, 0);
       issuer.drain();
+      if constexpr (STAGED)  // the staged attention's bulk copies of K and V rows (two buffer sets)
+        for (int i = 0; i < 4; ++i)
+          if (s_issued[6 + i] > 0)
+            wait_bar_drain(ctl, ((i & 1) ? bar_sv : bar_sk) + (i >= 2 ? 16u : 0u), (s_issued[6 + i] - 1u) & 1u);
     }
     __syncwarp();
   }
