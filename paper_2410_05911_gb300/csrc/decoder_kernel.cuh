@@ -790,9 +790,6 @@ template <int ATT>
 struct Issuer<128, ATT> {
   static constexpr int D = 128;
   using L = SmemLayout<D, ATT == 1>;
-  // staged attention (ATT == 2) gathers each head's keys and values into the operand tile and the
-  // weight stages, so O's weights (W0, W1) are fetched after attention (stage_o) instead of with QKV's
-  static constexpr bool kStaged = ATT == 2;
   using W = WeightSchedule<D>;
   static constexpr uint32_t kChunk = W::kStageBytes;
   static_assert(W::kCPL == 24 && W::kStages == 3 && kChunk == 16384, "d = 128 schedule");
@@ -874,14 +871,10 @@ struct Issuer<128, ATT> {
     arm(slot(P).id, W::chunk(P).bytes);
     copies<P, P + 1>(src);
   }
-  // QKV (region U) and O (W0, W1) of a block; staged attention: QKV only
+  // QKV (region U) and O (W0, W1) of a block
   __device__ __forceinline__ void stage_qkv_o(const uint8_t *src) const {
     arm(3, 6 * kChunk);
     copies<0, 6>(src);
-    if constexpr (!kStaged) stage_o(src);
-  }
-  // O's weights into W0, W1
-  __device__ __forceinline__ void stage_o(const uint8_t *src) const {
     copy1<6>(src);
     copy1<7>(src);
   }
@@ -1582,10 +1575,9 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           // ---------------- S5: HPSA (Sec. 4.2), per-row lists over per-head staged rows (d = 128).
           // Every CTA of the cluster has left the K and V rows of its token rows in the cluster's
           // scratch in global memory (L2).  Head by head, one bulk copy brings the K rows of the
-          // head for every row of the group into a K buffer and another the V rows into a V buffer
-          // (the operand tile and the weight stages, idle here: 40 KB each).  The next head's K is
-          // fetched while this head's exponentials and fold run, its V while its scores run.  The
-          // row's 4 threads share the head: each takes 4 keys of every 16-key block for the scores
+          // head for every row of the group into a K buffer and another the V rows into a V buffer;
+          // two sets of buffers (region U and the operand tile, idle here) let the next head's rows
+          // arrive while this head computes.  The row's 4 threads share the head: each takes 4 keys of every 16-key block for the scores
           // and their exponentials (the row's TMEM lane, columns from kSc), and then folds every
           // key, in ascending order, into 4 of the 16 features of num.  The arithmetic is the
           // canonical one, key for key and feature for feature.
@@ -1606,28 +1598,24 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           }
           cluster_arrive(bar_kvr);
           cluster_wait(bar_kvr, kvr_ph);
-          static_assert(L::kOffW == L::kOffAop + L::kAopBytes && L::kAopBytes + 3 * L::kStageBytes >= 2 * 40960,
-                        "the K and V buffers span the operand tile and the weight stages");
+          static_assert(L::kOffU == 0 && L::kOffAop == L::kRegionU &&
+                            L::kRegionU + L::kAopBytes >= 4u * kStagedMaxRows * 64u,
+                        "two sets of K and V buffers span region U and the operand tile");
           constexpr uint32_t kSc = 128;  // the dead K and V accumulator columns [128, 384)
           // row rho of the group: 64 bytes at rho * 64, 16-byte piece f at f ^ ((rho >> 1) & 3)
           const int nrows = p.G * Tp;  // <= 640 (checked at create)
           const int rowbase = g * Tp;
           const uint32_t fetch_bytes = static_cast<uint32_t>(nrows) * 64u;
-          // two sets of K and V buffers when they fit (LDPC(128,64): 4 x 12 KB): head e uses set
-          // e & 1 and the next-but-one head is fetched after head e, so each head needs one CTA
-          // barrier; one set otherwise (40 KB each), the next head fetched into each buffer as
-          // soon as its reads are over
-          const bool dbuf = 4u * fetch_bytes <= 81920u;
+          // two sets of K and V buffers in region U (its K and V went to the scratch: idle here) and
+          // the operand tile, [K0 | V0 | K1 | V1]: head e uses set e & 1 and the next-but-one head is
+          // fetched after head e, so each head needs one CTA barrier
           const float *kvs = p.kv_scratch + static_cast<size_t>(cluster_id) * kHeads * 2 * (p.C * kRows) * DH;
           auto buf_of = [&](int e, int kind) -> uint32_t {
-            return dbuf ? sb + L::kOffAop + (static_cast<uint32_t>(e & 1) * 2u + kind) * fetch_bytes
-                        : sb + L::kOffAop + static_cast<uint32_t>(kind) * 40960u;
+            return sb + L::kOffU + (static_cast<uint32_t>(e & 1) * 2u + kind) * fetch_bytes;
           };
-          auto bar_of = [&](int e, int kind) -> uint32_t {
-            return (kind ? bar_sv : bar_sk) + ((dbuf && (e & 1)) ? 16u : 0u);
-          };
-          // phase parity of head e's barrier: one completion per head (one set), per two heads (two)
-          auto par_of = [&](int e) -> uint32_t { return static_cast<uint32_t>(dbuf ? (e >> 1) & 1 : e & 1); };
+          auto bar_of = [&](int e, int kind) -> uint32_t { return (kind ? bar_sv : bar_sk) + ((e & 1) ? 16u : 0u); };
+          // phase parity of head e's barrier: one completion per two heads, 4 a block
+          auto par_of = [&](int e) -> uint32_t { return static_cast<uint32_t>((e >> 1) & 1); };
           // thread 0: the bulk copy of head e's K (kind 0) or V (kind 1) rows (nothing once a wait
           // gave up, so that the teardown knows every copy in flight)
           auto fetch = [&](int e, int kind) {
@@ -1636,12 +1624,9 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             mbar_arrive_expect_tx(bar, fetch_bytes);
             bulk_g2s(buf_of(e, kind), kvs + (static_cast<size_t>(e) * 2 + kind) * (p.C * kRows) * DH, fetch_bytes,
                      bar);
-            ++s_issued[6 + kind + ((dbuf && (e & 1)) ? 2 : 0)];
+            ++s_issued[6 + kind + ((e & 1) ? 2 : 0)];
           };
-          if (tid == 0) {
-            fetch(0, 0), fetch(0, 1);
-            if (dbuf) fetch(1, 0), fetch(1, 1);
-          }
+          if (tid == 0) fetch(0, 0), fetch(0, 1), fetch(1, 0), fetch(1, 1);
           auto dot16 = [&](const float *q, const float4 *kk) -> float {
             float2 d2 = make_float2(0.0f, 0.0f);
 #pragma unroll
@@ -1652,7 +1637,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             return __fadd_rn(d2.x, d2.y);
           };
           for (int e = 0; e < kHeads; ++e) {
-            // the barriers complete 8 (one set) or 4 (two sets) times a block: an even number
+            // each barrier completes 4 times a block: an even number
             const uint32_t ph = par_of(e);
             const uint32_t kbuf = buf_of(e, 0), vbuf = buf_of(e, 1);
             const int mk = (e < p.h_first) ? 0 : 1;
@@ -1699,11 +1684,6 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             tc_fence_before();
             mx = row_max(mx);
             tc_fence_after();
-            if (!dbuf) {
-              // every thread is past its reads of the K buffer: fetch the next head's K into it
-              named_bar_sync(5, kEpiThreads);
-              if (tid == 0 && e + 1 < kHeads) fetch(e + 1, 0);
-            }
             // pass 2: p = 2^(sigma - m) of the same keys, written over their scores
             for (int b = 0; b < nmax; b += 16) {
               const int k0 = b + 4 * sl;
@@ -1754,20 +1734,15 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             }
             tmem_wait_st();
             tc_fence_before();
-            // every thread is past its reads of this head's buffers: fetch the next head's V (one
-            // set) or the next-but-one head's K and V (two sets) into them (after the last head the
-            // attention outputs in TMEM are ordered before Quant(A))
+            // every thread is past its reads of this head's buffers: fetch the next-but-one head's K
+            // and V into them (after the last head the attention outputs in TMEM are ordered before
+            // Quant(A))
             named_bar_sync(5, kEpiThreads);
             tc_fence_after();
-            if (tid == 0) {
-              if (!dbuf && e + 1 < kHeads) fetch(e + 1, 1);
-              if (dbuf && e + 2 < kHeads) fetch(e + 2, 0), fetch(e + 2, 1);
-            }
+            if (tid == 0 && e + 2 < kHeads) fetch(e + 2, 0), fetch(e + 2, 1);
           }
           // every read of the cluster's K/V scratch of this block is done
           kvf_signal();
-          // O's weights into W0, W1 (free again), while the codes of A are made
-          if (warp == 0) issuer.stage_o(p.wstream + static_cast<size_t>(l) * p.layer_bytes);
           // Quant(A) -> O operand: columns [sl XS, sl XS + XS) = heads 2 sl and 2 sl + 1, from TMEM
           float av[XS];
           tmem_ld<XS>(tl + sl * XS, av);
