@@ -401,6 +401,21 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
       return AECCT_ERR_UNSUPPORTED;
     }
   }
+  // staged mode with the cluster size left open: the size with the most words resident on the
+  // device, words per group x clusters that fit at once (LDPC(128,64): three CTAs hold two words
+  // in 46 clusters, 92 words, against 76 with two CTAs per word).  The group's rows stay within
+  // the staged row limit.
+  if (att == 2 && d.cluster_ctas == 0 && d.alpha_mode == 0) {
+    int top = 0;
+    for (int C = cmin; C <= kMaxCluster; ++C) {
+      const int G = std::min(C * kRows / T, kStagedMaxRows / T);
+      if (G < 1 || ((G + C - 1) / C) * n > kOutBitsBytes || G * ((n + 31) / 32) > 128) continue;
+      int mc = 0;
+      e = prepare_variant(d.activation, d.linear_mode, D, att, C, plan_bound, &mc);
+      if (e != cudaSuccess) return cuda_fail(e, "kernel occupancy");
+      if (G * mc > top) top = G * mc, best_C = C, best_G = G;
+    }
+  }
   int max_clusters = 0;
   e = prepare_variant(d.activation, d.linear_mode, D, att, best_C, plan_bound, &max_clusters);
   if (e != cudaSuccess) return cuda_fail(e, "kernel occupancy");

@@ -77,8 +77,8 @@ LAYOUTS = {
     # next 32-row boundary), per-row lists over per-head staged rows (d = 128; one CTA or a cluster)
     "bch31_16": [(0, 1), (1, 1), (0, 2)],
     "polar64_32": [(0, 1), (1, 1), (0, 2)],
-    "bch63_36": [(0, 1), (1, 1), (0, 2), (2, 1), (0, 3), (2, 3)],
-    "ldpc128_64": [(0, 1), (0, 3), (3, 3)],
+    "bch63_36": [(0, 1), (1, 1), (0, 2), (2, 1), (0, 3), (1, 3), (2, 3)],
+    "ldpc128_64": [(0, 1), (0, 3), (2, 3), (4, 3)],
     "ldpc384_192": [(0, 1), (0, 3), (6, 3)],
 }
 
@@ -94,6 +94,26 @@ def test_result_independent_of_layout_and_attention_mode(key):
         q = dec.query()
         assert q["attention_mode"] == mode and (cc == 0 or q["cluster_ctas"] == cc)
         assert_same(gpu_decode(dec, ch.y), ref, f"{key} C={q['cluster_ctas']} mode={mode}")
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("key", ["bch63_36", "ldpc128_64", "ldpc384_192"])
+def test_staged_cluster_size_holds_the_most_words(key):
+    # staged attention with the cluster size left open takes the size with the most words
+    # resident on the device (words per group x clusters that fit at once)
+    model = I.workload_model(key)
+    dec = A.Decoder(model, attention_mode=3)
+    q = dec.query()
+    dec.close()
+    best = q["words_per_group"] * q["max_clusters"]
+    for c in range(1, 9):
+        try:
+            d2 = A.Decoder(model, cluster_ctas=c, attention_mode=3)
+        except A.AecctError:
+            continue  # no word fits, or the group passes the staged row limit
+        q2 = d2.query()
+        d2.close()
+        assert q2["words_per_group"] * q2["max_clusters"] <= best, (c, q2, q)
 
 
 @pytest.mark.gpu
