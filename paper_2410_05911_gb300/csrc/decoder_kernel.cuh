@@ -654,7 +654,8 @@ struct BlockCtx {
   uint32_t lpar;    // parity of the block's index in this CTA's sequence of blocks
   uint32_t kvf;     // cluster barrier: every CTA of the cluster has finished reading this CTA's K/V
   uint32_t kvf_ph;  // its phase parity for this block
-  bool cluster;     // more than one CTA per cluster
+  bool u_own;       // region U is this CTA's alone once its own attention is done (one-CTA cluster,
+                    // or staged attention, whose peers read the K/V scratch in global memory)
 };
 
 template <int D, int ATT>
@@ -941,11 +942,11 @@ struct Issuer<128, ATT> {
       wait(bar(1), parity<7>(lp));
       mmas<1, 7>();
       commit(bar_acc());
-      // FFN1 weights into region U: a one-CTA cluster has finished reading its K/V (every warp
-      // published the O operand); a larger cluster stages them at FFN1 instead, so that the O
-      // epilogue overlaps the peers' attention.  FFN2 chunk 18 into W2 (last read by the
-      // previous block's FFN2).
-      if (!bc.cluster) {
+      // FFN1 weights into region U: this CTA has finished reading it (every warp published the O
+      // operand) and no peer reads it (one-CTA cluster, staged attention); a cluster whose peers
+      // read this CTA's K/V stages them at FFN1 instead, so that the O epilogue overlaps the
+      // peers' attention.  FFN2 chunk 18 into W2 (last read by the previous block's FFN2).
+      if (bc.u_own) {
         arm(3, 8 * kChunk);
         copies<8, 16>(w_cur);
       }
@@ -955,7 +956,7 @@ struct Issuer<128, ATT> {
       copy1<16>(w_cur);  // W0, W1 were O's
       copy1<17>(w_cur);
     } else if constexpr (G == 2) {
-      if (bc.cluster) {  // every CTA of the cluster is done with this CTA's K/V
+      if (!bc.u_own) {  // every CTA of the cluster is done with this CTA's K/V
         wait(bc.kvf, bc.kvf_ph, true);
         arm(3, 8 * kChunk);
         copies<8, 16>(w_cur);
@@ -1166,7 +1167,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         const uint8_t *w_cur = p.wstream + static_cast<size_t>(blk) * p.layer_bytes;
         const uint8_t *w_next = last_blk ? p.wstream : w_cur + p.layer_bytes;
         const bool has_next = !last_blk || gi + p.n_clusters < p.n_groups;
-        const BlockCtx bc{(blk_base + static_cast<uint32_t>(blk)) & 1u, bar_kvf, kvf_ph, p.C > 1};
+        const BlockCtx bc{(blk_base + static_cast<uint32_t>(blk)) & 1u, bar_kvf, kvf_ph, p.C == 1 || STAGED};
         if (gemm == 0) issuer.template gemm<0>(w_cur, w_next, has_next, bc);
         if (gemm == 1) issuer.template gemm<1>(w_cur, w_next, has_next, bc);
         if (gemm == 2) issuer.template gemm<2>(w_cur, w_next, has_next, bc);
@@ -1185,10 +1186,11 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
       }
       __syncwarp();
     };
-    // after a CTA-wide barrier: this CTA no longer reads any CTA's K/V of this block
-    auto kvf_signal = [&]() {
+    // after a CTA-wide barrier: this CTA no longer reads any CTA's K/V of this block (signalled by
+    // thread `who`)
+    auto kvf_signal = [&](int who) {
       if (p.C == 1) return;
-      if (tid == 0) {
+      if (tid == who) {
         fence_acq_rel_cluster();
         for (int c = 0; c < p.C; ++c) mbar_arrive_cluster(mapa_cluster(bar_kvf, c));
       }
@@ -1741,8 +1743,6 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             tc_fence_after();
             if (tid == 0 && e + 2 < kHeads) fetch(e + 2, 0), fetch(e + 2, 1);
           }
-          // every read of the cluster's K/V scratch of this block is done
-          kvf_signal();
           // Quant(A) -> O operand: columns [sl XS, sl XS + XS) = heads 2 sl and 2 sl + 1, from TMEM
           float av[XS];
           tmem_ld<XS>(tl + sl * XS, av);
@@ -1764,10 +1764,13 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           }
         }
         // this CTA no longer reads any K/V of this block (arrived before the O GEMM is issued: the
-        // d = 128 schedule stages FFN1's weights over the K/V region once every CTA has arrived);
-        // the staged mode has arrived after its last gather
+        // d = 128 schedule stages FFN1's weights over the K/V region once every CTA has arrived)
         if constexpr (ATT == 0) cluster_arrive(bar_kvf);
         signal_op(1, l, gi);
+        // staged mode: every fetch from the cluster's K/V scratch of this block has landed (the
+        // last head's barrier); a thread of warp 1, which next waits for the O accumulators, tells
+        // the cluster, off warp 0's path to the O GEMM
+        if constexpr (STAGED) kvf_signal(32);
 
         // ---------------- S6: O projection + residual + LayerNorm (Sec. 5, Post-LN)
         {
