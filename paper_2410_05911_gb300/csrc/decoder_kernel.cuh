@@ -812,6 +812,8 @@ struct Issuer<128, ATT> {
   }
   __device__ __forceinline__ uint32_t bar_op() const { return sb + L::kOffBar + 48; }
   __device__ __forceinline__ uint32_t bar_acc() const { return sb + L::kOffBar + 56; }
+  // FFN1's N tiles 0 and 1 (hidden units [0, 256)) are complete: once per block
+  __device__ __forceinline__ uint32_t bar_acc_lo() const { return sb + L::kOffBar + 160; }
   // the accumulators are complete: let the CTA's other warps (waiting in wait_acc) go
   __device__ __forceinline__ static void release_acc() { named_bar_arrive(5, kEpiThreads); }
 
@@ -964,14 +966,17 @@ struct Issuer<128, ATT> {
       wait(bar(3), 1);  // FFN1 weights in region U
       mmas_pair<2, 8>();
       mmas_pair<2, 10>();
+      // the epilogue of hidden units [0, 256) (column slices 0 and 1) starts while the MMAs of
+      // [256, 512) run; each warp waits on the barrier of its own half (no release by this warp)
+      commit(bar_acc_lo());
       mmas_pair<2, 12>();
       mmas_pair<2, 14>();
       commit(bar_acc());
-      wait(bar_acc(), 0);
-      release_acc();
-      copy1<19>(w_cur);  // the operand tile is free: FFN1's MMAs are done
-      copy1<20>(w_cur);
     } else {
+      // the operand tile is free: every warp saw FFN1's accumulators complete before it
+      // published FFN2's operand
+      copy1<19>(w_cur);
+      copy1<20>(w_cur);
       wait(bar(0), parity<16>(lp));
       mmas<3, 16>();
       commit(bar_empty(0));
@@ -1066,8 +1071,9 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
     mbar_init(bar_zr, p.C);
     mbar_init(bar_zf, p.C);
     mbar_init(bar_fin, 1);
-    if constexpr (D == 128)  // region U and the two operand-tile halves (d = 128 weight schedule)
-      for (int i = 0; i < 7; ++i) mbar_init(bar_fin + 8 + 8 * i, 1);
+    if constexpr (D == 128)  // region U, the two operand-tile halves (d = 128 weight schedule), the
+                             // staged K/V buffers, FFN1's first half
+      for (int i = 0; i < 8; ++i) mbar_init(bar_fin + 8 + 8 * i, 1);
     *s_abort = 0;
     for (int i = 0; i < 10; ++i) s_issued[i] = 0;
     // base of the K/V area of every CTA of the cluster as a shared::cluster address, and generic
@@ -1798,7 +1804,16 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         // ---------------- S7: FFN1 + ReLU (Sec. 4 item 4) or GELU, Quant(u) -> FFN2 operand
         {
           const float f1 = dq_factor(sw + 4);
-          wait_acc();
+          if constexpr (D == 128) {
+            // column slices 0 and 1 (hidden units [0, 256)) wait for the first half of FFN1's
+            // MMAs, slices 2 and 3 for all of them (the block's third accumulator phase)
+            static_assert(16 * S + 48 + 64 == 160, "bar_fin + 64 is the issuer's bar_acc_lo");
+            if (sl < 2) wait_bar_warp(ctl, bar_fin + 64, (blk_base + static_cast<uint32_t>(l)) & 1u, false);
+            else wait_bar_warp(ctl, bar_acc, 0, false);
+            tc_fence_after();
+          } else {
+            wait_acc();
+          }
           // ACT 0 = ReLU, 1 = GELU.  u = act(acc f1 + b1) in 32-column chunks of this thread's D
           // hidden columns.  AAP: u is stored over its own accumulators in TMEM (this thread's
           // lane and columns) between the row maximum and the codes, which leaves the registers
