@@ -1805,10 +1805,14 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         {
           const float f1 = dq_factor(sw + 4);
           if constexpr (D == 128) {
-            // column slices 0 and 1 (hidden units [0, 256)) wait for the first half of FFN1's
-            // MMAs, slices 2 and 3 for all of them (the block's third accumulator phase)
+            // AAP: column slices 0 and 1 (hidden units [0, 256)) wait for the first half of FFN1's
+            // MMAs, slices 2 and 3 for all of them (the block's third accumulator phase).  Their
+            // first pass only writes TMEM columns of the finished half; the codes go to region U,
+            // where the second half's weights are, after the row maximum, which needs every
+            // slice.  Full-precision linears write u to region U in their only pass: every slice
+            // waits for all of FFN1.
             static_assert(16 * S + 48 + 64 == 160, "bar_fin + 64 is the issuer's bar_acc_lo");
-            if (sl < 2) wait_bar_warp(ctl, bar_fin + 64, (blk_base + static_cast<uint32_t>(l)) & 1u, false);
+            if (LIN == 0 && sl < 2) wait_bar_warp(ctl, bar_fin + 64, (blk_base + static_cast<uint32_t>(l)) & 1u, false);
             else wait_bar_warp(ctl, bar_acc, 0, false);
             tc_fence_after();
           } else {
