@@ -783,8 +783,9 @@ struct Issuer {
 //   QKV  -> region U (free between the previous FFN2 and this block's K/V), one barrier bar_U;
 //   O    -> stages W0, W1;
 //   FFN1 -> region U again (free once every CTA of the cluster has finished attention);
-//   FFN2 -> W0, W1, W2, then the operand tile (free once FFN1's MMAs are done) as A0, A1, then
-//           W0, W1, W2 again once chunks 16-18 are consumed.
+//   FFN2 -> W0, W1, W2, then the operand tile as A0, A1 (copied as soon as FFN1's MMAs, its last
+//           readers, are complete: during FFN1's epilogue), then W0, W1, W2 again once chunks
+//           16-18 are consumed.
 // A barrier armed u times per block (u odd for W0, W1, A0, A1) completes phase parity
 // (lpar if u is odd) ^ (index of the use within the block), with lpar the block's parity.
 template <int ATT>
@@ -882,6 +883,13 @@ struct Issuer<128, ATT> {
     copy1<7>(src);
   }
   __device__ __forceinline__ void prologue(const uint8_t *w0) const { stage_qkv_o(w0); }
+  // FFN2's chunks 19 and 20 into the operand tile.  Called by warp 0 during FFN1's epilogue once
+  // FFN1's MMAs, the tile's last readers in this block, are known to be complete (warp 0 waited
+  // for them, or synchronised with warps that did).
+  __device__ __forceinline__ void stage_ffn2_aop(const uint8_t *w_cur) const {
+    copy1<19>(w_cur);
+    copy1<20>(w_cur);
+  }
 
   // the MMAs of chunk P (its weights have landed)
   template <int G, int P>
@@ -973,10 +981,7 @@ struct Issuer<128, ATT> {
       mmas_pair<2, 14>();
       commit(bar_acc());
     } else {
-      // the operand tile is free: every warp saw FFN1's accumulators complete before it
-      // published FFN2's operand
-      copy1<19>(w_cur);
-      copy1<20>(w_cur);
+      // chunks 19 and 20 were copied into the operand tile during FFN1's epilogue
       wait(bar(0), parity<16>(lp));
       mmas<3, 16>();
       commit(bar_empty(0));
@@ -1815,6 +1820,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             if (LIN == 0 && sl < 2) wait_bar_warp(ctl, bar_fin + 64, (blk_base + static_cast<uint32_t>(l)) & 1u, false);
             else wait_bar_warp(ctl, bar_acc, 0, false);
             tc_fence_after();
+            // full-precision linears: warp 0 itself waited for all of FFN1, so the operand tile
+            // takes FFN2's chunks 19 and 20 now
+            if constexpr (LIN == 1)
+              if (warp == 0) issuer.stage_ffn2_aop(p.wstream + static_cast<size_t>(l) * p.layer_bytes);
           } else {
             wait_acc();
           }
@@ -1856,6 +1865,11 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             }
             tmem_wait_st();
             float a = word_alpha(row_max(umax));
+            // FFN1's MMAs are complete (the row maximum synchronised warp 0 with the warps of
+            // column slices 2 and 3, which waited for all of them): the operand tile takes FFN2's
+            // chunks 19 and 20
+            if constexpr (D == 128)
+              if (warp == 0) issuer.stage_ffn2_aop(p.wstream + static_cast<size_t>(l) * p.layer_bytes);
             a = (a > p.alpha_floor) ? a : p.alpha_floor;
             alpha_in = a;
             const float rr = __fdiv_rn(127.0f, a);
