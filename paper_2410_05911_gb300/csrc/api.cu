@@ -195,6 +195,79 @@ int schedule_chunks(int D, ChunkDesc *out) {
   return D == 32 ? schedule_chunks_t<32>(out) : D == 64 ? schedule_chunks_t<64>(out) : schedule_chunks_t<128>(out);
 }
 
+// ---- warp-task attention plan: which warp runs which task
+// A task (one head for one query group) costs the length of its union key list + 4 (its fixed
+// part).  Warps w with the same w % 4 issue from one scheduler and share its issue slots.  Measured
+// on the GPU: a warp alone issues at about 0.36 of a scheduler's rate (its own dependency chains
+// limit it) and about three warps saturate a scheduler, so four warps with unequal loads leave a
+// tail where one warp runs alone (Polar(64,32): its tasks on three warps per scheduler decode 2.2%
+// faster than on four; BCH(63,36)'s on two warps per lane quadrant instead of four make the
+// attention 1.38x slower).  A scheduler's time is modelled in phases: while k of its warps have
+// work left, each advances at min(1, k s) / k.  The plan minimises the largest modelled time.
+constexpr double kWarpIssueShare = 0.36;
+
+double scheduler_time(std::vector<long> loads) {
+  loads.erase(std::remove(loads.begin(), loads.end(), 0L), loads.end());
+  std::sort(loads.begin(), loads.end());
+  double t = 0.0;
+  long done = 0;
+  const int n = static_cast<int>(loads.size());
+  for (int i = 0; i < n; ++i) {
+    const int k = n - i;  // warps with work left
+    const double per_warp = std::min(1.0, k * kWarpIssueShare) / k;
+    t += static_cast<double>(loads[i] - done) / per_warp;
+    done = loads[i];
+  }
+  return t;
+}
+
+// The tasks of one scheduler (costs in descending order) onto its four warps, minimising
+// scheduler_time: every assignment for up to 10 tasks (a task opens at most the first empty warp,
+// which skips permutations of equivalent warps), else the best of longest-first onto 1..4 warps.
+// out[i] is the warp slot (0..3) of task i; false if no assignment keeps each warp within `cap`.
+bool assign_scheduler(const std::vector<int> &cost, int cap, std::vector<int> &out) {
+  const int m = static_cast<int>(cost.size());
+  out.assign(m, 0);
+  if (m == 0) return true;
+  double best = 1e300;
+  std::vector<int> cur(m, 0);
+  if (m <= 10) {
+    long load[4] = {0, 0, 0, 0};
+    int cnt[4] = {0, 0, 0, 0};
+    auto rec = [&](auto &&self, int i, int used) -> void {
+      if (i == m) {
+        const double t = scheduler_time({load[0], load[1], load[2], load[3]});
+        if (t < best) best = t, out = cur;
+        return;
+      }
+      for (int w = 0; w < std::min(used + 1, 4); ++w) {
+        if (cnt[w] >= cap) continue;
+        load[w] += cost[i], ++cnt[w], cur[i] = w;
+        self(self, i + 1, std::max(used, w + 1));
+        load[w] -= cost[i], --cnt[w];
+      }
+    };
+    rec(rec, 0, 0);
+  } else {
+    for (int k = 1; k <= 4; ++k) {
+      std::vector<long> load(k, 0);
+      std::vector<int> cnt(k, 0);
+      bool ok = true;
+      for (int i = 0; i < m && ok; ++i) {
+        int b = -1;
+        for (int w = 0; w < k; ++w)
+          if (cnt[w] < cap && (b < 0 || load[w] < load[b])) b = w;
+        if (b < 0) ok = false;
+        else load[b] += cost[i], ++cnt[b], cur[i] = b;
+      }
+      if (!ok) continue;
+      const double t = scheduler_time(load);
+      if (t < best) best = t, out = cur;
+    }
+  }
+  return best < 1e300;
+}
+
 // the compiled kernel for (d, attention path ATT, activation ACT, linear mode LIN)
 template <int ACT, int LIN>
 cudaError_t prepare_any(int D, int att, int C, uint32_t pb, int *max_clusters) {
@@ -536,29 +609,43 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
         }
       }
     }
-    // tasks (group, head), longest first, each to the least-loaded warp (d = 128: to a warp of the
-    // group's TMEM lane quadrant, where its rows' Q and A live)
+    // tasks (group, head), longest first.  d = 128: each on a warp of its group's TMEM lane quadrant,
+    // where its rows' Q and A live (warps w with w % 4 = quadrant: one scheduler); d <= 64: the
+    // schedulers by longest first onto the least-loaded one.  Then the warps of each scheduler by
+    // assign_scheduler.
     std::vector<std::pair<int, int>> tl;  // (cost, task)
     for (int gi = 0; gi < ng; ++gi)
       for (int e = 0; e < kHeads; ++e) tl.push_back({ucount[gi * 2 + (e < d.h_first ? 0 : 1)] + 4, gi * 8 + e});
     std::stable_sort(tl.begin(), tl.end(), [](const std::pair<int, int> &x, const std::pair<int, int> &y) {
       return x.first > y.first;
     });
-    ptask.assign((size_t)kEpiWarps * kMaxTasks, 0xFFFFu);
-    std::vector<long> load(kEpiWarps, 0);
-    std::vector<int> cnt(kEpiWarps, 0);
+    std::vector<std::pair<int, int>> per_sched[4];
+    long sched_load[4] = {0, 0, 0, 0};
     for (const auto &tk : tl) {
-      int best = -1;
-      const int quad = (grps[tk.second / 8].row0 / 32) & 3;
-      for (int w = 0; w < kEpiWarps; ++w)
-        if (cnt[w] < kMaxTasks && (D != 128 || (w & 3) == quad) && (best < 0 || load[w] < load[best])) best = w;
-      if (best < 0) {
+      int q = 0;
+      if (D == 128) {
+        q = (grps[tk.second / 8].row0 / 32) & 3;
+      } else {
+        for (int c = 1; c < 4; ++c)
+          if (sched_load[c] < sched_load[q]) q = c;
+      }
+      per_sched[q].push_back(tk);
+      sched_load[q] += tk.first;
+    }
+    ptask.assign((size_t)kEpiWarps * kMaxTasks, 0xFFFFu);
+    for (int q = 0; q < 4; ++q) {
+      std::vector<int> cost, slot;
+      for (const auto &tk : per_sched[q]) cost.push_back(tk.first);
+      if (!assign_scheduler(cost, kMaxTasks, slot)) {
         free_handle(h);
         g_last_error = "attention plan: too many tasks for a warp";
         return AECCT_ERR_UNSUPPORTED;
       }
-      ptask[(size_t)best * kMaxTasks + cnt[best]++] = static_cast<uint16_t>(tk.second);
-      load[best] += tk.first;
+      int cnt[4] = {0, 0, 0, 0};
+      for (size_t i = 0; i < per_sched[q].size(); ++i) {
+        const int w = q + 4 * slot[i];
+        ptask[(size_t)w * kMaxTasks + cnt[slot[i]]++] = static_cast<uint16_t>(per_sched[q][i].second);
+      }
     }
   }
 
