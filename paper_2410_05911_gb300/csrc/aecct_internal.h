@@ -15,6 +15,7 @@ constexpr int kThreads = kEpiThreads;  // warp 0 also streams weights and issues
 constexpr int kMaxCluster = 8;
 constexpr int kOutBitsBytes = 4096;      // decoded bits of the codewords one CTA finishes
 constexpr int kMaxTasks = 16;            // attention tasks per warp (task mode)
+constexpr int kQSlots = 8;               // d = 128 tasks run off their quadrant (2 KB Q/A slots in W2)
 constexpr int kMaxGroups = 32;           // 32-row query groups per CTA (task mode)
 constexpr int kTaskCache = 64;           // attention scores per task kept in TMEM (task mode)
 constexpr int kRowCache = 64;            // attention scores per (row, head) kept in TMEM (row mode)
@@ -158,9 +159,12 @@ struct DecodeParams {
   //   uinfo [groups][2 rings] uint32: (start << 8) | count of the union list
   //   ulist union lists: 16 row offsets (one byte each) per 16-byte entry
   //   mask  [groups][2][32 lanes] uint4: 128 membership bits over the union list
+  //   qslot (d = 128) uint8 [4] group of each TMEM lane quadrant (0xFF: none), then
+  //         [groups][8 heads] the Q/A slot of the task (group, head): 0xFF when it runs on a warp of
+  //         its group's quadrant (Q and A in TMEM), else a 2 KB slot of weight stage W2
   const uint4 *plan_blob;
   uint32_t plan_bytes;  // a multiple of 16; 0 without warp tasks
-  uint32_t off_task, off_grp, off_uinfo, off_ulist, off_mask;
+  uint32_t off_task, off_grp, off_uinfo, off_ulist, off_mask, off_qslot;
 
   float ln_eps, alpha_floor, att_scale;
   int alpha_mode;  // 0 = absmax alpha per token row, 1 = per quantised matrix of a word (C == 1)

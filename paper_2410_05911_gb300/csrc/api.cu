@@ -52,7 +52,7 @@ struct aecct_handle {
   uint16_t *perm = nullptr, *pos = nullptr;
   float *kv_scratch = nullptr;  // staged attention: K and V rows per cluster
   uint8_t *plan_blob = nullptr;  // the attention plan (task mode), copied into shared memory by the kernel
-  uint32_t plan_bytes = 0, off_task = 0, off_grp = 0, off_uinfo = 0, off_ulist = 0, off_mask = 0;
+  uint32_t plan_bytes = 0, off_task = 0, off_grp = 0, off_uinfo = 0, off_ulist = 0, off_mask = 0, off_qslot = 0;
   int *d_err = nullptr;
   int *h_err = nullptr;  // pinned
   cudaEvent_t ev = nullptr;
@@ -222,16 +222,17 @@ double scheduler_time(std::vector<long> loads) {
 }
 
 // The tasks of one scheduler (costs in descending order) onto its four warps, minimising
-// scheduler_time: every assignment for up to 10 tasks (a task opens at most the first empty warp,
+// scheduler_time: every assignment for up to 9 tasks (a task opens at most the first empty warp,
 // which skips permutations of equivalent warps), else the best of longest-first onto 1..4 warps.
 // out[i] is the warp slot (0..3) of task i; false if no assignment keeps each warp within `cap`.
-bool assign_scheduler(const std::vector<int> &cost, int cap, std::vector<int> &out) {
+bool assign_scheduler(const std::vector<int> &cost, int cap, std::vector<int> &out, double *time = nullptr) {
   const int m = static_cast<int>(cost.size());
   out.assign(m, 0);
+  if (time) *time = 0.0;
   if (m == 0) return true;
   double best = 1e300;
   std::vector<int> cur(m, 0);
-  if (m <= 10) {
+  if (m <= 9) {
     long load[4] = {0, 0, 0, 0};
     int cnt[4] = {0, 0, 0, 0};
     auto rec = [&](auto &&self, int i, int used) -> void {
@@ -265,6 +266,7 @@ bool assign_scheduler(const std::vector<int> &cost, int cap, std::vector<int> &o
       if (t < best) best = t, out = cur;
     }
   }
+  if (time) *time = best;
   return best < 1e300;
 }
 
@@ -466,7 +468,8 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
                                   : static_cast<uint32_t>(best_G * ((T + 31) / 32));
     auto r16 = [](uint32_t v) { return (v + 15u) & ~15u; };
     plan_bound = r16(2u * kEpiWarps * kMaxTasks) + 16u * ngb +
-                 r16(8u * ngb) + 2u * ngb * r16(static_cast<uint32_t>(T)) + 16u * 2u * 32u * ngb;
+                 r16(8u * ngb) + 2u * ngb * r16(static_cast<uint32_t>(T)) + 16u * 2u * 32u * ngb +
+                 r16(4u + 8u * ngb);
     const uint32_t fixed = D == 32 ? SmemLayout<32, true>::kTotal
                            : D == 64 ? SmemLayout<64, true>::kTotal : SmemLayout<128, true>::kTotal;
     if (fixed + plan_bound > kMaxDynSmem) {
@@ -562,6 +565,7 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
   // ---- task-mode attention plan (every CTA holds the same layout: G codewords of T rows)
   std::vector<uint16_t> ptask;
   std::vector<uint32_t> pgrp, puinfo, pmask;
+  std::vector<uint8_t> pqslot;
   std::vector<uint8_t> pulist;
   if (tasks) {
     const int G = best_G;
@@ -631,6 +635,63 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
       }
       per_sched[q].push_back(tk);
       sched_load[q] += tk.first;
+    }
+    // d = 128: a task may also run on a warp of a scheduler whose lane quadrant holds no token row,
+    // its Q and A then in a 2 KB slot of weight stage W2 (idle from the previous block's FFN2 to this
+    // block's O GEMM) instead of its rows' TMEM lanes.  Every loaded scheduler hands over the subset
+    // of its tasks (at most kQSlots in all) whose cost comes closest to its excess over the mean load
+    // without passing it; each goes to the free scheduler with the least load.  BCH(63,36): the fourth
+    // quadrant holds no token row, and each of the other three hands it a 67 and a 31 (all at 294).
+    std::vector<uint8_t> slot_of((size_t)ng * 8, 0xFFu);
+    if (D == 128) {
+      auto by_cost = [](const std::pair<int, int> &x, const std::pair<int, int> &y) { return x.first > y.first; };
+      std::vector<int> free_q;
+      long total = 0;
+      for (int q = 0; q < 4; ++q) {
+        total += sched_load[q];
+        if (per_sched[q].empty()) free_q.push_back(q);
+      }
+      const long mean = total / 4;
+      int nmoved = 0;
+      for (int pass = 0; pass < 4 && !free_q.empty(); ++pass) {
+        int q = -1;  // the most loaded scheduler not handled yet
+        for (int c = 0; c < 4; ++c)
+          if (!per_sched[c].empty() && std::find(free_q.begin(), free_q.end(), c) == free_q.end() &&
+              sched_load[c] > mean && (q < 0 || sched_load[c] > sched_load[q]))
+            q = c;
+        if (q < 0) break;
+        const long excess = sched_load[q] - mean;
+        const int mt = static_cast<int>(std::min<size_t>(per_sched[q].size(), 12));
+        uint32_t best_set = 0;
+        long best_sum = 0;
+        for (uint32_t set = 1; set < (1u << mt); ++set) {
+          const int k = __builtin_popcount(set);
+          if (nmoved + k > kQSlots) continue;
+          long sum = 0;
+          for (int t = 0; t < mt; ++t)
+            if (set >> t & 1u) sum += per_sched[q][t].first;
+          if (sum <= excess && (sum > best_sum || (sum == best_sum && k < __builtin_popcount(best_set))))
+            best_sum = sum, best_set = set;
+        }
+        for (int t = mt - 1; t >= 0; --t) {
+          if (!(best_set >> t & 1u)) continue;
+          int fq = free_q[0];
+          for (int c : free_q)
+            if (sched_load[c] < sched_load[fq]) fq = c;
+          const std::pair<int, int> tk = per_sched[q][t];
+          per_sched[q].erase(per_sched[q].begin() + t);
+          sched_load[q] -= tk.first;
+          per_sched[fq].push_back(tk);
+          sched_load[fq] += tk.first;
+          slot_of[tk.second] = static_cast<uint8_t>(nmoved++);
+        }
+        sched_load[q] = std::min(sched_load[q], mean);  // handled: not picked again
+      }
+      for (int q = 0; q < 4; ++q) std::stable_sort(per_sched[q].begin(), per_sched[q].end(), by_cost);
+      // the group of each lane quadrant (every group of a d = 128 word starts on one), then the slots
+      pqslot.assign(4 + (size_t)ng * 8, 0xFFu);
+      for (int gi = 0; gi < ng; ++gi) pqslot[(grps[gi].row0 / 32) & 3] = static_cast<uint8_t>(gi);
+      std::copy(slot_of.begin(), slot_of.end(), pqslot.begin() + 4);
     }
     ptask.assign((size_t)kEpiWarps * kMaxTasks, 0xFFFFu);
     for (int q = 0; q < 4; ++q) {
@@ -727,6 +788,7 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
     h->off_uinfo = put(puinfo.data(), puinfo.size() * 4);
     h->off_ulist = put(pulist.data(), pulist.size());
     h->off_mask = put(pmask.data(), pmask.size() * 4);
+    h->off_qslot = put(pqslot.data(), pqslot.size());
     h->plan_bytes = static_cast<uint32_t>(blob.size());
     if (h->plan_bytes > plan_bound) {
       free_handle(h);
@@ -798,7 +860,7 @@ static DecodeParams decode_params(const aecct_handle *h, int64_t B, const float 
   p.perm = h->perm, p.pos = h->pos;
   p.plan_blob = reinterpret_cast<const uint4 *>(h->plan_blob), p.plan_bytes = h->plan_bytes;
   p.off_task = h->off_task, p.off_grp = h->off_grp;
-  p.off_uinfo = h->off_uinfo, p.off_ulist = h->off_ulist, p.off_mask = h->off_mask;
+  p.off_uinfo = h->off_uinfo, p.off_ulist = h->off_ulist, p.off_mask = h->off_mask, p.off_qslot = h->off_qslot;
   p.mask_info[0] = h->mask_info[0], p.mask_info[1] = h->mask_info[1];
   p.mask_list[0] = reinterpret_cast<const uint4 *>(h->mask_list[0]);
   p.mask_list[1] = reinterpret_cast<const uint4 *>(h->mask_list[1]);

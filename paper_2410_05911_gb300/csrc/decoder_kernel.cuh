@@ -1123,6 +1123,16 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
     uint32_t *bitw = reinterpret_cast<uint32_t *>(smem + L::kOffBitWords);  // [G][hwords] bitmasks
     const int W = p.hwords;
     const uint32_t qbar = 1 + qd;  // named barrier of the 4 warps sharing a lane quadrant
+    // d = 128 warp tasks run off their rows' quadrant: the Q/A slots (2 KB: 32 rows of 16 floats,
+    // 16-byte piece f of row i at f ^ ((i >> 1) & 3)) in weight stage W2, idle from the previous
+    // block's FFN2 to this block's O GEMM; the plan's table gives each quadrant's group and each
+    // (group, head)'s slot (0xFF: none)
+    const uint8_t *qtab = splan + p.off_qslot;
+    const uint32_t qslot_base = sb + L::kOffW + 2u * WeightSchedule<D>::kStageBytes;
+    static_assert(D != 128 || kQSlots * 2048u <= WeightSchedule<D>::kStageBytes, "the Q/A slots fit W2");
+    auto qslot_piece = [&](uint32_t slot, int i, int f) -> uint32_t {
+      return qslot_base + slot * 2048u + static_cast<uint32_t>(i) * 64u + static_cast<uint32_t>((f ^ ((i >> 1) & 3)) << 4);
+    };
     const int T = p.T, Tp = p.Tp, n = p.n, m = p.m, de = D - p.d_spe;
     const int W4 = 4 * D;
     const float inv_d = 1.0f / static_cast<float>(D);
@@ -1406,6 +1416,21 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             dequant<DH>(qa, fq, bq, qa);
 #pragma unroll
             for (int i = 0; i < DH; i += 4) st_shared_f4(qdst + 4 * i, qa[i], qa[i + 1], qa[i + 2], qa[i + 3]);
+          } else if constexpr (TASKS) {
+            // this row's Q of head e into the slot of a task (group, e) that runs off this quadrant
+            const uint32_t qg = qtab[qd];
+            const uint32_t qs = qg != 0xFFu ? qtab[4 + qg * 8 + e] : 0xFFu;
+            if (qs != 0xFFu) {
+              float qa[DH], bq[DH];
+              ldg_vec<DH>(lp + LP::bqkv(D) + e * DH, bq);
+              tmem_ld<DH>(tl + e * DH, qa);
+              tmem_wait_ld();
+              if (cap) capture_acc(l, 0, qa, e * DH, DH);
+              dequant<DH>(qa, fq, bq, qa);
+#pragma unroll
+              for (int f = 0; f < DH / 4; ++f)
+                st_shared_f4(qslot_piece(qs, lane, f), qa[4 * f], qa[4 * f + 1], qa[4 * f + 2], qa[4 * f + 3]);
+            }
           }
         }
         if constexpr (TASKS) {
@@ -1434,12 +1459,20 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
                                  : make_uint4(~0u, ~0u, ~0u, ~0u);
             const uint32_t ui = reinterpret_cast<const uint32_t *>(splan + p.off_uinfo)[grp * 2 + ring];
             float q[DH], a[DH];
+            // d = 128: a task off its rows' quadrant has Q and A in a W2 slot (row = lane)
+            const uint32_t qs = L::kQInSmem ? 0xFFu : qtab[4 + grp * 8 + e];
             if constexpr (L::kQInSmem) {
               const float4 *qp = reinterpret_cast<const float4 *>(smem + L::kOffU + row * L::kKvStride + e * L::kSlot);
 #pragma unroll
               for (int i = 0; i < DH / 4; ++i) {
                 const float4 v = qp[i];
                 q[4 * i] = v.x, q[4 * i + 1] = v.y, q[4 * i + 2] = v.z, q[4 * i + 3] = v.w;
+              }
+            } else if (qs != 0xFFu) {
+#pragma unroll
+              for (int f = 0; f < DH / 4; ++f) {
+                const float4 v = ld_shared_f4(qslot_piece(qs, lane, f));
+                q[4 * f] = v.x, q[4 * f + 1] = v.y, q[4 * f + 2] = v.z, q[4 * f + 3] = v.w;
               }
             } else {
               float qa[DH], bq[DH];
@@ -1460,6 +1493,10 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
 #pragma unroll
                 for (int i = 0; i < DH / 4; ++i) ap[i] = make_float4(a[4 * i], a[4 * i + 1], a[4 * i + 2], a[4 * i + 3]);
               }
+            } else if (qs != 0xFFu) {
+              // A of (row, head e) over its Q in the slot (this task was its only reader)
+#pragma unroll
+              for (int f = 0; f < DH / 4; ++f) st_shared_f4(qslot_piece(qs, lane, f), a[4 * f], a[4 * f + 1], a[4 * f + 2], a[4 * f + 3]);
             } else {
               // every lane's own row: A of (row, head e) over the head's Q accumulators (a lane past
               // the group's rows writes a padding or empty row, which nothing reads)
@@ -1492,6 +1529,22 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             tc_fence_after();  // the tasks' TMEM stores of other warps are ordered by the barrier above
             tmem_ld<XS>(tl + sl * XS, av);
             tmem_wait_ld();
+            // heads whose task ran off this quadrant: A from their slots
+            const uint32_t qg = qtab[qd];
+            if (qg != 0xFFu) {
+#pragma unroll
+              for (int hh = 0; hh < 2; ++hh) {
+                const uint32_t qs = qtab[4 + qg * 8 + 2 * sl + hh];
+                if (qs != 0xFFu) {
+#pragma unroll
+                  for (int f = 0; f < DH / 4; ++f) {
+                    const float4 v = ld_shared_f4(qslot_piece(qs, lane, f));
+                    av[hh * DH + 4 * f] = v.x, av[hh * DH + 4 * f + 1] = v.y;
+                    av[hh * DH + 4 * f + 2] = v.z, av[hh * DH + 4 * f + 3] = v.w;
+                  }
+                }
+              }
+            }
           }
           if constexpr (LIN == 1) {
             store_bf16<XS>(aop, r, sl * XS, D, av);
