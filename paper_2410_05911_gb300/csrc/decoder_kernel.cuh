@@ -1061,6 +1061,8 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
   uint32_t *s_kvcl = reinterpret_cast<uint32_t *>(smem + L::kOffMisc + 8);   // [8] shared::cluster K/V bases per CTA
   uint64_t *s_zgen = reinterpret_cast<uint64_t *>(smem + L::kOffMisc + 72);   // [8] generic z bases per CTA
   uint32_t *s_issued = reinterpret_cast<uint32_t *>(smem + L::kOffMisc + 136);  // [10] weight copies / phases armed
+  // staged attention: warps past their reads of a buffer set in the current head round ([2] sets)
+  uint32_t *s_headdone = reinterpret_cast<uint32_t *>(smem + L::kOffMisc + 176);
   // staged attention: the barriers of the K and V buffers (buffer set 0; set 1 when two heads fit)
   const uint32_t bar_sk = bar_fin + 32, bar_sv = bar_fin + 40;  // + 16: set 1
 
@@ -1081,6 +1083,7 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
       for (int i = 0; i < 8; ++i) mbar_init(bar_fin + 8 + 8 * i, 1);
     *s_abort = 0;
     for (int i = 0; i < 10; ++i) s_issued[i] = 0;
+    s_headdone[0] = s_headdone[1] = 0;
     // base of the K/V area of every CTA of the cluster as a shared::cluster address, and generic
     // base of its z area: this CTA's own through its plain shared-memory window, the others
     // through the distributed shared window
@@ -1800,12 +1803,27 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
             }
             tmem_wait_st();
             tc_fence_before();
-            // every thread is past its reads of this head's buffers: fetch the next-but-one head's K
-            // and V into them (after the last head the attention outputs in TMEM are ordered before
-            // Quant(A))
-            named_bar_sync(5, kEpiThreads);
+            // the row's four threads (the quadrant's warps) are past this head's reads of the
+            // score columns, which the next head's pass 1 rewrites; after the last head every
+            // attention output in TMEM is ordered before Quant(A)
+            if (e == kHeads - 1) named_bar_sync(5, kEpiThreads);
+            else named_bar_sync(qbar, 128);
             tc_fence_after();
-            if (tid == 0 && e + 2 < kHeads) fetch(e + 2, 0), fetch(e + 2, 1);
+            if (e + 2 < kHeads) {
+              // this warp is past its reads of this head's buffers; the last warp of the CTA to get
+              // here fetches the next-but-one head's K and V into them (no quadrant waits for the
+              // slowest one between heads; a warp that runs ahead waits for those rows to land)
+              if (lane == 0) {
+                __threadfence_block();
+                if (atomicAdd(s_headdone + (e & 1), 1u) == static_cast<uint32_t>(kEpiWarps - 1)) {
+                  s_headdone[e & 1] = 0u;
+                  __threadfence_block();
+                  fence_proxy_async_smem();
+                  fetch(e + 2, 0), fetch(e + 2, 1);
+                }
+              }
+              __syncwarp();
+            }
           }
           // Quant(A) -> O operand: columns [sl XS, sl XS + XS) = heads 2 sl and 2 sl + 1, from TMEM
           float av[XS];
