@@ -132,12 +132,12 @@ __global__ void unpack_weights_kernel(const uint8_t *__restrict__ packed, int n_
   const int rr = static_cast<int>(item / (ch.kcols / 8)), cg = static_cast<int>(item % (ch.kcols / 8));
   const int n = ch.n0 + rr, k = ch.k0 + 8 * cg;
   // the ABI tensor and row of GEMM row n: QKV rows [0, D) W_q, [D, 2D) W_k, [2D, 3D) W_v; O W_o;
-  // FFN1 W_1 [F][D]; FFN2 W_2 [D][F]
+  // FFN1 W_1 [F][D] (output column n holds hidden unit ffn1_unit_of_column(D, n)); FFN2 W_2 [D][F]
   size_t toff;
   int row, din;
   if (ch.gemm == 0) toff = static_cast<size_t>(n / D) * D * D / 4, row = n % D, din = D;
   else if (ch.gemm == 1) toff = 3u * static_cast<size_t>(D) * D / 4, row = n, din = D;
-  else if (ch.gemm == 2) toff = static_cast<size_t>(D) * D, row = n, din = D;
+  else if (ch.gemm == 2) toff = static_cast<size_t>(D) * D, row = ffn1_unit_of_column(D, n), din = D;
   else toff = static_cast<size_t>(D) * D + static_cast<size_t>(F) * D / 4, row = n, din = F;
   const uint8_t *src = packed + per_layer_packed * l + toff + static_cast<size_t>(row) * (din / 4) + k / 4;
   const uint32_t bits = static_cast<uint32_t>(src[0]) | (static_cast<uint32_t>(src[1]) << 8);

@@ -88,6 +88,17 @@ struct WeightSchedule {
   }
   static constexpr uint32_t kLayerBytes = chunk(kCPL - 1).off + chunk_bytes(kCPL - 1);
 };
+// d = 128: the hidden unit whose FFN1 accumulator sits in TMEM column c (the weight row that the
+// weight stream places at FFN1 output column c).  Column slice s of a row owns hidden units
+// [128 s, 128 s + 128): units 128 s + [0, 64) in columns [64 s, 64 s + 64), done with FFN1's first
+// N-tile pair, and units 128 s + [64, 128) in columns [256 + 64 s, 256 + 64 s + 64).  The FFN2
+// operand codes of unit h, two to a 32-bit column, then go to column h / 2, which lies in the
+// slice's own first range and was read before it is written; FFN2's accumulators take [256, 384).
+// Other widths keep the identity.
+__host__ __device__ constexpr int ffn1_unit_of_column(int D, int c) {
+  return D == 128 ? 128 * ((c % 256) / 64) + 64 * (c / 256) + (c % 64) : c;
+}
+
 // the tcgen05.mma shape rules (M = 128: 16 <= N <= 256, N % 16 == 0) and the stage sizes
 template <int D>
 __host__ __device__ constexpr bool schedule_ok() {

@@ -755,7 +755,9 @@ int aecct_create(const aecct_model_desc *desc, aecct_handle **out) {
         uint8_t *base = reinterpret_cast<uint8_t *>(lw) + ch.off;
         for (int rr = 0; rr < ch.nrows; ++rr)
           for (int cc = 0; cc < ch.kcols; ++cc) {
-            const uint16_t bits = W[ch.gemm][(size_t)(ch.n0 + rr) * gm.K + ch.k0 + cc];
+            // FFN1's output column n0 + rr holds hidden unit ffn1_unit_of_column (d = 128)
+            const int row = ch.gemm == 2 ? ffn1_unit_of_column(D, ch.n0 + rr) : ch.n0 + rr;
+            const uint16_t bits = W[ch.gemm][(size_t)row * gm.K + ch.k0 + cc];
             std::memcpy(base + core_off(rr, cc, ch.kcols), &bits, 2);
           }
       }

@@ -783,11 +783,12 @@ struct Issuer {
 //   QKV  -> region U (free between the previous FFN2 and this block's K/V), one barrier bar_U;
 //   O    -> stages W0, W1;
 //   FFN1 -> region U again (free once every CTA of the cluster has finished attention);
-//   FFN2 -> W0, W1, W2, then the operand tile as A0, A1 (copied as soon as FFN1's MMAs, its last
-//           readers, are complete: during FFN1's epilogue), then W0, W1, W2 again once chunks
-//           16-18 are consumed.
-// A barrier armed u times per block (u odd for W0, W1, A0, A1) completes phase parity
-// (lpar if u is odd) ^ (index of the use within the block), with lpar the block's parity.
+//   FFN2 -> region U a third time, all eight chunks, copied during FFN1's epilogue as soon as
+//           FFN1's MMAs (their last readers) are complete: FFN2's operand (the codes of u) is in
+//           TMEM, columns [0, 256), and its accumulators in [256, 384), so no in-GEMM refill.
+// Stage W2 and the operand-tile halves A0, A1 hold no weights (W2 holds the Q/A slots of tasks
+// off their quadrant).  A barrier armed u times per block (u odd for U, W0, W1) completes phase
+// parity (lpar if u is odd) ^ (index of the use within the block), with lpar the block's parity.
 template <int ATT>
 struct Issuer<128, ATT> {
   static constexpr int D = 128;
@@ -796,6 +797,7 @@ struct Issuer<128, ATT> {
   static constexpr uint32_t kChunk = W::kStageBytes;
   static_assert(W::kCPL == 24 && W::kStages == 3 && kChunk == 16384, "d = 128 schedule");
   static_assert(L::kRegionU >= 8 * kChunk && L::kAopBytes == 2 * kChunk, "d = 128 regions");
+  static constexpr uint32_t kFfn2Acc = 256;  // TMEM columns of FFN2's accumulators (codes of u in [0, 256))
   uint32_t sb, tmem;
   Ctl ctl;
   uint32_t *n_armed;  // [6] phases armed per weight barrier (W0, W1, W2, U, A0, A1), for the drain
@@ -824,12 +826,10 @@ struct Issuer<128, ATT> {
     int id, uses, idx;
   };
   __host__ __device__ static constexpr Slot slot(int p) {
-    return p < 6    ? Slot{L::kOffU + kChunk * p, 3, 2, 0}
-           : p < 8  ? Slot{L::kOffW + kChunk * (p - 6), p - 6, 3, 0}
-           : p < 16 ? Slot{L::kOffU + kChunk * (p - 8), 3, 2, 1}
-           : p < 19 ? Slot{L::kOffW + kChunk * (p - 16), p - 16, p - 16 < 2 ? 3 : 2, p - 16 < 2 ? 1 : 0}
-           : p < 21 ? Slot{L::kOffAop + kChunk * (p - 19), 4 + (p - 19), 1, 0}
-                    : Slot{L::kOffW + kChunk * (p - 21), p - 21, p - 21 < 2 ? 3 : 2, p - 21 < 2 ? 2 : 1};
+    return p < 6    ? Slot{L::kOffU + kChunk * p, 3, 3, 0}
+           : p < 8  ? Slot{L::kOffW + kChunk * (p - 6), p - 6, 1, 0}
+           : p < 16 ? Slot{L::kOffU + kChunk * (p - 8), 3, 3, 1}
+                    : Slot{L::kOffU + kChunk * (p - 16), 3, 3, 2};
   }
   template <int P>
   __device__ __forceinline__ static uint32_t parity(uint32_t lpar) {
@@ -883,12 +883,11 @@ struct Issuer<128, ATT> {
     copy1<7>(src);
   }
   __device__ __forceinline__ void prologue(const uint8_t *w0) const { stage_qkv_o(w0); }
-  // FFN2's chunks 19 and 20 into the operand tile.  Called by warp 0 during FFN1's epilogue once
-  // FFN1's MMAs, the tile's last readers in this block, are known to be complete (warp 0 waited
-  // for them, or synchronised with warps that did).
-  __device__ __forceinline__ void stage_ffn2_aop(const uint8_t *w_cur) const {
-    copy1<19>(w_cur);
-    copy1<20>(w_cur);
+  // FFN2's eight chunks into region U.  Called by warp 0 during FFN1's epilogue once it has seen
+  // FFN1's MMAs, the region's last readers in this block, complete.
+  __device__ __forceinline__ void stage_ffn2(const uint8_t *w_cur) const {
+    arm(3, 8 * kChunk);
+    copies<16, 24>(w_cur);
   }
 
   // the MMAs of chunk P (its weights have landed)
@@ -931,6 +930,24 @@ struct Issuer<128, ATT> {
     }
   }
 
+  // FFN2 chunk P: A (the codes of u) from TMEM, K element k of a row in column k / 2; the
+  // accumulators in columns [kFfn2Acc, kFfn2Acc + 128)
+  template <int P>
+  __device__ __forceinline__ void mmas_tmem_a() const {
+    constexpr ChunkDesc c = W::chunk(P);
+    static_assert(c.gemm == 3 && c.n0 == 0 && c.nrows == 128, "an FFN2 chunk");
+    constexpr uint32_t b_sbo = (c.kcols / 8u) * 128u;
+    constexpr uint32_t idesc = make_idesc_bf16(128, c.nrows);
+    const uint32_t b_tile = sb + slot(P).off;
+    if (!live()) return;
+#pragma unroll 1
+    for (int ks = 0; ks < c.kcols / 16; ++ks) {
+      const uint32_t kabs = c.k0 + 16u * ks;
+      mma_bf16_tmem_a_warp(tmem + kFfn2Acc, tmem + kabs / 2u, make_sdesc(b_tile + ks * 256u, 128u, b_sbo), idesc,
+                           kabs > 0 ? 1u : 0u);
+    }
+  }
+
   template <int G>
   __device__ __forceinline__ void gemm(const uint8_t *w_cur, const uint8_t *w_next, bool has_next,
                                        const BlockCtx &bc) const {
@@ -938,7 +955,7 @@ struct Issuer<128, ATT> {
     wait(bar_op(), G & 1);
     tc_fence_after();
     if constexpr (G == 0) {
-      wait(bar(3), 0);  // QKV weights in region U
+      wait(bar(3), parity<0>(lp));  // QKV weights in region U
       mmas_pair<0, 0>();  // N tiles 0 and 1, K 0..63
       mmas_pair<0, 2>();  // N tiles 0 and 1, K 64..127
       mmas<0, 4>();       // N tile 2
@@ -955,60 +972,40 @@ struct Issuer<128, ATT> {
       // FFN1 weights into region U: this CTA has finished reading it (every warp published the O
       // operand) and no peer reads it (one-CTA cluster, staged attention); a cluster whose peers
       // read this CTA's K/V stages them at FFN1 instead, so that the O epilogue overlaps the
-      // peers' attention.  FFN2 chunk 18 into W2 (last read by the previous block's FFN2).
+      // peers' attention.
       if (bc.u_own) {
         arm(3, 8 * kChunk);
         copies<8, 16>(w_cur);
       }
-      copy1<18>(w_cur);
       wait(bar_acc(), 1);
       release_acc();
-      copy1<16>(w_cur);  // W0, W1 were O's
-      copy1<17>(w_cur);
     } else if constexpr (G == 2) {
       if (!bc.u_own) {  // every CTA of the cluster is done with this CTA's K/V
         wait(bc.kvf, bc.kvf_ph, true);
         arm(3, 8 * kChunk);
         copies<8, 16>(w_cur);
       }
-      wait(bar(3), 1);  // FFN1 weights in region U
+      wait(bar(3), parity<8>(lp));  // FFN1 weights in region U
       mmas_pair<2, 8>();
       mmas_pair<2, 10>();
-      // the epilogue of hidden units [0, 256) (column slices 0 and 1) starts while the MMAs of
-      // [256, 512) run; each warp waits on the barrier of its own half (no release by this warp)
+      // the epilogue of accumulator columns [0, 256), the first half of every column slice's hidden
+      // units, starts while the MMAs of [256, 512) run (every warp waits on both barriers itself;
+      // no release by this warp)
       commit(bar_acc_lo());
       mmas_pair<2, 12>();
       mmas_pair<2, 14>();
       commit(bar_acc());
     } else {
-      // chunks 19 and 20 were copied into the operand tile during FFN1's epilogue
-      wait(bar(0), parity<16>(lp));
-      mmas<3, 16>();
-      commit(bar_empty(0));
-      wait(bar(1), parity<17>(lp));
-      mmas<3, 17>();
-      commit(bar_empty(1));
-      wait(bar(2), parity<18>(lp));
-      mmas<3, 18>();
-      commit(bar_empty(2));
-      wait(bar(4), parity<19>(lp));
-      mmas<3, 19>();
-      wait(bar(5), parity<20>(lp));
-      mmas<3, 20>();
-      // refill W0-W2 with chunks 21-23 as soon as chunks 16-18 are consumed; the MMAs of 19 and
-      // 20 keep the tensor pipe busy meanwhile
-      wait(bar_empty(0), lp);
-      copy1<21>(w_cur);
-      wait(bar_empty(1), lp);
-      copy1<22>(w_cur);
-      wait(bar_empty(2), lp);
-      copy1<23>(w_cur);
-      wait(bar(0), parity<21>(lp));
-      mmas<3, 21>();
-      wait(bar(1), parity<22>(lp));
-      mmas<3, 22>();
-      wait(bar(2), parity<23>(lp));
-      mmas<3, 23>();
+      // all eight chunks in region U (copied during FFN1's epilogue); A from TMEM
+      wait(bar(3), parity<16>(lp));
+      mmas_tmem_a<16>();
+      mmas_tmem_a<17>();
+      mmas_tmem_a<18>();
+      mmas_tmem_a<19>();
+      mmas_tmem_a<20>();
+      mmas_tmem_a<21>();
+      mmas_tmem_a<22>();
+      mmas_tmem_a<23>();
       commit(bar_acc());
       wait(bar_acc(), 1);
       release_acc();
@@ -1880,32 +1877,38 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
         // ---------------- S7: FFN1 + ReLU (Sec. 4 item 4) or GELU, Quant(u) -> FFN2 operand
         {
           const float f1 = dq_factor(sw + 4);
-          if constexpr (D == 128) {
-            // AAP: column slices 0 and 1 (hidden units [0, 256)) wait for the first half of FFN1's
-            // MMAs, slices 2 and 3 for all of them (the block's third accumulator phase).  Their
-            // first pass only writes TMEM columns of the finished half; the codes go to region U,
-            // where the second half's weights are, after the row maximum, which needs every
-            // slice.  Full-precision linears write u to region U in their only pass: every slice
-            // waits for all of FFN1.
-            static_assert(16 * S + 48 + 64 == 160, "bar_fin + 64 is the issuer's bar_acc_lo");
-            if (LIN == 0 && sl < 2) wait_bar_warp(ctl, bar_fin + 64, (blk_base + static_cast<uint32_t>(l)) & 1u, false);
-            else wait_bar_warp(ctl, bar_acc, 0, false);
-            tc_fence_after();
-            // full-precision linears: warp 0 itself waited for all of FFN1, so the operand tile
-            // takes FFN2's chunks 19 and 20 now
-            if constexpr (LIN == 1)
-              if (warp == 0) issuer.stage_ffn2_aop(p.wstream + static_cast<size_t>(l) * p.layer_bytes);
-          } else {
-            wait_acc();
-          }
-          // ACT 0 = ReLU, 1 = GELU.  u = act(acc f1 + b1) in 32-column chunks of this thread's D
-          // hidden columns.  AAP: u is stored over its own accumulators in TMEM (this thread's
-          // lane and columns) between the row maximum and the codes, which leaves the registers
-          // to the rest of the kernel.  Full-precision linears: one pass, u rounded to bf16.
           constexpr int NCH = D / 32;
-          auto hidden = [&](int c0, float *u, bool capture) {
+          // accumulator column of this thread's chunk ch of 32 hidden units (units sl D + 32 ch +
+          // [0, 32)).  d = 128 (ffn1_unit_of_column): chunks 0 and 1 in [64 sl, 64 sl + 64), done
+          // with FFN1's first N-tile pair, chunks 2 and 3 in [256 + 64 sl, 256 + 64 sl + 64).
+          auto acc_col = [&](int ch) -> int {
+            if constexpr (D == 128) return ch < 2 ? 64 * sl + 32 * ch : 256 + 64 * sl + 32 * (ch - 2);
+            else return sl * D + 32 * ch;
+          };
+          // before chunk ch.  d = 128: chunks 0 and 1 wait for the first half of FFN1's MMAs, 2 and 3
+          // for all of them (the block's third accumulator phase); then warp 0 stages FFN2's
+          // weights into region U, whose last readers, FFN1's MMAs, are complete
+          auto wait_chunk = [&](int ch) {
+            if constexpr (D == 128) {
+              static_assert(16 * S + 48 + 64 == 160, "bar_fin + 64 is the issuer's bar_acc_lo");
+              if (ch == 0 || ch == 2) {
+                if (ch == 0) wait_bar_warp(ctl, bar_fin + 64, (blk_base + static_cast<uint32_t>(l)) & 1u, false);
+                else wait_bar_warp(ctl, bar_acc, 0, false);
+                tc_fence_after();
+                if (ch == 2 && warp == 0) issuer.stage_ffn2(p.wstream + static_cast<size_t>(l) * p.layer_bytes);
+              }
+            } else {
+              if (ch == 0) wait_acc();
+            }
+          };
+          // ACT 0 = ReLU, 1 = GELU.  u = act(acc f1 + b1) in 32-column chunks of this thread's D
+          // hidden units.  AAP: u is stored over its own accumulators in TMEM (this thread's lane
+          // and columns) between the row maximum and the codes, which leaves the registers to the
+          // rest of the kernel.  Full-precision linears: one pass, u rounded to bf16.
+          auto hidden = [&](int ch, float *u, bool capture) {
+            const int c0 = sl * D + 32 * ch;
             float ac[32], bb[32];
-            tmem_ld<32>(tl + c0, ac);
+            tmem_ld<32>(tl + acc_col(ch), ac);
             tmem_wait_ld();
             if (capture) capture_acc(l, 2, ac, c0, 32);
             ldg_vec<32>(lp + LP::b1(D) + c0, bb);
@@ -1913,50 +1916,69 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
 #pragma unroll
             for (int j = 0; j < 32; ++j) u[j] = ACT == 0 ? (u[j] > 0.0f ? u[j] : 0.0f) : gelu_as(u[j]);
           };
+          // d = 128: FFN2's operand goes to TMEM, the 32 values of chunk ch packed two to a column
+          // into the 16 columns [64 sl + 16 ch, 64 sl + 16 ch + 16) of this thread's lane (hidden
+          // unit h at column h / 2, the even one in the low half).  Those columns belong to chunks
+          // 0 and 1, and the chunk that held them was read before (chunk order 0, 1, 2, 3).
+          auto put_operand = [&](int ch, const uint32_t *w) {
+            tmem_st_u32<16>(tl + 64 * sl + 16 * ch, w);
+          };
           if constexpr (LIN == 1) {
             // peers have finished reading this CTA's K/V: the shared region may now take u
             if constexpr (!TASKS) cluster_wait(bar_kvf, kvf_ph);
 #pragma unroll
             for (int ch = 0; ch < NCH; ++ch) {
-              const int c0 = sl * D + 32 * ch;
+              wait_chunk(ch);
               float u[32];
-              hidden(c0, u, cap);
-              store_bf16<32>(uqt, r, c0, 4 * D, u);
+              hidden(ch, u, cap);
+              if constexpr (D == 128) {
+                uint32_t w[16];
+#pragma unroll
+                for (int i = 0; i < 16; ++i) w[i] = pack_bf16x2_rn(u[2 * i], u[2 * i + 1]);
+                put_operand(ch, w);
+              } else {
+                store_bf16<32>(uqt, r, sl * D + 32 * ch, 4 * D, u);
+              }
             }
+            if constexpr (D == 128) tmem_wait_st();
           } else {
             float umax = 0.0f;
 #pragma unroll
             for (int ch = 0; ch < NCH; ++ch) {
-              const int c0 = sl * D + 32 * ch;
+              wait_chunk(ch);
               float u[32];
-              hidden(c0, u, cap);
+              hidden(ch, u, cap);
 #pragma unroll
               for (int j = 0; j < 32; ++j) umax = fmaxf(umax, fabsf(u[j]));
-              tmem_st<32>(tl + c0, u);
+              tmem_st<32>(tl + acc_col(ch), u);
             }
             tmem_wait_st();
             float a = word_alpha(row_max(umax));
-            // FFN1's MMAs are complete (the row maximum synchronised warp 0 with the warps of
-            // column slices 2 and 3, which waited for all of them): the operand tile takes FFN2's
-            // chunks 19 and 20
-            if constexpr (D == 128)
-              if (warp == 0) issuer.stage_ffn2_aop(p.wstream + static_cast<size_t>(l) * p.layer_bytes);
             a = (a > p.alpha_floor) ? a : p.alpha_floor;
             alpha_in = a;
             const float rr = __fdiv_rn(127.0f, a);
             // peers have finished reading this CTA's K/V: the shared region may now take u codes
+            // (d <= 64; at d = 128 the staged attention's scratch is free for the next block's K/V)
             if constexpr (!TASKS) cluster_wait(bar_kvf, kvf_ph);
 #pragma unroll
             for (int ch = 0; ch < NCH; ++ch) {
               const int c0 = sl * D + 32 * ch;
               float u[32];
-              tmem_ld<32>(tl + c0, u);
+              tmem_ld<32>(tl + acc_col(ch), u);
               tmem_wait_ld();
               float qv[32];
               codes<32>(u, rr, qv);
-              store_codes<32>(uqt, r, c0, 4 * D, qv);
+              if constexpr (D == 128) {
+                uint32_t w[16];
+#pragma unroll
+                for (int i = 0; i < 16; ++i) w[i] = pack_bf16x2(qv[2 * i], qv[2 * i + 1]);
+                put_operand(ch, w);
+              } else {
+                store_codes<32>(uqt, r, c0, 4 * D, qv);
+              }
               if (cap) capture_q(l, 3, qv, c0, 32, alpha_in);
             }
+            if constexpr (D == 128) tmem_wait_st();
           }
         }
         signal_op(3, l, gi);
@@ -1967,7 +1989,8 @@ __global__ void __launch_bounds__(kThreads, 1) aecct_decoder_kernel(const __grid
           float ac[XS], bb[XS];
           if constexpr (kEarlyBias) ldg_vec<XS>(lp + LP::b2(D) + sl * XS, bb);
           wait_acc();
-          tmem_ld<XS>(tl + sl * XS, ac);
+          // d = 128: FFN2's accumulators sit after its operand in TMEM, columns [256, 384)
+          tmem_ld<XS>(tl + (D == 128 ? 256 : 0) + sl * XS, ac);
           tmem_wait_ld();
           if (cap) capture_acc(l, 3, ac, sl * XS, XS);
           if constexpr (!kEarlyBias) ldg_vec<XS>(lp + LP::b2(D) + sl * XS, bb);

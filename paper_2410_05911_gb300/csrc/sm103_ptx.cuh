@@ -264,6 +264,29 @@ __device__ __forceinline__ void mma_bf16_warp(uint32_t tmem_d, uint64_t adesc, u
       "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+// The same with the A operand in tensor memory: M = 128 rows in the 128 lanes, the K elements of a
+// row along its columns, two bf16 to a 32-bit column (the even K index in the low half); tmem_a is
+// the column of K elements [0, 16) of this MMA.  B comes from shared memory as above.
+__device__ __forceinline__ void mma_bf16_tmem_a_warp(uint32_t tmem_d, uint32_t tmem_a, uint64_t bdesc, uint32_t idesc,
+                                                     uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p, e;\n\t.reg .b32 r;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "elect.sync r|e, 0xffffffff;\n\t"
+      "@e tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "r"(tmem_a), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// store N (multiple of 8) consecutive 32-bit columns of this thread's lane
+template <int N>
+__device__ __forceinline__ void tmem_st_u32(uint32_t taddr, const uint32_t *v) {
+  static_assert(N % 8 == 0, "tmem_st width");
+#pragma unroll
+  for (int i = 0; i < N; i += 8)
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"r"(taddr + i),
+                 "r"(v[i]), "r"(v[i + 1]), "r"(v[i + 2]), "r"(v[i + 3]), "r"(v[i + 4]), "r"(v[i + 5]), "r"(v[i + 6]),
+                 "r"(v[i + 7])
+                 : "memory");
+}
 __device__ __forceinline__ void mma_commit_warp(uint32_t bar) {
   asm volatile(
       "{\n\t.reg .pred e;\n\t.reg .b32 r;\n\telect.sync r|e, 0xffffffff;\n\t"
